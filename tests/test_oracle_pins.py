@@ -1,0 +1,256 @@
+"""Pins for the fp64 CPU oracle (oracle/): it is checked against things other
+than itself -- a hand-worked example, hand-written scan orders, brute-force
+quadratic forms, closed forms and invariants of the recurrence in Sec. 3.1 --
+so that a dropped term, a wrong sign or index, a transposed operand or a wrong
+scan order fails at least one test.  Everything here runs on the CPU."""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2609_26590_gb300 import workloads as wl
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+ORDERS = (oracle.ROW_FWD, oracle.ROW_REV, oracle.COL_FWD, oracle.COL_REV)
+
+
+def _scan_by_hand(order, gh, gw):
+    """Scan order written out as nested loops over rows / columns (independent
+    of the oracle's index formula)."""
+    row_major = [y * gw + x for y in range(gh) for x in range(gw)]
+    col_major = [y * gw + x for x in range(gw) for y in range(gh)]
+    return {oracle.ROW_FWD: row_major, oracle.ROW_REV: row_major[::-1],
+            oracle.COL_FWD: col_major, oracle.COL_REV: col_major[::-1]}[order]
+
+
+def _rand(rng, B, T, H, Dk, Dv, gate_scale=1.0):
+    q = rng.standard_normal((B, T, H, Dk))
+    k = rng.standard_normal((B, T, H, Dk))
+    v = rng.standard_normal((B, T, H, Dv))
+    g = -gate_scale * rng.random((B, T, H, Dk))          # log-decay <= 0
+    return q, k, v, g
+
+
+def _brute_force(q, k, v, g, gh, gw, order):
+    """o_t = sum_{s<=t} (q_t . (prod_{r=s+1..t} gamma_r * k_s)) v_s along the scan,
+    and final = sum_s Diag(prod_{r>s} gamma_r) k_s^T v_s (quadratic form)."""
+    B, T, H, Dk = q.shape
+    Dv = v.shape[3]
+    seq = _scan_by_hand(order, gh, gw)
+    out = np.zeros((B, T, H, Dv))
+    fs = np.zeros((B, H, Dk, Dv))
+    gam = np.exp(g)
+    for b in range(B):
+        for h in range(H):
+            for pt, t in enumerate(seq):
+                acc = np.zeros(Dv)
+                for ps in range(pt + 1):
+                    s = seq[ps]
+                    decay = np.ones(Dk)
+                    for pr in range(ps + 1, pt + 1):
+                        decay = decay * gam[b, seq[pr], h]
+                    acc += np.dot(q[b, t, h], decay * k[b, s, h]) * v[b, s, h]
+                out[b, t, h] = acc
+            for ps in range(T):
+                s = seq[ps]
+                decay = np.ones(Dk)
+                for pr in range(ps + 1, T):
+                    decay = decay * gam[b, seq[pr], h]
+                fs[b, h] += np.outer(decay * k[b, s, h], v[b, s, h])
+    return out, fs
+
+
+def _rel(a, b):
+    return np.linalg.norm((a - b).ravel()) / max(np.linalg.norm(b.ravel()), 1e-300)
+
+
+# --------------------------------------------------------------------------------------
+# hand-worked fixtures
+# --------------------------------------------------------------------------------------
+
+def test_scan_orders_match_hand_lists():
+    with open(os.path.join(GOLDEN, "scan_orders_2x3.json")) as f:
+        gold = json.load(f)
+    for order, name in oracle.ORDER_NAMES.items():
+        got = oracle.scan_tokens(order, gold["grid_h"], gold["grid_w"])
+        assert got.tolist() == gold[name], name
+        assert _scan_by_hand(order, gold["grid_h"], gold["grid_w"]) == gold[name], name
+
+
+def _golden_case():
+    with open(os.path.join(GOLDEN, "hand_worked_1x3.json")) as f:
+        gold = json.load(f)
+    q = np.array(gold["q"], float).reshape(1, 3, 1, 2)
+    k = np.array(gold["k"], float).reshape(1, 3, 1, 2)
+    v = np.array(gold["v"], float).reshape(1, 3, 1, 3)
+    g = np.log(np.array(gold["gamma"], float)).reshape(1, 3, 1, 2)
+    return gold, q, k, v, g
+
+
+@pytest.mark.parametrize("name,order", [("row_fwd", oracle.ROW_FWD), ("row_rev", oracle.ROW_REV)])
+def test_hand_worked_recurrence(name, order):
+    gold, q, k, v, g = _golden_case()
+    out, fs = oracle.recurrence(q, k, v, g, 1, 3, order)
+    np.testing.assert_allclose(out.reshape(3, 3), gold[name]["out"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(fs.reshape(2, 3), gold[name]["final_state"], rtol=0, atol=1e-14)
+
+
+@pytest.mark.parametrize("chunk", [1, 2, 3, 64])
+@pytest.mark.parametrize("name,order", [("row_fwd", oracle.ROW_FWD), ("row_rev", oracle.ROW_REV)])
+def test_hand_worked_chunkwise(name, order, chunk):
+    gold, q, k, v, g = _golden_case()
+    out, fs = oracle.chunkwise(q, k, v, g, 1, 3, order, chunk=chunk)
+    np.testing.assert_allclose(out.reshape(3, 3), gold[name]["out"], rtol=0, atol=1e-14)
+    np.testing.assert_allclose(fs.reshape(2, 3), gold[name]["final_state"], rtol=0, atol=1e-14)
+
+
+# --------------------------------------------------------------------------------------
+# brute force on tiny inputs
+# --------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("order", ORDERS)
+@pytest.mark.parametrize("gh,gw", [(3, 5), (4, 2), (1, 7), (6, 1)])
+def test_brute_force_quadratic_form(order, gh, gw):
+    rng = np.random.default_rng(100 + order * 10 + gh)
+    q, k, v, g = _rand(rng, 2, gh * gw, 2, 3, 4, gate_scale=0.7)
+    ref_o, ref_s = _brute_force(q, k, v, g, gh, gw, order)
+    o, s = oracle.recurrence(q, k, v, g, gh, gw, order)
+    assert _rel(o, ref_o) < 1e-12
+    assert _rel(s, ref_s) < 1e-12
+    oc, sc = oracle.chunkwise(q, k, v, g, gh, gw, order, chunk=4)
+    assert _rel(oc, ref_o) < 1e-12
+    assert _rel(sc, ref_s) < 1e-12
+
+
+def test_pairs_subset_matches_full():
+    rng = np.random.default_rng(7)
+    q, k, v, g = _rand(rng, 3, 12, 4, 5, 3)
+    full_o, full_s = oracle.recurrence(q, k, v, g, 3, 4, oracle.COL_REV)
+    pairs = [(2, 1), (0, 3)]
+    o, s = oracle.recurrence(q, k, v, g, 3, 4, oracle.COL_REV, pairs=pairs)
+    for b, h in pairs:
+        np.testing.assert_array_equal(o[b, :, h], full_o[b, :, h])
+        np.testing.assert_array_equal(s[b, h], full_s[b, h])
+    assert np.isnan(o[1, :, 0]).all()
+
+
+# --------------------------------------------------------------------------------------
+# closed forms
+# --------------------------------------------------------------------------------------
+
+@pytest.mark.parametrize("order", ORDERS)
+def test_gate_one_is_causal_linear_attention(order):
+    gh, gw = 5, 7
+    rng = np.random.default_rng(11)
+    q, k, v, _ = _rand(rng, 2, gh * gw, 3, 6, 5)
+    g = np.zeros_like(q)
+    o, s = oracle.recurrence(q, k, v, g, gh, gw, order)
+    seq = np.array(_scan_by_hand(order, gh, gw))
+    for b in range(2):
+        for h in range(3):
+            Q, K, V = q[b, seq, h], k[b, seq, h], v[b, seq, h]
+            ref = np.tril(Q @ K.T) @ V                      # ((Q K^T) * causal mask) V
+            assert _rel(o[b, seq, h], ref) < 1e-12
+            assert _rel(s[b, h], K.T @ V) < 1e-12            # no decay: S_T = K^T V
+
+
+@pytest.mark.parametrize("order", ORDERS)
+def test_gate_zero_is_diagonal(order):
+    gh, gw = 4, 6
+    rng = np.random.default_rng(12)
+    q, k, v, _ = _rand(rng, 1, gh * gw, 2, 5, 3)
+    g = np.full_like(q, -np.inf)                            # gamma = 0: state resets every token
+    o, s = oracle.recurrence(q, k, v, g, gh, gw, order)
+    ref = np.einsum("bthi,bthi->bth", q, k)[..., None] * v
+    assert _rel(o, ref) < 1e-14
+    last = _scan_by_hand(order, gh, gw)[-1]
+    ref_s = np.einsum("bhi,bhj->bhij", k[:, last], v[:, last])
+    assert _rel(s, ref_s) < 1e-14
+    # the chunkwise model needs finite log-decays; -1e4 is gamma = 0 in floating point
+    oc, sc = oracle.chunkwise(q, k, v, np.full_like(q, -1e4), gh, gw, order, chunk=5)
+    assert _rel(oc, ref) < 1e-14
+    assert _rel(sc, ref_s) < 1e-14
+
+
+def test_single_token():
+    rng = np.random.default_rng(13)
+    q, k, v, g = _rand(rng, 2, 1, 3, 4, 6)
+    o, s = oracle.recurrence(q, k, v, g, 1, 1, oracle.COL_FWD)
+    ref = np.einsum("bthi,bthi->bth", q, k)[..., None] * v
+    assert _rel(o, ref) < 1e-14
+    assert _rel(s, np.einsum("bhi,bhj->bhij", k[:, 0], v[:, 0])) < 1e-14
+
+
+# --------------------------------------------------------------------------------------
+# invariants
+# --------------------------------------------------------------------------------------
+
+def test_reverse_scan_is_forward_scan_on_reversed_tokens():
+    gh, gw = 6, 5
+    rng = np.random.default_rng(14)
+    q, k, v, g = _rand(rng, 2, gh * gw, 2, 4, 3)
+    o_rev, s_rev = oracle.recurrence(q, k, v, g, gh, gw, oracle.ROW_REV)
+    flip = lambda a: a[:, ::-1]
+    o_f, s_f = oracle.recurrence(flip(q), flip(k), flip(v), flip(g), gh, gw, oracle.ROW_FWD)
+    assert _rel(o_rev, flip(o_f)) < 1e-14
+    assert _rel(s_rev, s_f) < 1e-14
+
+
+@pytest.mark.parametrize("col_order,row_order", [(oracle.COL_FWD, oracle.ROW_FWD),
+                                                 (oracle.COL_REV, oracle.ROW_REV)])
+def test_column_scan_is_row_scan_of_transposed_grid(col_order, row_order):
+    gh, gw = 4, 7
+    rng = np.random.default_rng(15)
+    q, k, v, g = _rand(rng, 1, gh * gw, 3, 4, 5)
+
+    def transpose(a):   # token (y, x) of a gh x gw grid -> token (x, y) of a gw x gh grid
+        B, T, H, D = a.shape
+        return a.reshape(B, gh, gw, H, D).transpose(0, 2, 1, 3, 4).reshape(B, T, H, D)
+
+    o_c, s_c = oracle.recurrence(q, k, v, g, gh, gw, col_order)
+    o_r, s_r = oracle.recurrence(transpose(q), transpose(k), transpose(v), transpose(g), gw, gh,
+                                 row_order)
+    B, T, H, Dv = o_r.shape
+    back = o_r.reshape(B, gw, gh, H, Dv).transpose(0, 2, 1, 3, 4).reshape(B, T, H, Dv)
+    assert _rel(o_c, back) < 1e-14
+    assert _rel(s_c, s_r) < 1e-14
+
+
+def test_linearity_in_q_and_v():
+    gh, gw = 3, 8
+    rng = np.random.default_rng(16)
+    q1, k, v1, g = _rand(rng, 1, gh * gw, 2, 4, 4)
+    q2 = rng.standard_normal(q1.shape)
+    v2 = rng.standard_normal(v1.shape)
+    a, c = 0.75, -1.5
+    f = lambda qq, vv: oracle.recurrence(qq, k, vv, g, gh, gw, oracle.COL_FWD)[0]
+    assert _rel(f(a * q1 + c * q2, v1), a * f(q1, v1) + c * f(q2, v1)) < 1e-13
+    assert _rel(f(q1, a * v1 + c * v2), a * f(q1, v1) + c * f(q1, v2)) < 1e-13
+
+
+@pytest.mark.parametrize("chunk", [1, 7, 16, 64, 150])
+@pytest.mark.parametrize("wid", [2, 3])
+def test_chunk_size_invariance(chunk, wid):
+    """Any chunk size gives the recurrence's result (Sec. 3.3: the chunked form
+    changes only the schedule), under the workloads' gate distributions --
+    including workload 3's strong decay (|A| ~ 90 per 64 tokens) and workload
+    2's non-decaying channels."""
+    w = wl.WORKLOADS[wid]
+    inp = wl.make_inputs(1, 3, 10, 15, 16, 8, "f32", seed=77, tau=w.tau, z_mean=w.z_mean,
+                         frac_nodecay=0.25 if w.frac_nodecay else 0.0)
+    q, k, v, g = (inp[n].astype(np.float64) for n in ("q", "k", "v", "g"))
+    for order in ORDERS:
+        ref_o, ref_s = oracle.recurrence(q, k, v, g, 10, 15, order)
+        o, s = oracle.chunkwise(q, k, v, g, 10, 15, order, chunk=chunk)
+        assert _rel(o, ref_o) < 1e-12, (order, chunk)
+        assert _rel(s, ref_s) < 1e-12, (order, chunk)
+
+
+def test_rejects_bad_arguments():
+    q = np.zeros((1, 4, 1, 2))
+    with pytest.raises(ValueError):
+        oracle.recurrence(q, q, q, q, 3, 2)
+    with pytest.raises(RuntimeError):
+        oracle.recurrence(q, q, q, q, 2, 2, order=7)
