@@ -1,0 +1,367 @@
+#!/usr/bin/env python3
+"""Throughput of the GB300 chunkwise GLA forward (GTR token mixer).
+
+One step = one forward pass over one batch of the workload: the whole hot path
+(scan-order gather, in-chunk cumulative log-decay, chunk summaries, state
+carry, intra-chunk gated scores, outputs and the final state) in the library's
+kernels.  Default workload: the batched 1600-token mixer (B=32, 40x40 grid,
+H=12, Dk=Dv=64, bf16, scan order alternating per step across the four
+orders).  Prints ONE JSON line on rank 0.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload ID] [--impl reference]
+
+Multi-GPU (torchrun, one rank per GPU): every rank runs its own batch of the
+same workload (weak scaling, no collective on the data path); value = tokens
+of all ranks / max-over-ranks time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_26590_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "GLA-forward tokens/s (GB300, device-timed) and % of roofline at 1600 tokens"
+DEFAULT_WORKLOAD = 2
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--schedule", default="auto", choices=["auto", "simt", "tc"])
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-clocks", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+def workload_config(w: wl.Workload, world: int, extra=None):
+    cfg = {"workload": w.name, "B": w.B, "H": w.H, "grid": [w.grid_h, w.grid_w], "T": w.T,
+           "Dk": w.Dk, "Dv": w.Dv, "tokens_per_step_per_gpu": w.B * w.T,
+           "scan_orders": "alternating " + "/".join(wl.ORDER_NAMES[o] for o in w.orders),
+           "final_state": w.final_state,
+           "l2": "inputs larger than L2 (%.0f MB per step > 129 MB)" % (w.algorithmic_bytes() / 1e6),
+           "parallelism": f"replicas x{world} (independent batches, no collective)"}
+    if extra:
+        cfg.update(extra)
+    return cfg
+
+
+# --------------------------------------------------------------------------------------
+# clocks during the timed region
+# --------------------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, enabled: bool = True):
+        self.gpu_index = gpu_index
+        self.enabled = enabled
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        if not self.enabled:
+            return self
+        fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu_index}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        return False
+
+    def summary(self):
+        if not self.enabled or self.proc is None or not self.path:
+            return None
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append(parts)
+                except ValueError:
+                    continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in rows:
+            for n, val in zip(names, r[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": sorted(reasons),
+                "samples": len(rows)}
+
+
+# --------------------------------------------------------------------------------------
+# CPU baseline: the fp64 oracle as it stands, on the host cores
+# --------------------------------------------------------------------------------------
+
+def time_oracle(w: wl.Workload, inp64, order: int, budget_s: float = 10.0, max_pairs=None):
+    """Time the oracle over (b, h) pairs of the workload until ~budget_s of wall
+    time is spent (at least one full pass over the chosen pairs)."""
+    import oracle
+    pairs_all = [(b, h) for b in range(w.B) for h in range(w.H)]
+    pairs = pairs_all if max_pairs is None else pairs_all[:max_pairs]
+    n_done, t0 = 0, time.perf_counter()
+    while True:
+        oracle.recurrence(inp64["q"], inp64["k"], inp64["v"], inp64["g"], w.grid_h, w.grid_w,
+                          order, pairs=pairs)
+        n_done += len(pairs)
+        el = time.perf_counter() - t0
+        if el >= budget_s or (max_pairs is None and el > 0.5 * budget_s):
+            break
+    tokens = n_done / w.H * w.T      # (b, h) pairs -> image tokens (all heads of a batch item)
+    return tokens / el, el, n_done, oracle.max_threads()
+
+
+def run_reference(args, w: wl.Workload, rank: int, world: int):
+    """--impl reference: the oracle timed on the host cores, per step a bounded
+    sample of the same workload (a prefix of its (b, h) pairs)."""
+    if rank != 0:
+        return
+    import oracle
+    inp = wl.workload_inputs(w)
+    inp64 = {n: wl.storage_to_f64(inp[n], w.dtype) for n in ("q", "k", "v", "g")}
+    del inp
+    n_pairs = min(w.B * w.H, max(1, oracle.max_threads()))
+    for i in range(args.warmup):
+        oracle.recurrence(inp64["q"], inp64["k"], inp64["v"], inp64["g"], w.grid_h, w.grid_w,
+                          w.orders[i % len(w.orders)],
+                          pairs=[(b, h) for b in range(w.B) for h in range(w.H)][:n_pairs])
+    times = []
+    for i in range(args.steps):
+        order = w.orders[i % len(w.orders)]
+        pairs = [(b, h) for b in range(w.B) for h in range(w.H)][:n_pairs]
+        t0 = time.perf_counter()
+        oracle.recurrence(inp64["q"], inp64["k"], inp64["v"], inp64["g"], w.grid_h, w.grid_w,
+                          order, pairs=pairs)
+        times.append(time.perf_counter() - t0)
+    per_step = sum(times) / len(times)
+    tokens = n_pairs / w.H * w.T
+    value = tokens / per_step
+    sample = f"{n_pairs} of {w.B * w.H} (b,h) sequences of {w.T} tokens per step"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": per_step * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded, workload recipe)",
+            "config": workload_config(w, 1, {"reference": "fp64 CPU oracle (oracle/), as it stands"}),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.max_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------------------
+# GPU arm
+# --------------------------------------------------------------------------------------
+
+def main():
+    args = parse()
+    rank, world, local = dist_env()
+    w = wl.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, w, rank, world)
+        return
+
+    import torch
+    from paper_2609_26590_gb300 import gla
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+
+    gla.load()
+    dt = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}[w.dtype]
+
+    # inputs: rank r draws batch r of the workload (same distributions, own seed)
+    inp = wl.workload_inputs(w, seed=1234 + w.wid + 1000 * rank)
+
+    def to_dev(a):
+        if w.dtype == "bf16":
+            return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(dev)
+        return torch.from_numpy(a).to(dev)
+
+    t = {n: to_dev(inp[n]) for n in ("q", "k", "v", "g")}
+    out = torch.empty_like(t["v"])
+    fs = torch.empty((w.B, w.H, w.Dk, w.Dv), dtype=torch.float32, device=dev) if w.final_state else None
+    stream = torch.cuda.current_stream(dev)
+    orders = w.orders
+    schedule = args.schedule
+    tc = gla.tc_supported(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, orders[0], dt)
+    kernel_name = "tensor-core chunkwise (tcgen05/TMEM/TMA)" if (tc and schedule != "simt") else "simt recurrence"
+
+    def step(i):
+        gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, orders[i % len(orders)],
+                    out=out, final_state=fs if fs is not None else None, schedule=schedule)
+
+    for i in range(max(3, args.warmup)):
+        step(i)
+    torch.cuda.synchronize()
+    if gla.sync_status() != 0:
+        raise RuntimeError("device status word set during warm-up")
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local, enabled=not args.no_clocks) as clk:
+        t_begin = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_begin.record(stream)
+        for i in range(args.steps):
+            starts[i].record(stream)
+            step(i)
+            ends[i].record(stream)
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    total_ms = t_begin.elapsed_time(t_end)
+    per_launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    if gla.sync_status() != 0:
+        raise RuntimeError("device status word set during the timed region")
+    if pg:
+        tt = torch.tensor([total_ms], device=dev)
+        pg.all_reduce(tt, op=pg.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_per_step = total_ms / args.steps
+    tokens_per_step = w.B * w.T * world
+    value = tokens_per_step / (ms_per_step * 1e-3)
+
+    # roofline of the (single) kernel of a step
+    hbm_peak, peak_src = load_peaks()
+    alg_bytes = w.algorithmic_bytes()
+    kernel_ms = sum(per_launch_ms) / len(per_launch_ms)
+    achieved = alg_bytes / (kernel_ms * 1e-3) / 1e9
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        with open(tpath) as f:
+            tj = json.load(f)
+        key = f"{w.name}:{'tc' if (tc and schedule != 'simt') else 'simt'}"
+        traffic = tj.get(key)
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                "frac": achieved / hbm_peak, "traffic": traffic,
+                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback",
+                "kernel": kernel_name, "kernel_ms": kernel_ms,
+                "algorithmic_bytes_per_launch": alg_bytes}
+
+    # end to end through the host-memory entry point (pinned host buffers)
+    e2e = None
+    if args.e2e_steps > 0:
+        host = {n: (torch.from_numpy(inp[n].view(np.int16)).view(torch.bfloat16) if w.dtype == "bf16"
+                    else torch.from_numpy(inp[n])).pin_memory() for n in ("q", "k", "v", "g")}
+        hout = torch.empty(host["v"].shape, dtype=host["v"].dtype).pin_memory()
+        hfs = torch.empty((w.B, w.H, w.Dk, w.Dv), dtype=torch.float32).pin_memory() if w.final_state else None
+        nbytes = gla.host_buffer_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt, w.final_state)
+        dbuf = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        for i in range(2):
+            gla.forward_host(host["q"], host["k"], host["v"], host["g"], w.grid_h, w.grid_w,
+                             orders[i % len(orders)], hout, hfs, dbuf)
+        torch.cuda.synchronize()
+        if pg:
+            pg.barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for i in range(args.e2e_steps):
+            gla.forward_host(host["q"], host["k"], host["v"], host["g"], w.grid_h, w.grid_w,
+                             orders[i % len(orders)], hout, hfs, dbuf)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = e0.elapsed_time(e1)
+        if pg:
+            tt = torch.tensor([e_ms], device=dev)
+            pg.all_reduce(tt, op=pg.ReduceOp.MAX)
+            e_ms = float(tt.item())
+        es = w.B * w.T * world / (e_ms / args.e2e_steps * 1e-3)
+        h2d = sum(host[n].numel() * host[n].element_size() for n in ("q", "k", "v", "g"))
+        d2h = hout.numel() * hout.element_size() + (hfs.numel() * 4 if hfs is not None else 0)
+        e2e = {"value": es, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": e_ms / args.e2e_steps,
+               "api": "gtr_gla_fwd_host (pinned host buffers)"}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        inp64 = {n: wl.storage_to_f64(inp[n], w.dtype) for n in ("q", "k", "v", "g")}
+        val, el, n_pairs, cores = time_oracle(w, inp64, orders[0], budget_s=10.0)
+        cpu = {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+               "sample": f"{n_pairs} (b,h) sequences x {w.T} tokens ({el:.1f} s wall), "
+                         f"order {wl.ORDER_NAMES[orders[0]]}"}
+
+    if rank == 0:
+        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+                "dtype": w.dtype, "data": "synthetic (seeded, workload recipe in workloads.py)",
+                "config": workload_config(w, world, {"schedule": schedule}),
+                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": args.steps, "clocks": clk.summary(),
+                "token_heads_per_s": value * w.H}
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,149 @@
+/*
+ * gtr_gla.h -- C ABI of the GB300 (sm_103a) chunkwise gated-linear-attention
+ * forward: the token mixer of GTR ("GTR: Gated Token Recurrence for Efficient
+ * Dense Prediction").
+ *
+ * Operation (Sec. 3.1, "Key-only gated recurrence"; value-side decay fixed to
+ * one, Sec. 3.1 and App. C.3), per batch b and head h, along one scan order:
+ *
+ *     S_0 = 0,   S_t = Diag(exp(g_t)) S_{t-1} + k_t^T v_t,   o_t = q_t S_t
+ *
+ * with q_t, k_t, g_t in R^{1 x Dk}, v_t, o_t in R^{1 x Dv}, S_t in R^{Dk x Dv}.
+ * g_t = log(gamma_t) is the learned per-key-channel log-decay the operator takes
+ * as input (Sec. 3.3: "the same queries, keys, values, and learned
+ * log-decays").  The paper's output factor d_k^{-1/2} is not applied: fold it
+ * into k (or q) before the call.
+ *
+ * Scan orders (Sec. 3.1, "Directional scanning"): the T = grid_h * grid_w
+ * tokens of a patch grid are stored in spatial row-major order
+ * (t = y * grid_w + x).  The recurrence visits them in one of four raster
+ * orders, one sequence per image with the state carried across rows/columns;
+ * each output is written back at its token's spatial position (the block
+ * "restores the original spatial order"):
+ *     ROW_FWD  left-to-right:  position s visits t = s
+ *     ROW_REV  right-to-left:  t = T-1-s          (exact reversal of ROW_FWD)
+ *     COL_FWD  top-to-bottom:  t = (s mod grid_h) * grid_w + s div grid_h
+ *     COL_REV  bottom-to-top:  COL_FWD applied to T-1-s (exact reversal)
+ *
+ * Schedule (Sec. 3.3 and App. C.3): chunks of C = 64 scan positions; the
+ * in-chunk cumulative log-decay, the chunk summaries U_c, the boundary-state
+ * carry S_[c+1] = Diag(d_c) S_[c] + U_c and the intra-chunk gated scores are
+ * computed on the GPU; the scan permutation is applied inside the loads and
+ * the output store.  The result equals the recurrence up to floating-point
+ * rounding.
+ *
+ * Common argument rules (every entry point below):
+ *   - q, k, log_gate : [B, T, H, Dk]  element type `dtype`, contiguous.
+ *     v, out         : [B, T, H, Dv]  element type `dtype`, contiguous.
+ *     final_state    : [B, H, Dk, Dv] float32, contiguous, or NULL (not written).
+ *     All tensor pointers are device pointers unless stated otherwise, owned by
+ *     the caller, 16-byte aligned, and `out` / `final_state` must not overlap
+ *     the inputs.
+ *   - log_gate must be <= 0 or -inf; values below -1e4 act as -1e4, which is
+ *     gamma = 0 exactly in float32.  NaN inputs give NaN outputs.
+ *   - B, H, grid_h, grid_w >= 1 (B*H*T == 0 is allowed only as B == 0 or H == 0,
+ *     which launches nothing); 1 <= Dk, Dv <= 128.
+ *   - The call is asynchronous on `stream`: it validates, enqueues kernels and
+ *     returns.  Validation failures return before anything is enqueued.
+ *     Launch failures return GTR_ERR_CUDA.  Conditions the device detects
+ *     (a bounded wait that gave up) are recorded in a per-device status word
+ *     and reported by gtr_gla_sync_status().
+ *   - No call allocates device memory, synchronises, or reads device data on
+ *     the host, so gtr_gla_fwd can be captured in a CUDA graph.
+ */
+#ifndef GTR_GLA_H
+#define GTR_GLA_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    GTR_OK = 0,
+    GTR_ERR_INVALID_ARG = 1,  /* null / misaligned pointer, bad size or enum value   */
+    GTR_ERR_UNSUPPORTED = 2,  /* well-formed, but the requested schedule cannot run  */
+    GTR_ERR_WORKSPACE = 3,    /* workspace missing or smaller than required          */
+    GTR_ERR_CUDA = 4,         /* a CUDA call failed; see gtr_last_cuda_error()       */
+    GTR_ERR_TIMEOUT = 5       /* a bounded device-side wait gave up                  */
+} gtr_status_t;
+
+typedef enum { GTR_F32 = 0, GTR_F16 = 1, GTR_BF16 = 2 } gtr_dtype_t;
+
+typedef enum {
+    GTR_SCAN_ROW_FWD = 0,     /* left-to-right  */
+    GTR_SCAN_ROW_REV = 1,     /* right-to-left  */
+    GTR_SCAN_COL_FWD = 2,     /* top-to-bottom  */
+    GTR_SCAN_COL_REV = 3      /* bottom-to-top  */
+} gtr_scan_t;
+
+/* Kernel schedule.  AUTO picks the fastest schedule that supports the
+ * arguments.  SIMT is the plain fp32 CUDA-core recurrence (any dtype, any
+ * shape within the common rules; the float32 path).  TC is the tensor-core
+ * chunkwise schedule (tcgen05 MMAs, TMEM accumulators, TMA loads/stores):
+ * fp16/bf16 only, with the shape rules of gtr_gla_tc_supported(). */
+typedef enum { GTR_SCHED_AUTO = 0, GTR_SCHED_SIMT = 1, GTR_SCHED_TC = 2 } gtr_schedule_t;
+
+/* Forward of the token mixer with the AUTO schedule (argument rules above).
+ * Returns GTR_OK once the work is enqueued on `stream`. */
+gtr_status_t gtr_gla_fwd(const void *q, const void *k, const void *v, const void *log_gate,
+                         int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                         gtr_scan_t scan_order, gtr_dtype_t dtype,
+                         void *out, float *final_state, cudaStream_t stream);
+
+/* Same as gtr_gla_fwd with an explicit schedule.  Requesting a schedule that
+ * cannot run these arguments returns GTR_ERR_UNSUPPORTED (never a silent
+ * fallback). */
+gtr_status_t gtr_gla_fwd_sched(const void *q, const void *k, const void *v,
+                               const void *log_gate, int B, int H, int grid_h, int grid_w,
+                               int Dk, int Dv, gtr_scan_t scan_order, gtr_dtype_t dtype,
+                               void *out, float *final_state, gtr_schedule_t schedule,
+                               cudaStream_t stream);
+
+/* 1 when the tensor-core schedule supports these arguments, else 0. */
+int gtr_gla_tc_supported(int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                         gtr_scan_t scan_order, gtr_dtype_t dtype);
+
+/* Bytes of device memory gtr_gla_fwd_host needs as `dev_buffer` (inputs,
+ * output and final state staged on the device, each 256-byte aligned). */
+size_t gtr_gla_host_buffer_bytes(int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                                 gtr_dtype_t dtype, int with_final_state);
+
+/* End-to-end forward from HOST memory: copies q, k, v, log_gate (host
+ * pointers, same layouts as above; pinned memory makes the copies
+ * asynchronous) into `dev_buffer` (caller-owned device memory of at least
+ * gtr_gla_host_buffer_bytes() bytes), runs gtr_gla_fwd on `stream`, and
+ * copies `out` (and `final_state` when non-NULL) back to the host pointers.
+ * Everything is enqueued on `stream`; synchronise it before reading the
+ * results.  Errors as gtr_gla_fwd, plus GTR_ERR_WORKSPACE when dev_buffer is
+ * NULL or too small. */
+gtr_status_t gtr_gla_fwd_host(const void *q_host, const void *k_host, const void *v_host,
+                              const void *log_gate_host, int B, int H, int grid_h, int grid_w,
+                              int Dk, int Dv, gtr_scan_t scan_order, gtr_dtype_t dtype,
+                              void *out_host, float *final_state_host, void *dev_buffer,
+                              size_t dev_buffer_bytes, cudaStream_t stream);
+
+/* Synchronises `stream`, then returns and clears the device status word of the
+ * current device (GTR_OK when no device-side condition was recorded,
+ * GTR_ERR_TIMEOUT when a bounded wait gave up), or GTR_ERR_CUDA when the
+ * synchronisation itself failed. */
+gtr_status_t gtr_gla_sync_status(cudaStream_t stream);
+
+/* Static, NUL-terminated description of a status code. */
+const char *gtr_status_string(gtr_status_t status);
+
+/* The cudaError_t value behind the last GTR_ERR_CUDA returned on this host
+ * thread (0 when none). */
+int gtr_last_cuda_error(void);
+
+/* Library version, MAJOR * 10000 + MINOR * 100 + PATCH. */
+int gtr_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GTR_GLA_H */

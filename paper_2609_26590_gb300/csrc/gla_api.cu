@@ -1,0 +1,192 @@
+// gla_api.cu -- the C ABI of include/gtr_gla.h: argument validation, schedule
+// dispatch, the host-memory entry point and status reporting.  No kernel code.
+#include <cstdint>
+#include <cstring>
+
+#include "gla_internal.h"
+#include "gtr_gla.h"
+
+namespace {
+
+thread_local int t_last_cuda_error = 0;
+
+constexpr size_t kAlign = 16;
+constexpr int kMaxHeadDim = 128;
+
+bool aligned(const void *p) { return (reinterpret_cast<uintptr_t>(p) % kAlign) == 0; }
+
+size_t elem_size(int dtype) { return dtype == GTR_F32 ? 4 : 2; }
+
+bool overlaps(const void *a, size_t na, const void *b, size_t nb) {
+    if (a == nullptr || b == nullptr || na == 0 || nb == 0) return false;
+    auto pa = reinterpret_cast<uintptr_t>(a), pb = reinterpret_cast<uintptr_t>(b);
+    return pa < pb + nb && pb < pa + na;
+}
+
+gtr_status_t cuda_fail(cudaError_t e) {
+    t_last_cuda_error = static_cast<int>(e);
+    return GTR_ERR_CUDA;
+}
+
+// Shape / enum checks shared by every entry point.
+gtr_status_t check_shape(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int order,
+                         int dtype) {
+    if (B < 0 || H < 0 || grid_h < 1 || grid_w < 1) return GTR_ERR_INVALID_ARG;
+    if (Dk < 1 || Dv < 1 || Dk > kMaxHeadDim || Dv > kMaxHeadDim) return GTR_ERR_INVALID_ARG;
+    if (order < GTR_SCAN_ROW_FWD || order > GTR_SCAN_COL_REV) return GTR_ERR_INVALID_ARG;
+    if (dtype < GTR_F32 || dtype > GTR_BF16) return GTR_ERR_INVALID_ARG;
+    const long long T = (long long)grid_h * grid_w;
+    if (T > 0x7fffffffLL) return GTR_ERR_INVALID_ARG;
+    if ((long long)B * H > 0x7fffffffLL) return GTR_ERR_INVALID_ARG;
+    const long long D = Dk > Dv ? Dk : Dv;
+    // every element offset must fit in int64 with room to spare
+    if ((long long)B * T > (1LL << 40) / ((long long)H * D + 1)) return GTR_ERR_INVALID_ARG;
+    return GTR_OK;
+}
+
+gtr_status_t make_problem(const void *q, const void *k, const void *v, const void *g, int B,
+                          int H, int grid_h, int grid_w, int Dk, int Dv, int order, int dtype,
+                          void *out, float *final_state, gtr::Problem *p) {
+    gtr_status_t st = check_shape(B, H, grid_h, grid_w, Dk, Dv, order, dtype);
+    if (st != GTR_OK) return st;
+    if (!q || !k || !v || !g || !out) return GTR_ERR_INVALID_ARG;
+    if (!aligned(q) || !aligned(k) || !aligned(v) || !aligned(g) || !aligned(out) ||
+        !aligned(final_state))
+        return GTR_ERR_INVALID_ARG;
+    const long long T = (long long)grid_h * grid_w;
+    const size_t es = elem_size(dtype);
+    const size_t nk = (size_t)B * T * H * Dk * es, nv = (size_t)B * T * H * Dv * es;
+    const size_t nfs = (size_t)B * H * Dk * Dv * sizeof(float);
+    const void *ins[4] = {q, k, v, g};
+    const size_t ins_n[4] = {nk, nk, nv, nk};
+    for (int i = 0; i < 4; ++i) {
+        if (overlaps(out, nv, ins[i], ins_n[i])) return GTR_ERR_INVALID_ARG;
+        if (overlaps(final_state, nfs, ins[i], ins_n[i])) return GTR_ERR_INVALID_ARG;
+    }
+    if (overlaps(out, nv, final_state, nfs)) return GTR_ERR_INVALID_ARG;
+    *p = gtr::Problem{q, k, v, g, out, final_state, B, H, grid_h, grid_w, Dk, Dv, order, dtype, T};
+    return GTR_OK;
+}
+
+size_t round_up(size_t n, size_t a) { return (n + a - 1) / a * a; }
+
+}  // namespace
+
+extern "C" {
+
+gtr_status_t gtr_gla_fwd_sched(const void *q, const void *k, const void *v, const void *log_gate,
+                               int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                               gtr_scan_t scan_order, gtr_dtype_t dtype, void *out,
+                               float *final_state, gtr_schedule_t schedule, cudaStream_t stream) {
+    gtr::Problem p;
+    gtr_status_t st = make_problem(q, k, v, log_gate, B, H, grid_h, grid_w, Dk, Dv, scan_order,
+                                   dtype, out, final_state, &p);
+    if (st != GTR_OK) return st;
+    if (schedule < GTR_SCHED_AUTO || schedule > GTR_SCHED_TC) return GTR_ERR_INVALID_ARG;
+    if (B == 0 || H == 0) return GTR_OK;
+    cudaError_t e;
+    switch (schedule) {
+    case GTR_SCHED_SIMT:
+        e = gtr::launch_simt(p, stream);
+        break;
+    case GTR_SCHED_TC:
+        if (!gtr::tc_supported(p)) return GTR_ERR_UNSUPPORTED;
+        e = gtr::launch_tc(p, stream);
+        break;
+    default:
+        e = gtr::tc_supported(p) ? gtr::launch_tc(p, stream) : gtr::launch_simt(p, stream);
+        break;
+    }
+    if (e != cudaSuccess) return cuda_fail(e);
+    return GTR_OK;
+}
+
+gtr_status_t gtr_gla_fwd(const void *q, const void *k, const void *v, const void *log_gate, int B,
+                         int H, int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
+                         gtr_dtype_t dtype, void *out, float *final_state, cudaStream_t stream) {
+    return gtr_gla_fwd_sched(q, k, v, log_gate, B, H, grid_h, grid_w, Dk, Dv, scan_order, dtype,
+                             out, final_state, GTR_SCHED_AUTO, stream);
+}
+
+int gtr_gla_tc_supported(int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                         gtr_scan_t scan_order, gtr_dtype_t dtype) {
+    if (check_shape(B, H, grid_h, grid_w, Dk, Dv, scan_order, dtype) != GTR_OK) return 0;
+    gtr::Problem p{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, B, H, grid_h, grid_w,
+                   Dk, Dv, scan_order, dtype, (long long)grid_h * grid_w};
+    return gtr::tc_supported(p) ? 1 : 0;
+}
+
+size_t gtr_gla_host_buffer_bytes(int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                                 gtr_dtype_t dtype, int with_final_state) {
+    if (check_shape(B, H, grid_h, grid_w, Dk, Dv, 0, dtype) != GTR_OK) return 0;
+    const size_t T = (size_t)grid_h * grid_w, es = elem_size(dtype);
+    const size_t nk = round_up((size_t)B * T * H * Dk * es, 256);
+    const size_t nv = round_up((size_t)B * T * H * Dv * es, 256);
+    const size_t nfs = with_final_state ? round_up((size_t)B * H * Dk * Dv * 4, 256) : 0;
+    return 3 * nk + 2 * nv + nfs;
+}
+
+gtr_status_t gtr_gla_fwd_host(const void *q_host, const void *k_host, const void *v_host,
+                              const void *log_gate_host, int B, int H, int grid_h, int grid_w,
+                              int Dk, int Dv, gtr_scan_t scan_order, gtr_dtype_t dtype,
+                              void *out_host, float *final_state_host, void *dev_buffer,
+                              size_t dev_buffer_bytes, cudaStream_t stream) {
+    gtr_status_t st = check_shape(B, H, grid_h, grid_w, Dk, Dv, scan_order, dtype);
+    if (st != GTR_OK) return st;
+    if (!q_host || !k_host || !v_host || !log_gate_host || !out_host) return GTR_ERR_INVALID_ARG;
+    const int with_fs = final_state_host != nullptr;
+    const size_t need = gtr_gla_host_buffer_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype, with_fs);
+    if (dev_buffer == nullptr || dev_buffer_bytes < need) return GTR_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(dev_buffer) % 256) != 0) return GTR_ERR_INVALID_ARG;
+    if (B == 0 || H == 0) return GTR_OK;
+    const size_t T = (size_t)grid_h * grid_w, es = elem_size(dtype);
+    const size_t bk = (size_t)B * T * H * Dk * es, bv = (size_t)B * T * H * Dv * es;
+    const size_t bfs = (size_t)B * H * Dk * Dv * 4;
+    char *base = static_cast<char *>(dev_buffer);
+    char *dq = base, *dk = dq + round_up(bk, 256), *dg = dk + round_up(bk, 256);
+    char *dv = dg + round_up(bk, 256), *dout = dv + round_up(bv, 256);
+    float *dfs = with_fs ? reinterpret_cast<float *>(dout + round_up(bv, 256)) : nullptr;
+    cudaError_t e;
+    if ((e = cudaMemcpyAsync(dq, q_host, bk, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dk, k_host, bk, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dg, log_gate_host, bk, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(dv, v_host, bv, cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+        return cuda_fail(e);
+    st = gtr_gla_fwd(dq, dk, dv, dg, B, H, grid_h, grid_w, Dk, Dv, scan_order, dtype, dout, dfs,
+                     stream);
+    if (st != GTR_OK) return st;
+    if ((e = cudaMemcpyAsync(out_host, dout, bv, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+        return cuda_fail(e);
+    if (with_fs &&
+        (e = cudaMemcpyAsync(final_state_host, dfs, bfs, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+        return cuda_fail(e);
+    return GTR_OK;
+}
+
+gtr_status_t gtr_gla_sync_status(cudaStream_t stream) {
+    cudaError_t e = cudaStreamSynchronize(stream);
+    if (e != cudaSuccess) return cuda_fail(e);
+    unsigned int word = 0;
+    e = gtr::read_and_clear_device_status(&word);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (word & gtr::kStatusTimeout) return GTR_ERR_TIMEOUT;
+    return GTR_OK;
+}
+
+const char *gtr_status_string(gtr_status_t status) {
+    switch (status) {
+    case GTR_OK: return "ok";
+    case GTR_ERR_INVALID_ARG: return "invalid argument";
+    case GTR_ERR_UNSUPPORTED: return "unsupported by the requested schedule";
+    case GTR_ERR_WORKSPACE: return "workspace missing or too small";
+    case GTR_ERR_CUDA: return "CUDA error";
+    case GTR_ERR_TIMEOUT: return "device-side wait timed out";
+    default: return "unknown status";
+    }
+}
+
+int gtr_last_cuda_error(void) { return t_last_cuda_error; }
+
+int gtr_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,33 @@
+// gla_internal.h -- declarations shared by the translation units of the GB300
+// GLA library (host side only; kernels live in their own .cu files).
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace gtr {
+
+// One forward call, as validated by the C ABI (include/gtr_gla.h).
+struct Problem {
+    const void *q, *k, *v, *g;  // [B,T,H,Dk] x3, [B,T,H,Dv]
+    void *out;                  // [B,T,H,Dv]
+    float *final_state;         // [B,H,Dk,Dv] or nullptr
+    int B, H, grid_h, grid_w, Dk, Dv;
+    int order;                  // gtr_scan_t
+    int dtype;                  // gtr_dtype_t
+    long long T;                // grid_h * grid_w
+};
+
+// Plain fp32 CUDA-core recurrence (gla_simt.cu).  Any dtype, Dk, Dv <= 128.
+cudaError_t launch_simt(const Problem &p, cudaStream_t stream);
+
+// Tensor-core chunkwise schedule (gla_tc.cu).
+bool tc_supported(const Problem &p);
+cudaError_t launch_tc(const Problem &p, cudaStream_t stream);
+
+// Device status word of the current device (set by bounded device waits).
+cudaError_t read_and_clear_device_status(unsigned int *status);
+
+enum : unsigned int { kStatusTimeout = 1u };
+
+}  // namespace gtr

@@ -1,0 +1,162 @@
+"""Thin ctypes binding over the C ABI in ``include/gtr_gla.h``.
+
+Argument marshalling only: every step of the forward runs in the library's
+CUDA kernels.  PyTorch supplies device memory and the current CUDA stream.
+There is no CPU fallback: if the library is not built, importing the entry
+points raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import Optional, Tuple
+
+import torch
+
+from . import build as _build
+
+ROW_FWD, ROW_REV, COL_FWD, COL_REV = 0, 1, 2, 3
+SCHEDULES = {"auto": 0, "simt": 1, "tc": 2}
+STATUS = {0: "GTR_OK", 1: "GTR_ERR_INVALID_ARG", 2: "GTR_ERR_UNSUPPORTED", 3: "GTR_ERR_WORKSPACE",
+          4: "GTR_ERR_CUDA", 5: "GTR_ERR_TIMEOUT"}
+_DTYPES = {torch.float32: 0, torch.float16: 1, torch.bfloat16: 2}
+
+_lock = threading.Lock()
+_lib = None
+
+
+class GLAError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {STATUS.get(status, status)}")
+
+
+def lib_path() -> str:
+    return _build.LIB_PATH
+
+
+def load(path: Optional[str] = None):
+    """Load the CUDA library (built by ``__graft_entry__.build()``)."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or _build.LIB_PATH
+        if not os.path.exists(p):
+            raise RuntimeError(f"CUDA library not built: {p} (run __graft_entry__.build())")
+        lib = ctypes.CDLL(p)
+        vp, ci, st = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+        lib.gtr_gla_fwd.restype = ci
+        lib.gtr_gla_fwd.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp]
+        lib.gtr_gla_fwd_sched.restype = ci
+        lib.gtr_gla_fwd_sched.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, ci, vp]
+        lib.gtr_gla_tc_supported.restype = ci
+        lib.gtr_gla_tc_supported.argtypes = [ci] * 8
+        lib.gtr_gla_host_buffer_bytes.restype = st
+        lib.gtr_gla_host_buffer_bytes.argtypes = [ci] * 8
+        lib.gtr_gla_fwd_host.restype = ci
+        lib.gtr_gla_fwd_host.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp, st, vp]
+        lib.gtr_gla_sync_status.restype = ci
+        lib.gtr_gla_sync_status.argtypes = [vp]
+        lib.gtr_status_string.restype = ctypes.c_char_p
+        lib.gtr_status_string.argtypes = [ci]
+        lib.gtr_last_cuda_error.restype = ci
+        lib.gtr_last_cuda_error.argtypes = []
+        lib.gtr_version.restype = ci
+        lib.gtr_version.argtypes = []
+        if path is None:
+            _lib = lib
+        return lib
+
+
+def _stream_ptr(stream) -> int:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return int(s.cuda_stream)
+
+
+def _dims(q, v, grid_h, grid_w):
+    if q.dim() != 4 or v.dim() != 4:
+        raise ValueError("q/k/log_gate must be [B,T,H,Dk] and v [B,T,H,Dv]")
+    B, T, H, Dk = q.shape
+    if T != grid_h * grid_w:
+        raise ValueError(f"T={T} != grid_h*grid_w={grid_h * grid_w}")
+    return B, H, Dk, v.shape[3]
+
+
+def _check(status: int, what: str, lib) -> None:
+    if status != 0:
+        msg = what
+        if status == 4:
+            msg += f" (cudaError {lib.gtr_last_cuda_error()})"
+        raise GLAError(status, msg)
+
+
+def tc_supported(B, H, grid_h, grid_w, Dk, Dv, order, dtype: torch.dtype) -> bool:
+    return bool(load().gtr_gla_tc_supported(B, H, grid_h, grid_w, Dk, Dv, order, _DTYPES[dtype]))
+
+
+def forward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,
+            grid_h: int, grid_w: int, order: int = ROW_FWD, out: Optional[torch.Tensor] = None,
+            final_state=True, schedule: str = "auto",
+            stream: Optional[torch.cuda.Stream] = None) -> Tuple[torch.Tensor, Optional[torch.Tensor]]:
+    """Chunkwise GLA forward through ``gtr_gla_fwd_sched``.
+
+    q, k, log_gate: [B, T, H, Dk]; v: [B, T, H, Dv]; contiguous CUDA tensors of
+    one dtype (float32 / float16 / bfloat16), T = grid_h * grid_w in spatial
+    row-major order.  ``final_state``: True (allocate), None/False (skip) or a
+    preallocated [B, H, Dk, Dv] float32 tensor.  Returns (out, final_state).
+    """
+    lib = load()
+    for name, t in (("q", q), ("k", k), ("v", v), ("log_gate", log_gate)):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+        if t.dtype != q.dtype:
+            raise ValueError("all inputs must share one dtype")
+    if q.dtype not in _DTYPES:
+        raise ValueError(f"unsupported dtype {q.dtype}")
+    B, H, Dk, Dv = _dims(q, v, grid_h, grid_w)
+    if out is None:
+        out = torch.empty(v.shape, dtype=v.dtype, device=v.device)
+    fs = None
+    if final_state is True:
+        fs = torch.empty((B, H, Dk, Dv), dtype=torch.float32, device=q.device)
+    elif isinstance(final_state, torch.Tensor):
+        fs = final_state
+    status = lib.gtr_gla_fwd_sched(
+        q.data_ptr(), k.data_ptr(), v.data_ptr(), log_gate.data_ptr(), B, H, grid_h, grid_w,
+        Dk, Dv, order, _DTYPES[q.dtype], out.data_ptr(), fs.data_ptr() if fs is not None else None,
+        SCHEDULES[schedule], _stream_ptr(stream))
+    _check(status, "gtr_gla_fwd", lib)
+    return out, fs
+
+
+def host_buffer_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype: torch.dtype, with_final_state=True):
+    return int(load().gtr_gla_host_buffer_bytes(B, H, grid_h, grid_w, Dk, Dv, _DTYPES[dtype],
+                                                int(bool(with_final_state))))
+
+
+def forward_host(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,
+                 grid_h: int, grid_w: int, order: int, out: torch.Tensor,
+                 final_state: Optional[torch.Tensor], dev_buffer: torch.Tensor,
+                 stream: Optional[torch.cuda.Stream] = None) -> None:
+    """End-to-end forward from host tensors through ``gtr_gla_fwd_host``: the
+    library copies the inputs into ``dev_buffer`` (a CUDA uint8 tensor of
+    host_buffer_bytes()), runs the forward and copies ``out`` / ``final_state``
+    back, all enqueued on the stream.  Synchronise before reading results."""
+    lib = load()
+    B, H, Dk, Dv = _dims(q, v, grid_h, grid_w)
+    for t in (q, k, v, log_gate, out):
+        if t.is_cuda or not t.is_contiguous():
+            raise ValueError("host tensors must be contiguous CPU tensors")
+    status = lib.gtr_gla_fwd_host(
+        q.data_ptr(), k.data_ptr(), v.data_ptr(), log_gate.data_ptr(), B, H, grid_h, grid_w, Dk,
+        Dv, order, _DTYPES[q.dtype], out.data_ptr(),
+        final_state.data_ptr() if final_state is not None else None, dev_buffer.data_ptr(),
+        dev_buffer.numel() * dev_buffer.element_size(), _stream_ptr(stream))
+    _check(status, "gtr_gla_fwd_host", lib)
+
+
+def sync_status(stream: Optional[torch.cuda.Stream] = None) -> int:
+    """Synchronise the stream and return/clear the device status word."""
+    return int(load().gtr_gla_sync_status(_stream_ptr(stream)))

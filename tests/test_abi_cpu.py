@@ -1,0 +1,95 @@
+"""The C-ABI library builds, loads and exports every symbol include/gtr_gla.h
+declares; host-only entry points (argument validation, support queries,
+sizes, status strings) behave as documented.  No compute is launched, so
+these run without a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2609_26590_gb300 import build as gbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADERS = [os.path.join(ROOT, "include", f) for f in os.listdir(os.path.join(ROOT, "include"))
+           if f.endswith(".h")]
+
+
+@pytest.fixture(scope="module")
+def lib():
+    path = gbuild.build()
+    from paper_2609_26590_gb300 import gla
+    return gla.load(path)
+
+
+def declared_functions():
+    names = set()
+    for h in HEADERS:
+        src = open(h).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", "", src)
+        for m in re.finditer(r"\b(gtr_[a-z0-9_]+)\s*\(", src):
+            names.add(m.group(1))
+    return sorted(names)
+
+
+def test_header_declares_entry_points():
+    names = declared_functions()
+    for must in ("gtr_gla_fwd", "gtr_gla_fwd_sched", "gtr_gla_fwd_host", "gtr_gla_sync_status",
+                 "gtr_status_string"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    raw = ctypes.CDLL(gbuild.LIB_PATH)
+    missing = [n for n in declared_functions() if not hasattr(raw, n)]
+    assert not missing, missing
+
+
+def test_status_strings_and_version(lib):
+    for s in range(6):
+        assert lib.gtr_status_string(s)
+    assert lib.gtr_status_string(99) == b"unknown status"
+    assert lib.gtr_version() >= 100
+
+
+def _fwd(lib, q=16, k=16, v=16, g=16, out=16, fs=None, B=1, H=1, gh=8, gw=8, Dk=64, Dv=64,
+         order=0, dtype=1, sched=0):
+    return lib.gtr_gla_fwd_sched(q, k, v, g, B, H, gh, gw, Dk, Dv, order, dtype, out, fs, sched,
+                                 None)
+
+
+def test_validation_rejects_before_launch(lib):
+    # null / misaligned pointers, bad sizes and enums never reach the GPU
+    assert _fwd(lib, q=None) == 1
+    assert _fwd(lib, out=None) == 1
+    assert _fwd(lib, k=24) == 1              # not 16-byte aligned
+    assert _fwd(lib, fs=8) == 1
+    assert _fwd(lib, Dk=0) == 1
+    assert _fwd(lib, Dv=129) == 1
+    assert _fwd(lib, gh=0) == 1
+    assert _fwd(lib, B=-1) == 1
+    assert _fwd(lib, order=4) == 1
+    assert _fwd(lib, dtype=3) == 1
+    assert _fwd(lib, sched=7) == 1
+    # output overlapping an input
+    assert lib.gtr_gla_fwd_sched(4096, 1 << 20, 2 << 20, 3 << 20, 1, 1, 8, 8, 64, 64, 0, 1,
+                                 4096 + 64, None, 0, None) == 1
+    # empty batch: valid, nothing to launch
+    assert _fwd(lib, B=0, q=1 << 20, k=2 << 20, v=3 << 20, g=4 << 20, out=5 << 20) == 0
+
+
+def test_host_buffer_bytes(lib):
+    n = lib.gtr_gla_host_buffer_bytes(2, 3, 4, 5, 64, 32, 1, 1)
+    T = 20
+    rnd = lambda x: (x + 255) // 256 * 256
+    assert n == 3 * rnd(2 * T * 3 * 64 * 2) + 2 * rnd(2 * T * 3 * 32 * 2) + rnd(2 * 3 * 64 * 32 * 4)
+    assert lib.gtr_gla_host_buffer_bytes(1, 1, 0, 5, 64, 64, 1, 1) == 0
+    # host entry point: missing device buffer
+    assert lib.gtr_gla_fwd_host(16, 16, 16, 16, 1, 1, 8, 8, 64, 64, 0, 1, 16, None, None, 0,
+                                None) == 3
+
+
+def test_tc_support_query_is_host_only(lib):
+    assert lib.gtr_gla_tc_supported(1, 1, 8, 8, 64, 64, 0, 0) == 0    # fp32 never on tensor cores
+    assert lib.gtr_gla_tc_supported(1, 1, 8, 8, 0, 64, 0, 1) == 0     # invalid shape

@@ -1,0 +1,217 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 CPU oracle on
+the same seeded inputs, element by element, at the five workloads' full sizes
+(every scan order) and at small ragged shapes, plus edge cases, determinism,
+CUDA-graph capture, the host-memory entry point and guard bands."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gla_testutil import assert_within_bar, errors, inputs_f64, to_torch
+from paper_2609_26590_gb300 import build as gbuild
+from paper_2609_26590_gb300 import gla
+from paper_2609_26590_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+TORCH_DT = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    gbuild.build()
+    gla.load()
+
+
+class _Cache:
+    """Inputs and oracle results of one workload at a time (the big ones take GBs)."""
+    wid = None
+    inp = None
+    f64 = None
+    ref = {}
+
+    @classmethod
+    def get(cls, wid):
+        if cls.wid != wid:
+            cls.wid, cls.ref = wid, {}
+            w = wl.WORKLOADS[wid]
+            cls.inp = wl.workload_inputs(w)
+            cls.f64 = inputs_f64(cls.inp, w.dtype)
+        return cls.inp, cls.f64
+
+    @classmethod
+    def oracle(cls, wid, order):
+        if order not in cls.ref:
+            w = wl.WORKLOADS[wid]
+            _, f = cls.get(wid)
+            cls.ref[order] = oracle.recurrence(f["q"], f["k"], f["v"], f["g"], w.grid_h, w.grid_w,
+                                               order)
+        return cls.ref[order]
+
+
+def _run(inp, dtype, gh, gw, order, schedule="auto", final_state=True):
+    t = {n: to_torch(inp[n], dtype) for n in ("q", "k", "v", "g")}
+    out, fs = gla.forward(t["q"], t["k"], t["v"], t["g"], gh, gw, order,
+                          final_state=final_state, schedule=schedule)
+    torch.cuda.synchronize()
+    assert gla.sync_status() == 0
+    return out, fs
+
+
+def _np(t):
+    return t.float().cpu().numpy().astype(np.float64)
+
+
+WORKLOAD_CASES = [(w.wid, o, s) for w in wl.WORKLOADS.values() for o in w.orders
+                  for s in ("auto", "simt")]
+
+
+@pytest.mark.parametrize("wid,order,schedule", WORKLOAD_CASES,
+                         ids=[f"w{w}-{wl.ORDER_NAMES[o]}-{s}" for w, o, s in WORKLOAD_CASES])
+def test_workload_full_size(wid, order, schedule):
+    w = wl.WORKLOADS[wid]
+    inp, _ = _Cache.get(wid)
+    ref_o, ref_s = _Cache.oracle(wid, order)
+    out, fs = _run(inp, w.dtype, w.grid_h, w.grid_w, order, schedule)
+    assert_within_bar(_np(out), ref_o, w.dtype, f"out w{wid} {schedule}")
+    assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, w.dtype, f"state w{wid}")
+
+
+# (B, H, grid_h, grid_w, Dk, Dv, dtype, tau, z_mean) -- several chunks, ragged tails,
+# fewer tokens than a chunk, non-square grids, Dk != Dv, strong decay.
+SMALL = [
+    (2, 3, 9, 13, 64, 64, "f16", 16.0, 0.0),
+    (1, 2, 5, 5, 64, 64, "bf16", 16.0, 0.0),
+    (2, 2, 16, 24, 64, 64, "bf16", 1.0, -1.0),
+    (1, 3, 40, 8, 64, 64, "f16", 1.0, -1.0),
+    (1, 1, 1, 1, 64, 64, "f32", 16.0, 0.0),
+    (1, 2, 3, 100, 128, 128, "bf16", 16.0, 0.0),
+    (2, 1, 8, 16, 128, 128, "f16", 1.0, -1.0),
+    (1, 2, 16, 16, 32, 64, "f16", 16.0, 0.0),
+    (1, 2, 12, 12, 64, 32, "f32", 16.0, 0.0),
+    (2, 2, 24, 16, 64, 64, "f16", 1.0, -3.0),
+]
+
+
+@pytest.mark.parametrize("case", SMALL, ids=[f"{c[0]}x{c[1]}-{c[2]}x{c[3]}-d{c[4]}_{c[5]}-{c[6]}"
+                                             for c in SMALL])
+@pytest.mark.parametrize("schedule", ["auto", "simt", "tc"])
+def test_small_shapes_all_orders(case, schedule):
+    B, H, gh, gw, Dk, Dv, dtype, tau, zm = case
+    if schedule == "tc" and not gla.tc_supported(B, H, gh, gw, Dk, Dv, 0, TORCH_DT[dtype]):
+        pytest.skip("tensor-core schedule does not take this shape")
+    inp = wl.make_inputs(B, H, gh, gw, Dk, Dv, dtype, seed=1000 + SMALL.index(case), tau=tau,
+                         z_mean=zm)
+    f = inputs_f64(inp, dtype)
+    for order in wl.ALL_ORDERS:
+        ref_o, ref_s = oracle.recurrence(f["q"], f["k"], f["v"], f["g"], gh, gw, order)
+        out, fs = _run(inp, dtype, gh, gw, order, schedule)
+        assert_within_bar(_np(out), ref_o, dtype, f"out order {order}")
+        assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, dtype, f"state {order}")
+
+
+@pytest.mark.parametrize("dtype", ["f16", "bf16", "f32"])
+@pytest.mark.parametrize("gate", ["one", "zero"])
+def test_gate_extremes(dtype, gate):
+    """gamma = 1 (g = 0: causal linear attention) and gamma = 0 (g = -inf:
+    o_t = (q_t . k_t) v_t) on every schedule that takes the shape."""
+    B, H, gh, gw, D = 2, 2, 16, 12, 64
+    inp = wl.make_inputs(B, H, gh, gw, D, D, dtype, seed=5)
+    g = np.zeros((B, gh * gw, H, D)) if gate == "one" else np.full((B, gh * gw, H, D), -np.inf)
+    inp["g"] = wl.round_to_storage(g, dtype)
+    f = inputs_f64(inp, dtype)
+    for schedule in ("auto", "simt"):
+        for order in wl.ALL_ORDERS:
+            ref_o, ref_s = oracle.recurrence(f["q"], f["k"], f["v"], f["g"], gh, gw, order)
+            out, fs = _run(inp, dtype, gh, gw, order, schedule)
+            assert_within_bar(_np(out), ref_o, dtype, f"{gate} {schedule} {order}")
+            assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, dtype, "state")
+
+
+def test_no_final_state_and_empty_batch():
+    inp = wl.make_inputs(1, 2, 8, 8, 64, 64, "f16", seed=3)
+    f = inputs_f64(inp, "f16")
+    out, fs = _run(inp, "f16", 8, 8, wl.COL_FWD, final_state=None)
+    assert fs is None
+    ref_o, _ = oracle.recurrence(f["q"], f["k"], f["v"], f["g"], 8, 8, wl.COL_FWD)
+    assert_within_bar(_np(out), ref_o, "f16")
+    z = torch.empty((0, 64, 2, 64), dtype=torch.float16, device="cuda")
+    o, s = gla.forward(z, z, z, z, 8, 8, 0)
+    assert o.shape == z.shape and s.shape == (0, 2, 64, 64)
+
+
+@pytest.mark.parametrize("wid", [1, 3])
+def test_deterministic(wid):
+    w = wl.WORKLOADS[wid]
+    inp, _ = _Cache.get(wid)
+    a, sa = _run(inp, w.dtype, w.grid_h, w.grid_w, wl.COL_REV)
+    b, sb = _run(inp, w.dtype, w.grid_h, w.grid_w, wl.COL_REV)
+    assert torch.equal(a, b) and torch.equal(sa, sb)
+
+
+def test_guard_bands_and_full_coverage():
+    """Outputs pre-filled with NaN inside a sentinel-padded allocation: every
+    output element is written, nothing outside is touched."""
+    B, H, gh, gw, D = 2, 3, 9, 13, 64
+    inp = wl.make_inputs(B, H, gh, gw, D, D, "bf16", seed=9)
+    t = {n: to_torch(inp[n], "bf16") for n in ("q", "k", "v", "g")}
+    n_out = B * gh * gw * H * D
+    pad = 4096
+    buf = torch.full((n_out + 2 * pad,), 1024.0, dtype=torch.bfloat16, device="cuda")
+    buf[pad:pad + n_out] = float("nan")
+    out = buf[pad:pad + n_out].view(B, gh * gw, H, D)
+    fbuf = torch.full((B * H * D * D + 2 * pad,), -777.0, device="cuda")
+    fbuf[pad:pad + B * H * D * D] = float("nan")
+    fs = fbuf[pad:pad + B * H * D * D].view(B, H, D, D)
+    for order in wl.ALL_ORDERS:
+        gla.forward(t["q"], t["k"], t["v"], t["g"], gh, gw, order, out=out, final_state=fs)
+        torch.cuda.synchronize()
+        assert not torch.isnan(out).any() and not torch.isnan(fs).any()
+        assert (buf[:pad] == 1024.0).all() and (buf[pad + n_out:] == 1024.0).all()
+        assert (fbuf[:pad] == -777.0).all() and (fbuf[pad + B * H * D * D:] == -777.0).all()
+
+
+def test_cuda_graph_capture():
+    w = wl.WORKLOADS[1]
+    inp, _ = _Cache.get(1)
+    t = {n: to_torch(inp[n], w.dtype) for n in ("q", "k", "v", "g")}
+    out = torch.empty_like(t["v"])
+    fs = torch.empty((w.B, w.H, w.Dk, w.Dv), device="cuda")
+    gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, wl.ROW_REV, out=out,
+                final_state=fs)   # warm-up outside capture
+    torch.cuda.synchronize()
+    ref = out.clone()
+    out.zero_()
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, wl.ROW_REV, out=out,
+                        final_state=fs, stream=s)
+    g.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(out, ref)
+
+
+def test_host_memory_entry_point():
+    w = wl.WORKLOADS[1]
+    inp, f = _Cache.get(1)
+    host = {n: to_torch(inp[n], w.dtype, device="cpu").pin_memory() for n in ("q", "k", "v", "g")}
+    out = torch.empty(host["v"].shape, dtype=host["v"].dtype).pin_memory()
+    fs = torch.empty((w.B, w.H, w.Dk, w.Dv)).pin_memory()
+    nbytes = gla.host_buffer_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, host["q"].dtype)
+    dev = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    gla.forward_host(host["q"], host["k"], host["v"], host["g"], w.grid_h, w.grid_w, wl.COL_FWD,
+                     out, fs, dev)
+    torch.cuda.synchronize()
+    ref_o, ref_s = _Cache.oracle(1, wl.COL_FWD)
+    assert_within_bar(out.float().numpy().astype(np.float64), ref_o, w.dtype, "host out")
+    assert_within_bar(fs.numpy().astype(np.float64), ref_s, w.dtype, "host state")
+
+
+def test_explicit_schedule_rejects_unsupported():
+    inp = wl.make_inputs(1, 1, 4, 4, 64, 64, "f32", seed=1)
+    t = {n: to_torch(inp[n], "f32") for n in ("q", "k", "v", "g")}
+    with pytest.raises(gla.GLAError) as ei:
+        gla.forward(t["q"], t["k"], t["v"], t["g"], 4, 4, 0, schedule="tc")
+    assert ei.value.status == 2
