@@ -49,11 +49,15 @@ gtr_status_t make_problem(const void *q, const void *k, const void *v, const voi
                           void *out, float *final_state, gtr::Problem *p) {
     gtr_status_t st = check_shape(B, H, grid_h, grid_w, Dk, Dv, order, dtype);
     if (st != GTR_OK) return st;
+    const long long T = (long long)grid_h * grid_w;
+    if (B == 0 || H == 0) {  // nothing is read or written: pointers may be null
+        *p = gtr::Problem{q, k, v, g, out, final_state, B, H, grid_h, grid_w, Dk, Dv, order, dtype, T};
+        return GTR_OK;
+    }
     if (!q || !k || !v || !g || !out) return GTR_ERR_INVALID_ARG;
     if (!aligned(q) || !aligned(k) || !aligned(v) || !aligned(g) || !aligned(out) ||
         !aligned(final_state))
         return GTR_ERR_INVALID_ARG;
-    const long long T = (long long)grid_h * grid_w;
     const size_t es = elem_size(dtype);
     const size_t nk = (size_t)B * T * H * Dk * es, nv = (size_t)B * T * H * Dv * es;
     const size_t nfs = (size_t)B * H * Dk * Dv * sizeof(float);

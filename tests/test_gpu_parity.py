@@ -90,6 +90,11 @@ SMALL = [
     (1, 2, 16, 16, 32, 64, "f16", 16.0, 0.0),
     (1, 2, 12, 12, 64, 32, "f32", 16.0, 0.0),
     (2, 2, 24, 16, 64, 64, "f16", 1.0, -3.0),
+    (1, 2, 8, 8, 64, 64, "bf16", 16.0, 0.0),
+    (1, 2, 8, 13, 64, 64, "bf16", 16.0, 0.0),
+    (2, 1, 16, 9, 64, 64, "f16", 1.0, -1.0),
+    (3, 2, 8, 24, 64, 64, "f16", 16.0, 0.0),
+    (1, 1, 48, 40, 64, 64, "bf16", 1.0, -1.0),
 ]
 
 
