@@ -48,6 +48,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override the workload's batch size (smaller cases for profiling)")
     return ap.parse_args()
 
 
@@ -215,6 +217,9 @@ def main():
     args = parse()
     rank, world, local = dist_env()
     w = wl.WORKLOADS[args.workload]
+    if args.batch is not None:
+        import dataclasses
+        w = dataclasses.replace(w, B=args.batch, name=f"{w.name}_b{args.batch}")
     if args.impl == "reference":
         run_reference(args, w, rank, world)
         return
@@ -234,7 +239,7 @@ def main():
     dt = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}[w.dtype]
 
     # inputs: rank r draws batch r of the workload (same distributions, own seed)
-    inp = wl.workload_inputs(w, seed=1234 + w.wid + 1000 * rank)
+    inp = wl.workload_inputs(w, B=w.B, seed=1234 + w.wid + 1000 * rank)
 
     def to_dev(a):
         if w.dtype == "bf16":
