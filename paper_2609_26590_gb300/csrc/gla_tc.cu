@@ -6,27 +6,34 @@
 //   o_r      = (q_r . e^{A_r}) S_[c] + sum_{j<=r} (sum_i q_ri k_ji e^{A_ri - A_ji}) v_j
 //   U_c      = sum_r (k_r . e^{A_last - A_r})^T v_r,   d_c = e^{A_last}
 //   S_[c+1]  = Diag(d_c) S_[c] + U_c
-// One CTA walks all chunks of one (b, h) sequence (single pass: every input is
-// read once and o, S_final written once; S stays on chip between chunks).
+// One CTA walks all chunks of one (b, h) sequence (single pass: q, k, v, g are
+// read once, o and S_final written once; S stays on chip between chunks).
 //
-// Warp roles (320 threads):
-//   warp 0      TMA producer: 8-row boxes of q, k, v, g gathered in scan order
-//               (the scan permutation is applied in the box coordinates).
-//   warp 1      TMEM allocator + single-thread tcgen05 MMA issuer.
-//   warps 2-5   "gen" warpgroup: in-chunk prefix sum of the log-gates (fp32,
-//               log2 domain), then the decay-scaled MMA operands.
-//   warps 6-9   "epi" warpgroup: reads accumulators from TMEM, applies the
-//               causal mask, carries the fp32 state S in registers, converts
-//               and stores o through TMA (scatter back to spatial order).
+// Per chunk, five tensor-core products (tcgen05.mma, fp32 accumulators in TMEM):
+//   A = L G          in-chunk cumulative log-decay: L is the 64x64 triangle of
+//                    ones in scan order, G the gate tile as loaded (exact products)
+//   P = Q^ K^^T      intra-chunk scores with e^{A_r - A_j} split at the mid-chunk
+//                    reference: Q^ = q e^{A_r - A_mid}, K^ = k e^{A_mid - A_j}
+//   U = Kbar^T V     chunk summary, Kbar = k e^{A_last - A}
+//   O = Qtil S_[c] + P V   outputs, Qtil = q e^{A}
+// The split factors of P lie within 2^{+-M}, M = max_i max(-A_mid, A_mid - A_last)
+// (log2 units).  M <= 12: Q^, K^ are fp16 (kind::f16); M <= 100: tf32 (fp32
+// range, kind::tf32); larger (extreme decay, gamma -> 0) or non-finite gates: the
+// chunk's scores and log-decays are computed exactly by CUDA cores.  All other
+// operands carry factors <= 1 and are fp16; bf16 values become fp16 operands.
 //
-// Intra-chunk scores: e^{A_r - A_j} is split at the mid-chunk reference
-// A_mid = A_31 as e^{A_r - A_mid} e^{A_mid - A_j}.  Both factors lie within
-// 2^{+-M}, M = max_i max(-A_mid, A_mid - A_last) (log2 units); when M <= 100 the
-// two scaled operands are exact enough in tf32 and P = Q^ K^^T runs on the tensor
-// core (kind::tf32).  Otherwise (extreme decay, e.g. gamma = 0) the chunk's scores
-// are computed exactly by the gen warpgroup with per-element exponentials.
-// All other operands carry factors <= 1 and are fp16 (kind::f16):
-//   U = Kbar^T V   (Kbar = k e^{A_last - A}),  O = Qtil S + P V  (Qtil = q e^{A}).
+// Warp roles (448 threads, one CTA per SM):
+//   warp 0       TMA producer: q, k, v, g tiles gathered in scan order (64-row
+//                boxes for row orders, 8-row boxes down a column for column
+//                orders); the scan permutation lives in the box coordinates.
+//   warp 1       TMEM allocator + single-thread MMA issuer (issues in data-flow
+//                order: whichever product has its inputs ready).
+//   warps 2-5    gen: reads A from TMEM, builds the decay-scaled operands.
+//   warps 6-9    epi-P: masks P into fp16, carries the fp32 state S in registers.
+//   warps 10-13  epi-O: converts O, TMA-stores it back in spatial order.
+// A warp reads the TMEM lanes of sub-partition (warp % 4); an M = 64 accumulator
+// keeps rows 16q..16q+15 in lanes 32q..32q+15, and each thread takes one row and
+// 32 of its 64 columns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -49,70 +56,72 @@ using namespace ptx;
 constexpr int kC = 64;                    // chunk length
 constexpr int kD = 64;                    // Dk = Dv handled by this kernel
 constexpr int kStages = 3;                // input stage ring
-constexpr int kTile16 = kC * kD * 2;      // one 64 x 64 16-bit tile (SW128, 128-byte rows)
-constexpr int kTile32 = kC * kD * 4;      // one 64 x 64 fp32 tile (two 32-column K-blocks)
-constexpr int kThreads = 320;
+constexpr int kTile16 = kC * kD * 2;      // 64 x 64 16-bit tile (SW128, 128-byte rows)
+constexpr int kTile32 = kC * kD * 4;      // 64 x 64 fp32 tile (two 32-column K-blocks)
+constexpr int kThreads = 448;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kGateMinLog2 = -1.0e4f * 1.4426950408889634f;  // g < -1e4 acts as -1e4
-constexpr float kMaxRefExp = 100.0f;      // tf32 score path bound (log2 units)
+constexpr float kMaxRefF16 = 12.0f;       // fp16 score operands: factors within 2^{+-12}
+constexpr float kMaxRefTF32 = 100.0f;     // tf32 score operands: factors within 2^{+-100}
 
-enum : uint32_t { kModeTF32 = 0, kModeExact = 1 };
+enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
 
 // Shared-memory map (byte offsets from a 1024-aligned base).
-constexpr int kOffStage = 0;                                   // kStages x {q,k,v,g}
-constexpr int kStageBytes = 4 * kTile16;
-constexpr int kOffOp = kOffStage + kStages * kStageBytes;      // 2 x {Q^, K^} tf32
+constexpr int kStageBytes = 4 * kTile16;                       // q, k, v, g
+constexpr int kOffStage = 0;
+constexpr int kOffOp = kOffStage + kStages * kStageBytes;      // 2 x {Q^ | K^} (tf32 size)
 constexpr int kOpBytes = 2 * kTile32;
-constexpr int kOffS = kOffOp + 2 * kOpBytes;                   // 2 x S (fp16, MN-major)
+constexpr int kOffS = kOffOp + 2 * kOpBytes;                   // 2 x S_[c] (fp16, MN-major)
 constexpr int kOffO = kOffS + 2 * kTile16;                     // 2 x O staging
-constexpr int kOffDecay = kOffO + 2 * kTile16;                 // kStages x 64 fp32
-constexpr int kOffMode = kOffDecay + kStages * kD * 4;         // kStages x u32
-constexpr int kOffTot = kOffMode + 64;                         // 2 x 4 x 64 fp32 quarter totals
-constexpr int kOffBar = kOffTot + 2 * 4 * kD * 4;              // mbarriers
-constexpr int kNumBars = 32;
+constexpr int kOffL = kOffO + 2 * kTile16;                     // triangle of ones
+constexpr int kRefFloats = 5 * kD;                             // raw mid, raw last, mid*log2e, c1, c2
+constexpr int kOffRef = kOffL + kTile16;                       // 2 x kRefFloats
+constexpr int kOffDecay = kOffRef + 2 * kRefFloats * 4;        // kStages x 64 fp32
+constexpr int kOffMode = kOffDecay + kStages * kD * 4;         // kStages x u32, 2 x 2 maxima
+constexpr int kOffBar = kOffMode + 64;
+constexpr int kNumBars = 40;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;               // tmem base, abort flag
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;               // + alignment slack
+static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
-// mbarrier indices
 enum {
-    BAR_FULL = 0,                 // [kStages] TMA -> gen
+    BAR_FULL = 0,                    // [kStages] TMA -> MMA/gen (tiles landed)
     BAR_EMPTY = BAR_FULL + kStages,  // [kStages] MMA (O done) -> producer
-    BAR_OPND = BAR_EMPTY + kStages,  // [2] gen -> MMA (operands ready)
-    BAR_OPFREE = BAR_OPND + 2,       // [2] MMA (P done) -> gen (Q^/K^ buffers free)
-    BAR_PFULL = BAR_OPFREE + 2,      // [2] MMA -> epi (P accumulator ready)
-    BAR_UFULL = BAR_PFULL + 2,       // [2] MMA -> epi (U accumulator ready)
-    BAR_OFULL = BAR_UFULL + 2,       // [2] MMA -> epi (O accumulator ready)
-    BAR_PREADY = BAR_OFULL + 2,      // [2] epi -> MMA (masked fp16 P in smem)
-    BAR_SREADY = BAR_PREADY + 2,     // [2] epi -> MMA (S_[c] fp16 in smem)
-    BAR_TFREE_P = BAR_SREADY + 2,    // [2] epi -> MMA (TMEM P drained)
-    BAR_TFREE_U = BAR_TFREE_P + 2,   // [2]
-    BAR_TFREE_O = BAR_TFREE_U + 2,   // [2]
-    BAR_DONE = BAR_TFREE_O + 2,      // MMA: all issued MMAs completed
+    BAR_AFULL = BAR_EMPTY + kStages, // [2] MMA -> gen (A accumulator ready)
+    BAR_TFREE_A = BAR_AFULL + 2,     // [2] gen -> MMA (A drained)
+    BAR_OPND = BAR_TFREE_A + 2,      // [2] gen -> MMA (operands ready)
+    BAR_OPFREE = BAR_OPND + 2,       // [2] MMA (P done) -> gen (Q^/K^ buffer free)
+    BAR_PFULL = BAR_OPFREE + 2,      // [2] MMA -> epi-P
+    BAR_UFULL = BAR_PFULL + 2,       // [2] MMA -> epi-P
+    BAR_OFULL = BAR_UFULL + 2,       // [2] MMA -> epi-O (and epi-P: S buffer free)
+    BAR_PREADY = BAR_OFULL + 2,      // [2] epi-P -> MMA (masked fp16 P in smem)
+    BAR_SREADY = BAR_PREADY + 2,     // [2] epi-P -> MMA (S_[c] fp16 in smem)
+    BAR_TFREE_P = BAR_SREADY + 2,    // [2] epi-P -> MMA
+    BAR_TFREE_U = BAR_TFREE_P + 2,   // [2] epi-P -> MMA
+    BAR_TFREE_O = BAR_TFREE_U + 2,   // [2] epi-O -> MMA
+    BAR_DONE = BAR_TFREE_O + 2,      // MMA: every issued MMA completed
     BAR_COUNT
 };
 static_assert(BAR_COUNT <= kNumBars, "barrier space");
 
-// TMEM columns (fp32 accumulators, M = 64 layout)
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColP = 0, kColU = 128, kColO = 256;
+constexpr uint32_t kColA = 0, kColP = 128, kColU = 256, kColO = 384;
 
 struct TmaMaps {
-    CUtensorMap q, k, v, g, o;
+    CUtensorMap q, k, v, g, o, o8;  // o8: 8-row store boxes (row orders, ragged reversed chunk)
 };
 
 struct TcParams {
     TmaMaps maps;
     float *final_state;
-    int H, grid_h, grid_w, order, n_chunks;
-    int T;
+    int H, grid_h, grid_w, order, n_chunks, T;
 };
 
-// ---------------------------------------------------------------- small helpers
+// ---------------------------------------------------------------- helpers
 __device__ __forceinline__ uint32_t sw128(uint32_t row, uint32_t byte) {
     return row * 128u + ((((byte >> 4) ^ (row & 7u)) << 4) | (byte & 15u));
 }
-// 64 x 64 fp32 tile stored as two K-blocks of 32 columns (8 KB each)
 __device__ __forceinline__ uint32_t off32(uint32_t row, uint32_t col) {
     return (col >> 5) * 8192u + sw128(row, (col & 31u) * 4u);
 }
@@ -126,60 +135,114 @@ __device__ __forceinline__ float to_tf32(float x) {
     asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
     return __uint_as_float(r);
 }
+__device__ __forceinline__ uint32_t h2bits(float a, float b) {
+    __half2 h = __floats2half2_rn(a, b);
+    return *reinterpret_cast<uint32_t *>(&h);
+}
 
-template <typename E> struct Pack;
-template <> struct Pack<__half> {
-    static __device__ __forceinline__ float2 load(const uint8_t *p) {
-        return __half22float2(*reinterpret_cast<const __half2 *>(p));
+template <typename E> struct Elem;
+template <> struct Elem<__half> {
+    static constexpr uint32_t fmt = kFmtF16;
+    static constexpr uint16_t one = 0x3C00;
+    static __device__ __forceinline__ float2 unpack(uint32_t w) {
+        return __half22float2(*reinterpret_cast<const __half2 *>(&w));
     }
-    static __device__ __forceinline__ uint32_t from2(float a, float b) {
-        __half2 h = __floats2half2_rn(a, b);
-        return *reinterpret_cast<uint32_t *>(&h);
-    }
+    static __device__ __forceinline__ uint32_t pack(float a, float b) { return h2bits(a, b); }
 };
-template <> struct Pack<__nv_bfloat16> {
-    static __device__ __forceinline__ float2 load(const uint8_t *p) {
-        return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(p));
+template <> struct Elem<__nv_bfloat16> {
+    static constexpr uint32_t fmt = kFmtBF16;
+    static constexpr uint16_t one = 0x3F80;
+    static __device__ __forceinline__ float2 unpack(uint32_t w) {
+        return __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w));
     }
-    static __device__ __forceinline__ uint32_t from2(float a, float b) {
+    static __device__ __forceinline__ uint32_t pack(float a, float b) {
         __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
         return *reinterpret_cast<uint32_t *>(&h);
     }
 };
-__device__ __forceinline__ uint32_t half2_bits(float a, float b) {
-    __half2 h = __floats2half2_rn(a, b);
-    return *reinterpret_cast<uint32_t *>(&h);
-}
 
 __device__ __forceinline__ void record_timeout(volatile uint32_t *abort_flag) {
     *abort_flag = 1u;
     atomicOr(&g_device_status, kStatusTimeout);
 }
 
-// TMA box coordinates of 8-row group `grp` of chunk `c` (scan positions
-// 64c + 8grp .. +7, in smem rows 8grp .. 8grp+7).  Row orders use maps with dims
-// (D, H, T, 1, B); column orders (D, H, W, Hg, B).  Reverse orders address the
-// reversed range, so smem row rho holds scan position 64c + 63 - rho.  Returns
-// false when the whole group lies outside the sequence.
+// Scan positions 64c + 8grp .. +7 (smem rows 8grp .. 8grp+7) as 8-row box
+// coordinates.  Row orders address dims (D, H, T, 1, B), column orders
+// (D, H, W, Hg, B).  Reverse orders address the mirrored range, so smem row
+// rho holds scan position 64c + 63 - rho.  Returns false when the group lies
+// entirely outside the sequence (loads then read zero fill, stores are skipped).
 __device__ __forceinline__ bool group_coords(int order, int T, int grid_h, int c, int grp,
                                              int &x2, int &x3) {
     const int rev = order & 1;
-    if ((order >> 1) == 0) {  // row orders: token index along dim 2
-        int t0 = rev ? (T - kC * (c + 1) + 8 * grp) : (kC * c + 8 * grp);
-        x2 = t0;
+    const int u0 = rev ? (T - kC * (c + 1) + 8 * grp) : (kC * c + 8 * grp);
+    if ((order >> 1) == 0) {
+        x2 = u0;
         x3 = 0;
-        return rev ? (t0 + 8 > 0) : (t0 < T);
+        return u0 >= 0 && u0 < T;
     }
-    // column orders: position u in the top-to-bottom column walk -> (x = u / Hg, y = u % Hg)
-    int u0 = rev ? (T - kC * (c + 1) + 8 * grp) : (kC * c + 8 * grp);
-    if (u0 < 0 || u0 >= T) {  // entirely outside: point past the last column (zero fill)
-        x2 = T / grid_h;
+    if (u0 < 0 || u0 >= T) {
+        x2 = T / grid_h;  // one past the last column: zero fill
         x3 = 0;
         return false;
     }
     x2 = u0 / grid_h;
     x3 = u0 % grid_h;
     return true;
+}
+
+// Exact scores for one chunk (extreme or non-finite log-decays): serial prefix
+// of the clamped gates, P[rho][sigma] = sum_i q k 2^{a_r,i - a_j,i} (j <= r) by
+// CUDA cores, Qtil = q 2^{a}, Kbar = k 2^{a_last - a}, and the chunk decay.
+template <typename E>
+__device__ __noinline__ void exact_chunk(uint8_t *tq, uint8_t *tk, uint8_t *tgate, float *as,
+                                         float *decay, int rev, int tg) {
+    if (tg < kD) {
+        float run = 0.f;
+        for (int r = 0; r < kC; ++r) {
+            const int rho = rev ? kC - 1 - r : r;
+            const uint16_t bits = *reinterpret_cast<const uint16_t *>(tgate + sw128(rho, tg * 2));
+            float x = Elem<E>::unpack(bits).x * kLog2e;
+            x = x < kGateMinLog2 ? kGateMinLog2 : x;
+            run += x;
+            as[rho * kD + tg] = run;
+        }
+        decay[tg] = ex2(run);
+    }
+    named_barrier_sync(1, 128);
+    const int rho = tg >> 1, half = tg & 1;
+    const int r = rev ? kC - 1 - rho : rho;
+    uint32_t packed[16];
+    for (int jj = 0; jj < 16; ++jj) {
+        float pv[2];
+        for (int u = 0; u < 2; ++u) {
+            const int sig = half * 32 + 2 * jj + u;
+            const int j = rev ? kC - 1 - sig : sig;
+            float acc = 0.f;
+            if (j <= r) {
+                for (int i = 0; i < kD; i += 2) {
+                    const float2 qi = Elem<E>::unpack(*reinterpret_cast<const uint32_t *>(tq + sw128(rho, i * 2)));
+                    const float2 ki = Elem<E>::unpack(*reinterpret_cast<const uint32_t *>(tk + sw128(sig, i * 2)));
+                    acc += qi.x * ki.x * ex2(as[rho * kD + i] - as[sig * kD + i]);
+                    acc += qi.y * ki.y * ex2(as[rho * kD + i + 1] - as[sig * kD + i + 1]);
+                }
+            }
+            pv[u] = acc;
+        }
+        packed[jj] = h2bits(pv[0], pv[1]);
+    }
+    const int rho_last = rev ? 0 : kC - 1;
+    named_barrier_sync(1, 128);  // every q/k/gate read of this chunk is done
+    for (int jj = 0; jj < 16; ++jj)
+        *reinterpret_cast<uint32_t *>(tgate + sw128(rho, (half * 32 + 2 * jj) * 2)) = packed[jj];
+    for (int i = half * 32; i < half * 32 + 32; i += 2) {
+        const uint32_t o16 = sw128(rho, i * 2);
+        const float2 q2 = Elem<E>::unpack(*reinterpret_cast<const uint32_t *>(tq + o16));
+        const float2 k2 = Elem<E>::unpack(*reinterpret_cast<const uint32_t *>(tk + o16));
+        const float a0 = as[rho * kD + i], a1 = as[rho * kD + i + 1];
+        const float l0 = as[rho_last * kD + i], l1 = as[rho_last * kD + i + 1];
+        *reinterpret_cast<uint32_t *>(tq + o16) = h2bits(q2.x * ex2(a0), q2.y * ex2(a1));
+        *reinterpret_cast<uint32_t *>(tk + o16) = h2bits(k2.x * ex2(l0 - a0), k2.y * ex2(l1 - a1));
+    }
 }
 
 template <typename E>
@@ -192,13 +255,14 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     volatile uint32_t *abort_flag = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc + 4);
     float *decay_s = reinterpret_cast<float *>(smem + kOffDecay);
     volatile uint32_t *mode_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMode);
-    float *tot_s = reinterpret_cast<float *>(smem + kOffTot);
+    float *mx_s = reinterpret_cast<float *>(smem + kOffMode + 16);   // [2][2] partial maxima
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int bh = blockIdx.x;
     const int b = bh / p.H, h = bh % p.H;
     const int N = p.n_chunks;
     const int rev = p.order & 1;
+    const bool col_order = (p.order >> 1) != 0;
 
     if (threadIdx.x == 0) {
         *abort_flag = 0u;
@@ -207,6 +271,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             mbar_init(&bars[BAR_EMPTY + i], 1);
         }
         for (int i = 0; i < 2; ++i) {
+            mbar_init(&bars[BAR_AFULL + i], 1);
+            mbar_init(&bars[BAR_TFREE_A + i], 4);
             mbar_init(&bars[BAR_OPND + i], 4);
             mbar_init(&bars[BAR_OPFREE + i], 1);
             mbar_init(&bars[BAR_PFULL + i], 1);
@@ -232,6 +298,32 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         tma_prefetch_desc(&p.maps.g);
         tma_prefetch_desc(&p.maps.o);
     }
+    if (warp >= 2 && warp < 6) {
+        // triangle of ones in scan order: L[rho][sigma] = 1 when sigma is at or before rho
+        const int tg = threadIdx.x - 64;
+        const int rho = tg >> 1, half = tg & 1;
+        uint8_t *L = smem + kOffL;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int s0 = half * 32 + u * 8 + 2 * e;
+                const bool k0 = rev ? (s0 >= rho) : (s0 <= rho);
+                const bool k1 = rev ? (s0 + 1 >= rho) : (s0 + 1 <= rho);
+                w[e] = (k0 ? (uint32_t)Elem<E>::one : 0u) | ((k1 ? (uint32_t)Elem<E>::one : 0u) << 16);
+            }
+            *reinterpret_cast<uint4 *>(L + sw128(rho, (half * 32 + u * 8) * 2)) = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        fence_proxy_async_smem();
+    }
+    if (warp >= 6 && warp < 10) {
+        // S_[0] = 0
+        const int te = threadIdx.x - 192;
+        for (int i = te; i < kTile16 / 16; i += 128)
+            reinterpret_cast<uint4 *>(smem + kOffS)[i] = make_uint4(0, 0, 0, 0);
+        fence_proxy_async_smem();
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -243,234 +335,265 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             int issued = 0;
             for (int c = 0; c < N; ++c) {
                 const int s = c % kStages;
-                if (!mbar_wait(&bars[BAR_EMPTY + s], ((c / kStages) & 1) ^ 1, abort_flag,
-                               kWaitLimitNs)) {
+                if (!mbar_wait(&bars[BAR_EMPTY + s], ((c / kStages) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
                     record_timeout(abort_flag);
                     break;
                 }
                 uint8_t *st = smem + kOffStage + s * kStageBytes;
-                mbar_arrive_expect_tx(&bars[BAR_FULL + s], kStageBytes);
-                for (int grp = 0; grp < 8; ++grp) {
-                    int x2, x3;
-                    group_coords(p.order, p.T, p.grid_h, c, grp, x2, x3);
-                    const uint32_t o = grp * 1024;
-                    tma_load_5d(st + 0 * kTile16 + o, &p.maps.q, &bars[BAR_FULL + s], 0, h, x2, x3, b);
-                    tma_load_5d(st + 1 * kTile16 + o, &p.maps.k, &bars[BAR_FULL + s], 0, h, x2, x3, b);
-                    tma_load_5d(st + 2 * kTile16 + o, &p.maps.v, &bars[BAR_FULL + s], 0, h, x2, x3, b);
-                    tma_load_5d(st + 3 * kTile16 + o, &p.maps.g, &bars[BAR_FULL + s], 0, h, x2, x3, b);
+                uint64_t *fb = &bars[BAR_FULL + s];
+                mbar_arrive_expect_tx(fb, kStageBytes);
+                if (!col_order) {
+                    const int t0 = rev ? (p.T - kC * (c + 1)) : kC * c;
+                    tma_load_5d(st + 0 * kTile16, &p.maps.q, fb, 0, h, t0, 0, b);
+                    tma_load_5d(st + 1 * kTile16, &p.maps.k, fb, 0, h, t0, 0, b);
+                    tma_load_5d(st + 2 * kTile16, &p.maps.v, fb, 0, h, t0, 0, b);
+                    tma_load_5d(st + 3 * kTile16, &p.maps.g, fb, 0, h, t0, 0, b);
+                } else {
+                    for (int grp = 0; grp < 8; ++grp) {
+                        int x2, x3;
+                        group_coords(p.order, p.T, p.grid_h, c, grp, x2, x3);
+                        const uint32_t o = grp * 1024;
+                        tma_load_5d(st + 0 * kTile16 + o, &p.maps.q, fb, 0, h, x2, x3, b);
+                        tma_load_5d(st + 1 * kTile16 + o, &p.maps.k, fb, 0, h, x2, x3, b);
+                        tma_load_5d(st + 2 * kTile16 + o, &p.maps.v, fb, 0, h, x2, x3, b);
+                        tma_load_5d(st + 3 * kTile16 + o, &p.maps.g, fb, 0, h, x2, x3, b);
+                    }
                 }
                 ++issued;
             }
-            // never leave the CTA while loads are in flight into its shared memory
-            if (*abort_flag) {
+            if (*abort_flag) {  // never leave while copies are still landing in shared memory
                 for (int c = (issued > kStages ? issued - kStages : 0); c < issued; ++c)
                     mbar_wait(&bars[BAR_FULL + c % kStages], (c / kStages) & 1, nullptr, kWaitLimitNs);
             }
         }
     } else if (warp == 1) {
-        // ======================================================= MMA issuer
+        // ======================================================= MMA issuer (data-flow order)
         if (lane == 0) {
-            const uint32_t idesc_p = instr_desc(kFmtTF32, 64, 64, 0, 0);
+            const uint32_t idesc_a = instr_desc(Elem<E>::fmt, 64, 64, 0, 1);
+            const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
+            const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
             const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
             const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
             const uint32_t sbase = smem_u32(smem);
+            int nA = 0, nPU = 0, nO = 0;
             bool ok = true;
-            auto issue_pu = [&](int c) -> bool {
-                const int s = c % kStages, bb = c & 1;
-                const uint32_t ph = (c >> 1) & 1;
-                if (!mbar_wait(&bars[BAR_OPND + bb], ph, abort_flag, kWaitLimitNs)) return false;
-                const uint32_t mode = mode_s[s];
-                if (mode == kModeTF32) {
-                    if (!mbar_wait(&bars[BAR_TFREE_P + bb], ph ^ 1, abort_flag, kWaitLimitNs)) return false;
-                    tc_fence_after();
-                    const uint32_t qh = sbase + kOffOp + bb * kOpBytes, kh = qh + kTile32;
-                    for (int ks = 0; ks < 8; ++ks) {
-                        const uint32_t off = (ks >> 2) * 8192 + (ks & 3) * 32;
-                        mma_tf32_ss(tmem + kColP + bb * 64, smem_desc(qh + off, 16, 1024, kLayoutSw128),
-                                    smem_desc(kh + off, 16, 1024, kLayoutSw128), idesc_p, ks > 0);
+            uint64_t t_idle = global_timer_ns();
+            uint32_t spins = 0;
+            while (nO < N) {
+                bool did = false;
+                if (nO < nPU) {  // O(c) = Qtil S_[c] + P V
+                    const int c = nO, s = c % kStages, bb = c & 1;
+                    const uint32_t ph = (c >> 1) & 1;
+                    if (mbar_test(&bars[BAR_PREADY + bb], ph) && mbar_test(&bars[BAR_SREADY + bb], ph) &&
+                        mbar_test(&bars[BAR_TFREE_O + bb], ph ^ 1)) {
+                        tc_fence_after();
+                        const uint32_t st = sbase + kOffStage + s * kStageBytes;
+                        const uint32_t qt = st, vv = st + 2 * kTile16, pp = st + 3 * kTile16;
+                        const uint32_t ss = sbase + kOffS + bb * kTile16;
+                        const uint32_t d = tmem + kColO + bb * 64;
+#pragma unroll
+                        for (int ks = 0; ks < 4; ++ks)
+                            mma_f16_ss(d, smem_desc(qt + ks * 32, 16, 1024, kLayoutSw128),
+                                       smem_desc(ss + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, ks > 0);
+#pragma unroll
+                        for (int ks = 0; ks < 4; ++ks)
+                            mma_f16_ss(d, smem_desc(pp + ks * 32, 16, 1024, kLayoutSw128),
+                                       smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
+                        mma_commit(&bars[BAR_OFULL + bb]);
+                        mma_commit(&bars[BAR_EMPTY + s]);
+                        ++nO;
+                        did = true;
                     }
-                    mma_commit(&bars[BAR_PFULL + bb]);
-                    mma_commit(&bars[BAR_OPFREE + bb]);
-                } else {
-                    mbar_arrive(&bars[BAR_PFULL + bb]);
-                    mbar_arrive(&bars[BAR_OPFREE + bb]);
                 }
-                if (!mbar_wait(&bars[BAR_TFREE_U + bb], ph ^ 1, abort_flag, kWaitLimitNs)) return false;
-                tc_fence_after();
-                const uint32_t st = sbase + kOffStage + s * kStageBytes;
-                const uint32_t kb = st + 1 * kTile16, vv = st + 2 * kTile16;
-                for (int ks = 0; ks < 4; ++ks) {
-                    mma_f16_ss(tmem + kColU + bb * 64, smem_desc(kb + ks * 2048, 8192, 1024, kLayoutSw128),
-                               smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_u, ks > 0);
+                if (!did && nPU < nA) {  // P(c) = Q^ K^^T and U(c) = Kbar^T V
+                    const int c = nPU, s = c % kStages, bb = c & 1;
+                    const uint32_t ph = (c >> 1) & 1;
+                    if (mbar_test(&bars[BAR_OPND + bb], ph) && mbar_test(&bars[BAR_TFREE_P + bb], ph ^ 1) &&
+                        mbar_test(&bars[BAR_TFREE_U + bb], ph ^ 1)) {
+                        tc_fence_after();
+                        const uint32_t mode = mode_s[s];
+                        const uint32_t qh = sbase + kOffOp + bb * kOpBytes, kh = qh + kTile32;
+                        if (mode == kModeTF32) {
+#pragma unroll
+                            for (int ks = 0; ks < 8; ++ks) {
+                                const uint32_t o = (ks >> 2) * 8192 + (ks & 3) * 32;
+                                mma_tf32_ss(tmem + kColP + bb * 64, smem_desc(qh + o, 16, 1024, kLayoutSw128),
+                                            smem_desc(kh + o, 16, 1024, kLayoutSw128), idesc_p32, ks > 0);
+                            }
+                            mma_commit(&bars[BAR_PFULL + bb]);
+                            mma_commit(&bars[BAR_OPFREE + bb]);
+                        } else if (mode == kModeF16) {
+#pragma unroll
+                            for (int ks = 0; ks < 4; ++ks)
+                                mma_f16_ss(tmem + kColP + bb * 64, smem_desc(qh + ks * 32, 16, 1024, kLayoutSw128),
+                                           smem_desc(kh + ks * 32, 16, 1024, kLayoutSw128), idesc_p16, ks > 0);
+                            mma_commit(&bars[BAR_PFULL + bb]);
+                            mma_commit(&bars[BAR_OPFREE + bb]);
+                        } else {
+                            mbar_arrive(&bars[BAR_PFULL + bb]);
+                            mbar_arrive(&bars[BAR_OPFREE + bb]);
+                        }
+                        const uint32_t st = sbase + kOffStage + s * kStageBytes;
+                        const uint32_t kb = st + 1 * kTile16, vv = st + 2 * kTile16;
+#pragma unroll
+                        for (int ks = 0; ks < 4; ++ks)
+                            mma_f16_ss(tmem + kColU + bb * 64, smem_desc(kb + ks * 2048, 8192, 1024, kLayoutSw128),
+                                       smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_u, ks > 0);
+                        mma_commit(&bars[BAR_UFULL + bb]);
+                        ++nPU;
+                        did = true;
+                    }
                 }
-                mma_commit(&bars[BAR_UFULL + bb]);
-                return true;
-            };
-            if (N > 0) ok = issue_pu(0);
-            for (int c = 0; c < N && ok; ++c) {
-                if (c + 1 < N && !(ok = issue_pu(c + 1))) break;
-                const int s = c % kStages, bb = c & 1;
-                const uint32_t ph = (c >> 1) & 1;
-                if (!mbar_wait(&bars[BAR_PREADY + bb], ph, abort_flag, kWaitLimitNs) ||
-                    !mbar_wait(&bars[BAR_SREADY + bb], ph, abort_flag, kWaitLimitNs) ||
-                    !mbar_wait(&bars[BAR_TFREE_O + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
-                    ok = false;
-                    break;
+                if (!did && nA < N) {  // A(c) = L G
+                    const int c = nA, s = c % kStages, bb = c & 1;
+                    if (mbar_test(&bars[BAR_FULL + s], (c / kStages) & 1) &&
+                        mbar_test(&bars[BAR_TFREE_A + bb], ((c >> 1) & 1) ^ 1)) {
+                        tc_fence_after();
+                        const uint32_t L = sbase + kOffL;
+                        const uint32_t gt = sbase + kOffStage + s * kStageBytes + 3 * kTile16;
+#pragma unroll
+                        for (int ks = 0; ks < 4; ++ks)
+                            mma_f16_ss(tmem + kColA + bb * 64, smem_desc(L + ks * 32, 16, 1024, kLayoutSw128),
+                                       smem_desc(gt + ks * 2048, 8192, 1024, kLayoutSw128), idesc_a, ks > 0);
+                        mma_commit(&bars[BAR_AFULL + bb]);
+                        ++nA;
+                        did = true;
+                    }
                 }
-                tc_fence_after();
-                const uint32_t st = sbase + kOffStage + s * kStageBytes;
-                const uint32_t qt = st, vv = st + 2 * kTile16, pp = st + 3 * kTile16;
-                const uint32_t ss = sbase + kOffS + bb * kTile16;
-                const uint32_t dcol = tmem + kColO + bb * 64;
-                for (int ks = 0; ks < 4; ++ks)  // O = Qtil S_[c]
-                    mma_f16_ss(dcol, smem_desc(qt + ks * 32, 16, 1024, kLayoutSw128),
-                               smem_desc(ss + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, ks > 0);
-                for (int ks = 0; ks < 4; ++ks)  // O += P V
-                    mma_f16_ss(dcol, smem_desc(pp + ks * 32, 16, 1024, kLayoutSw128),
-                               smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
-                mma_commit(&bars[BAR_OFULL + bb]);
-                mma_commit(&bars[BAR_EMPTY + s]);
+                if (did) {
+                    spins = 0;
+                    t_idle = global_timer_ns();
+                } else if ((++spins & 127u) == 0u) {
+                    if (*abort_flag || global_timer_ns() - t_idle > kWaitLimitNs) {
+                        ok = false;
+                        break;
+                    }
+                }
             }
             if (!ok) record_timeout(abort_flag);
-            // all MMAs this thread issued must finish before TMEM is released
-            mma_commit(&bars[BAR_DONE]);
+            mma_commit(&bars[BAR_DONE]);  // TMEM is released only after every MMA completed
             mbar_wait(&bars[BAR_DONE], 0, nullptr, kWaitLimitNs);
         }
     } else if (warp < 6) {
         // ======================================================= gen warpgroup
-        const int tq = warp - 2;          // scan positions 16 tq .. 16 tq + 15
-        const int ch = 2 * lane;          // key channels ch, ch + 1
-        const int tg = threadIdx.x - 64;  // 0..127
+        const int q4 = warp & 3, hc = lane >> 4;
+        const int row = 16 * q4 + (lane & 15);   // smem row rho of this thread's accumulator row
+        const int ch0 = 32 * hc;                 // its 32 key channels
+        const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
+        const int tg = threadIdx.x - 64;
+        const int rho_mid = rev ? 32 : 31, rho_last = rev ? 0 : 63;
         for (int c = 0; c < N; ++c) {
             const int s = c % kStages, bb = c & 1;
-            if (!mbar_wait(&bars[BAR_FULL + s], (c / kStages) & 1, abort_flag, kWaitLimitNs) ||
-                !mbar_wait(&bars[BAR_OPFREE + bb], ((c >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+            const uint32_t ph = (c >> 1) & 1;
+            if (!mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs) ||
+                !mbar_wait(&bars[BAR_OPFREE + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
                 record_timeout(abort_flag);
                 break;
             }
-            uint8_t *st = smem + kOffStage + s * kStageBytes;
-            uint8_t *tq_ = st, *tk = st + kTile16, *tv = st + 2 * kTile16, *tgate = st + 3 * kTile16;
-            // -- in-chunk cumulative log-decay (log2 units), Sec. 3.3: A_r = sum_{m<=r} g_m
-            float2 a[16];
-            float2 run = make_float2(0.f, 0.f);
+            tc_fence_after();
+            uint32_t ar[32];
+            tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&ar[0]));
+            tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&ar[16]));
+            tmem_ld_wait();
+            float *ref = reinterpret_cast<float *>(smem + kOffRef) + bb * kRefFloats;
+            if (row == rho_mid || row == rho_last) {
+                float *dst = ref + (row == rho_mid ? 0 : kD) + ch0;
 #pragma unroll
-            for (int t = 0; t < 16; ++t) {
-                const int r = 16 * tq + t;
-                const int rho = rev ? 63 - r : r;
-                float2 g2 = Pack<E>::load(tgate + sw128(rho, ch * 2));
-                float x = g2.x * kLog2e, y = g2.y * kLog2e;
-                x = x < kGateMinLog2 ? kGateMinLog2 : x;
-                y = y < kGateMinLog2 ? kGateMinLog2 : y;
-                run.x += x;
-                run.y += y;
-                a[t] = run;
+                for (int u = 0; u < 8; ++u)
+                    reinterpret_cast<float4 *>(dst)[u] = make_float4(__uint_as_float(ar[4 * u]), __uint_as_float(ar[4 * u + 1]),
+                                                                     __uint_as_float(ar[4 * u + 2]), __uint_as_float(ar[4 * u + 3]));
             }
-            float *tot = tot_s + bb * 4 * kD;  // double-buffered: chunk c+1 may write while c is read
-            *reinterpret_cast<float2 *>(tot + tq * kD + ch) = run;
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bars[BAR_TFREE_A + bb]);
             named_barrier_sync(1, 128);
-            float2 off = make_float2(0.f, 0.f), amid, alast;
-            {
-                const float2 t0 = *reinterpret_cast<const float2 *>(tot + 0 * kD + ch);
-                const float2 t1 = *reinterpret_cast<const float2 *>(tot + 1 * kD + ch);
-                const float2 t2 = *reinterpret_cast<const float2 *>(tot + 2 * kD + ch);
-                const float2 t3 = *reinterpret_cast<const float2 *>(tot + 3 * kD + ch);
-                if (tq > 0) { off.x += t0.x; off.y += t0.y; }
-                if (tq > 1) { off.x += t1.x; off.y += t1.y; }
-                if (tq > 2) { off.x += t2.x; off.y += t2.y; }
-                amid = make_float2(t0.x + t1.x, t0.y + t1.y);
-                alast = make_float2(amid.x + t2.x + t3.x, amid.y + t2.y + t3.y);
+            if (tg < kD) {  // per-channel references (log2 units) and split constants
+                const float am = ref[tg] * kLog2e, al = ref[kD + tg] * kLog2e;
+                float m = fmaxf(-am, am - al);
+                if (!(m <= 3.0e38f)) m = 3.0e38f;  // NaN / inf gates: exact path
+                ref[2 * kD + tg] = am;
+                ref[3 * kD + tg] = ex2(am);
+                ref[4 * kD + tg] = ex2(al - am);
+                decay_s[s * kD + tg] = ex2(al);
+                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 16));
+                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 8));
+                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 4));
+                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
+                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+                if (lane == 0) mx_s[bb * 2 + (tg >> 5)] = m;
             }
-#pragma unroll
-            for (int t = 0; t < 16; ++t) { a[t].x += off.x; a[t].y += off.y; }
-            // -- score-path selection: largest |exponent| of the mid-chunk split
-            float m = fmaxf(fmaxf(-amid.x, amid.x - alast.x), fmaxf(-amid.y, amid.y - alast.y));
-            if (m != m) m = 1e30f;  // NaN gates: exact path (propagates NaN)
-            const uint32_t mbits = __reduce_max_sync(0xffffffffu, __float_as_uint(fmaxf(m, 0.f)));
-            const uint32_t mode = (__uint_as_float(mbits) <= kMaxRefExp) ? kModeTF32 : kModeExact;
-            if (tq == 3) {
-                decay_s[s * kD + ch] = ex2(alast.x);
-                decay_s[s * kD + ch + 1] = ex2(alast.y);
-            }
+            named_barrier_sync(1, 128);
+            const float mmax = fmaxf(mx_s[bb * 2], mx_s[bb * 2 + 1]);
+            const uint32_t mode = mmax <= kMaxRefF16 ? kModeF16 : (mmax <= kMaxRefTF32 ? kModeTF32 : kModeExact);
             if (tg == 0) mode_s[s] = mode;
-            if (mode == kModeTF32) {
+            uint8_t *st = smem + kOffStage + s * kStageBytes;
+            uint8_t *tq = st, *tk = st + kTile16, *tv = st + 2 * kTile16, *tgt = st + 3 * kTile16;
+            if (mode != kModeExact) {
                 uint8_t *qh = smem + kOffOp + bb * kOpBytes, *kh = qh + kTile32;
-                const float c1x = ex2(amid.x), c1y = ex2(amid.y);                    // <= 1
-                const float c2x = ex2(alast.x - amid.x), c2y = ex2(alast.y - amid.y);  // <= 1
 #pragma unroll
-                for (int t = 0; t < 16; ++t) {
-                    const int r = 16 * tq + t;
-                    const int rho = rev ? 63 - r : r;
-                    const float ex = a[t].x - amid.x, ey = a[t].y - amid.y;
-                    const float fqx = ex2(ex), fqy = ex2(ey), fkx = ex2(-ex), fky = ex2(-ey);
-                    const uint32_t o16 = sw128(rho, ch * 2);
-                    const float2 q2 = Pack<E>::load(tq_ + o16);
-                    const float2 k2 = Pack<E>::load(tk + o16);
-                    const float qx = q2.x * fqx, qy = q2.y * fqy, kx = k2.x * fkx, ky = k2.y * fky;
-                    *reinterpret_cast<float2 *>(qh + off32(rho, ch)) = make_float2(to_tf32(qx), to_tf32(qy));
-                    *reinterpret_cast<float2 *>(kh + off32(rho, ch)) = make_float2(to_tf32(kx), to_tf32(ky));
-                    *reinterpret_cast<uint32_t *>(tq_ + o16) = half2_bits(qx * c1x, qy * c1y);
-                    *reinterpret_cast<uint32_t *>(tk + o16) = half2_bits(kx * c2x, ky * c2y);
+                for (int g8 = 0; g8 < 4; ++g8) {
+                    const int cl = ch0 + 8 * g8;
+                    const float4 am0 = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl);
+                    const float4 am1 = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl + 4);
+                    const float4 c10 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl);
+                    const float4 c11 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl + 4);
+                    const float4 c20 = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl);
+                    const float4 c21 = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl + 4);
+                    const float amv[8] = {am0.x, am0.y, am0.z, am0.w, am1.x, am1.y, am1.z, am1.w};
+                    const float c1v[8] = {c10.x, c10.y, c10.z, c10.w, c11.x, c11.y, c11.z, c11.w};
+                    const float c2v[8] = {c20.x, c20.y, c20.z, c20.w, c21.x, c21.y, c21.z, c21.w};
+                    const uint32_t o16 = sw128(row, cl * 2);
+                    const uint4 qw = *reinterpret_cast<const uint4 *>(tq + o16);
+                    const uint4 kw = *reinterpret_cast<const uint4 *>(tk + o16);
+                    const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w}, ka[4] = {kw.x, kw.y, kw.z, kw.w};
+                    float qs[8], ks[8];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float2 q2 = Elem<E>::unpack(qa[e]), k2 = Elem<E>::unpack(ka[e]);
+                        const float e0 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e]), kLog2e, -amv[2 * e]);
+                        const float e1 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e + 1]), kLog2e, -amv[2 * e + 1]);
+                        qs[2 * e] = q2.x * ex2(e0);
+                        qs[2 * e + 1] = q2.y * ex2(e1);
+                        ks[2 * e] = k2.x * ex2(-e0);
+                        ks[2 * e + 1] = k2.y * ex2(-e1);
+                    }
+                    if (mode == kModeF16) {
+                        *reinterpret_cast<uint4 *>(qh + o16) =
+                            make_uint4(h2bits(qs[0], qs[1]), h2bits(qs[2], qs[3]), h2bits(qs[4], qs[5]), h2bits(qs[6], qs[7]));
+                        *reinterpret_cast<uint4 *>(kh + o16) =
+                            make_uint4(h2bits(ks[0], ks[1]), h2bits(ks[2], ks[3]), h2bits(ks[4], ks[5]), h2bits(ks[6], ks[7]));
+                    } else {
+                        *reinterpret_cast<float4 *>(qh + off32(row, cl)) =
+                            make_float4(to_tf32(qs[0]), to_tf32(qs[1]), to_tf32(qs[2]), to_tf32(qs[3]));
+                        *reinterpret_cast<float4 *>(qh + off32(row, cl + 4)) =
+                            make_float4(to_tf32(qs[4]), to_tf32(qs[5]), to_tf32(qs[6]), to_tf32(qs[7]));
+                        *reinterpret_cast<float4 *>(kh + off32(row, cl)) =
+                            make_float4(to_tf32(ks[0]), to_tf32(ks[1]), to_tf32(ks[2]), to_tf32(ks[3]));
+                        *reinterpret_cast<float4 *>(kh + off32(row, cl + 4)) =
+                            make_float4(to_tf32(ks[4]), to_tf32(ks[5]), to_tf32(ks[6]), to_tf32(ks[7]));
+                    }
+                    *reinterpret_cast<uint4 *>(tq + o16) =
+                        make_uint4(h2bits(qs[0] * c1v[0], qs[1] * c1v[1]), h2bits(qs[2] * c1v[2], qs[3] * c1v[3]),
+                                   h2bits(qs[4] * c1v[4], qs[5] * c1v[5]), h2bits(qs[6] * c1v[6], qs[7] * c1v[7]));
+                    *reinterpret_cast<uint4 *>(tk + o16) =
+                        make_uint4(h2bits(ks[0] * c2v[0], ks[1] * c2v[1]), h2bits(ks[2] * c2v[2], ks[3] * c2v[3]),
+                                   h2bits(ks[4] * c2v[4], ks[5] * c2v[5]), h2bits(ks[6] * c2v[6], ks[7] * c2v[7]));
                 }
             } else {
-                // exact scores: P[rho][sigma] = sum_i q_i k_i 2^{a_r,i - a_j,i} for j <= r
-                float *as = reinterpret_cast<float *>(smem + kOffOp + bb * kOpBytes);  // [64][64] by rho
-#pragma unroll
-                for (int t = 0; t < 16; ++t) {
-                    const int r = 16 * tq + t;
-                    const int rho = rev ? 63 - r : r;
-                    *reinterpret_cast<float2 *>(as + rho * kD + ch) = a[t];
-                }
-                named_barrier_sync(1, 128);
-                {
-                    const int rho = tg >> 1, half = tg & 1;
-                    const int r = rev ? 63 - rho : rho;
-                    uint32_t packed[16];
-                    for (int jj = 0; jj < 32; jj += 2) {
-                        float pv[2];
-                        for (int u = 0; u < 2; ++u) {
-                            const int sig = half * 32 + jj + u;
-                            const int j = rev ? 63 - sig : sig;
-                            float acc = 0.f;
-                            if (j <= r) {
-                                for (int i = 0; i < kD; i += 2) {
-                                    const float2 qi = Pack<E>::load(tq_ + sw128(rho, i * 2));
-                                    const float2 ki = Pack<E>::load(tk + sw128(sig, i * 2));
-                                    acc += qi.x * ki.x * ex2(as[rho * kD + i] - as[sig * kD + i]);
-                                    acc += qi.y * ki.y * ex2(as[rho * kD + i + 1] - as[sig * kD + i + 1]);
-                                }
-                            }
-                            pv[u] = acc;
-                        }
-                        packed[jj >> 1] = half2_bits(pv[0], pv[1]);
-                    }
-                    for (int jj = 0; jj < 16; ++jj)
-                        *reinterpret_cast<uint32_t *>(tgate + sw128(rho, (half * 32 + 2 * jj) * 2)) = packed[jj];
-                }
-                named_barrier_sync(1, 128);
-#pragma unroll
-                for (int t = 0; t < 16; ++t) {
-                    const int r = 16 * tq + t;
-                    const int rho = rev ? 63 - r : r;
-                    const uint32_t o16 = sw128(rho, ch * 2);
-                    const float2 q2 = Pack<E>::load(tq_ + o16);
-                    const float2 k2 = Pack<E>::load(tk + o16);
-                    *reinterpret_cast<uint32_t *>(tq_ + o16) =
-                        half2_bits(q2.x * ex2(a[t].x), q2.y * ex2(a[t].y));
-                    *reinterpret_cast<uint32_t *>(tk + o16) =
-                        half2_bits(k2.x * ex2(alast.x - a[t].x), k2.y * ex2(alast.y - a[t].y));
-                }
+                exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp + bb * kOpBytes),
+                               decay_s + s * kD, rev, tg);
             }
-            // bf16 inputs: values become fp16 MMA operands (exact for |v| in the fp16 normal range)
             if constexpr (std::is_same<E, __nv_bfloat16>::value) {
+                // bf16 values become fp16 MMA operands (exact for |v| in the fp16 normal range)
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    uint4 *pv = reinterpret_cast<uint4 *>(tv) + tg * 4 + u;
+                    uint4 *pv = reinterpret_cast<uint4 *>(tv + sw128(row, (ch0 + 8 * u) * 2));
                     uint4 w = *pv;
                     uint32_t *wp = reinterpret_cast<uint32_t *>(&w);
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        const float2 f = __bfloat1622float2(*reinterpret_cast<__nv_bfloat162 *>(&wp[e]));
-                        wp[e] = half2_bits(f.x, f.y);
+                        const float2 f = Elem<E>::unpack(wp[e]);
+                        wp[e] = h2bits(f.x, f.y);
                     }
                     *pv = w;
                 }
@@ -479,133 +602,141 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_OPND + bb]);
         }
-    } else {
-        // ======================================================= epi warpgroup
-        const int qd = warp & 3;                     // TMEM sub-partition of this warp
-        const bool has_row = lane < 16;              // M = 64 layout: 16 rows per sub-partition
-        const int row = qd * 16 + (lane & 15);       // accumulator row (token rho or channel i)
-        const uint32_t lane_base = static_cast<uint32_t>(qd * 32) << 16;
-        const bool elected = (warp == 6 && lane == 0);
-        float S[kD];
+    } else if (warp < 10) {
+        // ======================================================= epi-P warpgroup
+        const int q4 = warp & 3, hc = lane >> 4;
+        const int row = 16 * q4 + (lane & 15);   // token rho for P, channel i for U / S
+        const int ch0 = 32 * hc;
+        const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
+        if (lane == 0) mbar_arrive(&bars[BAR_SREADY + 0]);  // S_[0] = 0 written before the CTA barrier
+        float S[32];
 #pragma unroll
-        for (int j = 0; j < kD; ++j) S[j] = 0.f;
-        // S_[0] = 0
-        {
-            const int te = threadIdx.x - 192;
-            uint4 z = make_uint4(0, 0, 0, 0);
-            for (int i = te; i < kTile16 / 16; i += 128)
-                reinterpret_cast<uint4 *>(smem + kOffS)[i] = z;
-            fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_SREADY + 0]);
-        }
+        for (int j = 0; j < 32; ++j) S[j] = 0.f;
         bool ok = true;
         for (int c = 0; c < N; ++c) {
             const int s = c % kStages, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
-            uint8_t *st = smem + kOffStage + s * kStageBytes;
             if (!mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs)) { ok = false; break; }
             const uint32_t mode = mode_s[s];
             const float dc = decay_s[s * kD + row];
-            if (mode == kModeTF32) {
+            if (mode != kModeExact) {
                 tc_fence_after();
-                uint8_t *pt = st + 3 * kTile16;
+                uint32_t r[32];
+                tmem_ld_16x32bx2_x16(tmem + lane_base + kColP + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+                tmem_ld_16x32bx2_x16(tmem + lane_base + kColP + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+                tmem_ld_wait();
+                uint8_t *pt = smem + kOffStage + s * kStageBytes + 3 * kTile16;
 #pragma unroll
-                for (int cb = 0; cb < 4; ++cb) {
-                    uint32_t r[16];
-                    tmem_ld_32x32b_x16(tmem + lane_base + kColP + bb * 64 + cb * 16, r);
-                    tmem_ld_wait();
-                    if (has_row) {
-                        uint32_t w[8];
+                for (int u = 0; u < 4; ++u) {
+                    uint32_t w[4];
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            const int s0 = cb * 16 + 2 * e;
-                            const bool k0 = rev ? (s0 >= row) : (s0 <= row);
-                            const bool k1 = rev ? (s0 + 1 >= row) : (s0 + 1 <= row);
-                            w[e] = half2_bits(k0 ? __uint_as_float(r[2 * e]) : 0.f,
-                                              k1 ? __uint_as_float(r[2 * e + 1]) : 0.f);
-                        }
-                        *reinterpret_cast<uint4 *>(pt + sw128(row, cb * 32)) = make_uint4(w[0], w[1], w[2], w[3]);
-                        *reinterpret_cast<uint4 *>(pt + sw128(row, cb * 32 + 16)) = make_uint4(w[4], w[5], w[6], w[7]);
+                    for (int e = 0; e < 4; ++e) {
+                        const int s0 = ch0 + 8 * u + 2 * e;
+                        const bool k0 = rev ? (s0 >= row) : (s0 <= row);
+                        const bool k1 = rev ? (s0 + 1 >= row) : (s0 + 1 <= row);
+                        w[e] = h2bits(k0 ? __uint_as_float(r[8 * u + 2 * e]) : 0.f,
+                                      k1 ? __uint_as_float(r[8 * u + 2 * e + 1]) : 0.f);
                     }
+                    *reinterpret_cast<uint4 *>(pt + sw128(row, (ch0 + 8 * u) * 2)) = make_uint4(w[0], w[1], w[2], w[3]);
                 }
             }
-            // arrived every chunk (also when the exact path skipped the P accumulator)
             tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_TFREE_P + bb]);
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_PREADY + bb]);
-            // -- state carry: S_[c+1] = Diag(d_c) S_[c] + U_c
+            if (lane == 0) {
+                mbar_arrive(&bars[BAR_TFREE_P + bb]);
+                mbar_arrive(&bars[BAR_PREADY + bb]);
+            }
+            // state carry: S_[c+1] = Diag(d_c) S_[c] + U_c
             if (!mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs)) { ok = false; break; }
             tc_fence_after();
-#pragma unroll
-            for (int cb = 0; cb < 4; ++cb) {
-                uint32_t r[16];
-                tmem_ld_32x32b_x16(tmem + lane_base + kColU + bb * 64 + cb * 16, r);
+            {
+                uint32_t r[32];
+                tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+                tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
 #pragma unroll
-                for (int e = 0; e < 16; ++e) S[cb * 16 + e] = fmaf(dc, S[cb * 16 + e], __uint_as_float(r[e]));
+                for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], __uint_as_float(r[j]));
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_U + bb]);
             if (c + 1 < N) {
-                uint8_t *sb = smem + kOffS + ((c + 1) & 1) * kTile16;
-                if (has_row) {
-#pragma unroll
-                    for (int cb = 0; cb < 8; ++cb) {
-                        uint32_t w[4];
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) w[e] = half2_bits(S[cb * 8 + 2 * e], S[cb * 8 + 2 * e + 1]);
-                        *reinterpret_cast<uint4 *>(sb + sw128(row, cb * 16)) = make_uint4(w[0], w[1], w[2], w[3]);
-                    }
+                const int nb = (c + 1) & 1;
+                // buffer nb was last read by O(c-1)
+                if (c >= 1 && !mbar_wait(&bars[BAR_OFULL + nb], ((c - 1) >> 1) & 1, abort_flag, kWaitLimitNs)) {
+                    ok = false;
+                    break;
                 }
+                uint8_t *sb = smem + kOffS + nb * kTile16;
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    *reinterpret_cast<uint4 *>(sb + sw128(row, (ch0 + 8 * u) * 2)) =
+                        make_uint4(h2bits(S[8 * u + 0], S[8 * u + 1]), h2bits(S[8 * u + 2], S[8 * u + 3]),
+                                   h2bits(S[8 * u + 4], S[8 * u + 5]), h2bits(S[8 * u + 6], S[8 * u + 7]));
                 fence_proxy_async_smem();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&bars[BAR_SREADY + ((c + 1) & 1)]);
+                if (lane == 0) mbar_arrive(&bars[BAR_SREADY + nb]);
             }
-            // -- output: TMEM -> dtype -> smem -> TMA store in spatial order
+        }
+        if (!ok) record_timeout(abort_flag);
+        if (ok && p.final_state != nullptr) {
+            float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)bh * kD + row) * kD + ch0);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
+        }
+    } else {
+        // ======================================================= epi-O warpgroup
+        const int q4 = warp & 3, hc = lane >> 4;
+        const int row = 16 * q4 + (lane & 15);
+        const int ch0 = 32 * hc;
+        const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
+        const bool elected = (warp == 10 && lane == 0);
+        bool ok = true;
+        for (int c = 0; c < N; ++c) {
+            const int bb = c & 1;
+            const uint32_t ph = (c >> 1) & 1;
             if (!mbar_wait(&bars[BAR_OFULL + bb], ph, abort_flag, kWaitLimitNs)) { ok = false; break; }
             if (elected) tma_store_wait_read<1>();
-            named_barrier_sync(2, 128);
+            named_barrier_sync(3, 128);
             tc_fence_after();
+            uint32_t r[32];
+            tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+            tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+            tmem_ld_wait();
             uint8_t *ob = smem + kOffO + bb * kTile16;
 #pragma unroll
-            for (int cb = 0; cb < 4; ++cb) {
-                uint32_t r[16];
-                tmem_ld_32x32b_x16(tmem + lane_base + kColO + bb * 64 + cb * 16, r);
-                tmem_ld_wait();
-                if (has_row) {
-                    uint32_t w[8];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        w[e] = Pack<E>::from2(__uint_as_float(r[2 * e]), __uint_as_float(r[2 * e + 1]));
-                    *reinterpret_cast<uint4 *>(ob + sw128(row, cb * 32)) = make_uint4(w[0], w[1], w[2], w[3]);
-                    *reinterpret_cast<uint4 *>(ob + sw128(row, cb * 32 + 16)) = make_uint4(w[4], w[5], w[6], w[7]);
-                }
-            }
+            for (int u = 0; u < 4; ++u)
+                *reinterpret_cast<uint4 *>(ob + sw128(row, (ch0 + 8 * u) * 2)) = make_uint4(
+                    Elem<E>::pack(__uint_as_float(r[8 * u + 0]), __uint_as_float(r[8 * u + 1])),
+                    Elem<E>::pack(__uint_as_float(r[8 * u + 2]), __uint_as_float(r[8 * u + 3])),
+                    Elem<E>::pack(__uint_as_float(r[8 * u + 4]), __uint_as_float(r[8 * u + 5])),
+                    Elem<E>::pack(__uint_as_float(r[8 * u + 6]), __uint_as_float(r[8 * u + 7])));
             tc_fence_before();
+            fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_O + bb]);
-            fence_proxy_async_smem();
-            named_barrier_sync(2, 128);
+            named_barrier_sync(3, 128);
             if (elected) {
-                for (int grp = 0; grp < 8; ++grp) {
-                    int x2, x3;
-                    if (group_coords(p.order, p.T, p.grid_h, c, grp, x2, x3))
-                        tma_store_5d(&p.maps.o, ob + grp * 1024, 0, h, x2, x3, b);
+                if (!col_order) {
+                    const int t0 = rev ? (p.T - kC * (c + 1)) : kC * c;
+                    if (t0 >= 0) {
+                        tma_store_5d(&p.maps.o, ob, 0, h, t0, 0, b);
+                    } else {  // ragged first-in-memory chunk of a reverse scan: 8-row boxes from t = 0
+                        for (int grp = 0; grp < 8; ++grp)
+                            if (t0 + 8 * grp >= 0) tma_store_5d(&p.maps.o8, ob + grp * 1024, 0, h, t0 + 8 * grp, 0, b);
+                    }
+                } else {
+                    for (int grp = 0; grp < 8; ++grp) {
+                        int x2, x3;
+                        if (group_coords(p.order, p.T, p.grid_h, c, grp, x2, x3))
+                            tma_store_5d(&p.maps.o, ob + grp * 1024, 0, h, x2, x3, b);
+                    }
                 }
                 tma_store_commit();
             }
         }
         if (!ok) record_timeout(abort_flag);
-        if (ok && p.final_state != nullptr && has_row) {
-            float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)bh * kD + row) * kD);
-#pragma unroll
-            for (int j = 0; j < kD / 4; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
-        }
         if (elected) tma_store_wait_all<0>();
     }
 
@@ -624,68 +755,59 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     std::call_once(once, [] {
         cudaDriverEntryPointQueryResult q;
         void *f = nullptr;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault,
-                                             &q) == cudaSuccess &&
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
             fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
     });
     return fn;
 }
 
-// dims (D, H, T, 1, B) for row orders, (D, H, W, Hg, B) for column orders; box 8 rows.
-bool encode_map(CUtensorMap *m, const void *ptr, int dtype, const Problem &p, int D) {
+// Row orders: dims (D, H, T, 1, B), box (64, 1, rows, 1, 1).
+// Column orders: dims (D, H, W, Hg, B), box (64, 1, 1, 8, 1).
+bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int rows) {
     auto enc = get_encode();
     if (!enc) return false;
-    const cuuint64_t es = 2;
+    const cuuint64_t es = 2, D = kD;
     const bool col = (p.order >> 1) != 0;
-    cuuint64_t dims[5], strides[4];
-    cuuint32_t box[5], estr[5] = {1, 1, 1, 1, 1};
-    dims[0] = D;
-    dims[1] = p.H;
-    strides[0] = (cuuint64_t)D * es;
-    strides[1] = (cuuint64_t)p.H * D * es;
+    cuuint64_t dims[5] = {D, (cuuint64_t)p.H, 0, 0, (cuuint64_t)p.B};
+    cuuint64_t strides[4] = {D * es, (cuuint64_t)p.H * D * es, 0, (cuuint64_t)p.T * p.H * D * es};
+    cuuint32_t box[5] = {64, 1, 1, 1, 1}, estr[5] = {1, 1, 1, 1, 1};
     if (!col) {
-        dims[2] = p.T;
+        dims[2] = (cuuint64_t)p.T;
         dims[3] = 1;
         strides[2] = (cuuint64_t)p.T * p.H * D * es;
-        box[2] = 8;
-        box[3] = 1;
+        box[2] = (cuuint32_t)rows;
     } else {
-        dims[2] = p.grid_w;
-        dims[3] = p.grid_h;
+        dims[2] = (cuuint64_t)p.grid_w;
+        dims[3] = (cuuint64_t)p.grid_h;
         strides[2] = (cuuint64_t)p.grid_w * p.H * D * es;
-        box[2] = 1;
         box[3] = 8;
     }
-    dims[4] = p.B;
-    strides[3] = (cuuint64_t)p.T * p.H * D * es;
-    box[0] = 64;
-    box[1] = 1;
-    box[4] = 1;
-    const CUtensorMapDataType dt =
-        dtype == 1 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
-    CUresult r = enc(m, dt, 5, const_cast<void *>(ptr), dims, strides, box, estr,
-                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
+    const CUtensorMapDataType dt = p.dtype == 1 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    return enc(m, dt, 5, const_cast<void *>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
 
 bool tc_supported(const Problem &p) {
-    if (p.dtype != 1 && p.dtype != 2) return false;      // fp16 / bf16 operands only
+    if (p.dtype != 1 && p.dtype != 2) return false;       // fp16 / bf16 operands only
     if (p.Dk != kD || p.Dv != kD) return false;
-    if (p.T % 8 != 0) return false;                       // 8-row boxes never straddle the end
-    if ((p.order >> 1) != 0 && p.grid_h % 8 != 0) return false;  // 8-row groups inside one column
+    if (p.T % 8 != 0) return false;                        // 8-row store boxes never straddle the end
+    if ((p.order >> 1) != 0 && p.grid_h % 8 != 0) return false;  // 8-row groups stay in one column
     if (p.T > (1 << 30)) return false;
     return get_encode() != nullptr;
 }
 
 cudaError_t launch_tc(const Problem &p, cudaStream_t stream) {
     TcParams tp;
-    if (!encode_map(&tp.maps.q, p.q, p.dtype, p, kD) || !encode_map(&tp.maps.k, p.k, p.dtype, p, kD) ||
-        !encode_map(&tp.maps.v, p.v, p.dtype, p, kD) || !encode_map(&tp.maps.g, p.g, p.dtype, p, kD) ||
-        !encode_map(&tp.maps.o, p.out, p.dtype, p, kD))
+    const bool col = (p.order >> 1) != 0;
+    const int rows = col ? 8 : 64;
+    if (!encode_map(&tp.maps.q, p.q, p, rows) || !encode_map(&tp.maps.k, p.k, p, rows) ||
+        !encode_map(&tp.maps.v, p.v, p, rows) || !encode_map(&tp.maps.g, p.g, p, rows) ||
+        !encode_map(&tp.maps.o, p.out, p, rows) || !encode_map(&tp.maps.o8, p.out, p, 8))
         return cudaErrorInvalidValue;
     tp.final_state = p.final_state;
     tp.H = p.H;
