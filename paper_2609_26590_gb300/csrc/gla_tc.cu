@@ -16,8 +16,12 @@
 //                    reference: Q^ = q e^{A_r - A_mid}, K^ = k e^{A_mid - A_j}
 //   U = Kbar^T V     chunk summary, Kbar = k e^{A_last - A}
 //   O = Qtil S_[c] + P V   outputs, Qtil = q e^{A}
+// With fp16 score operands the per-channel constants c1 = e^{A_mid} and
+// c2 = e^{A_last - A_mid} are folded into the state instead of the tiles:
+// Qtil S = Q^ (Diag(c1) S) and Kbar^T V = Diag(c2) K^^T V, so Q^ and K^ serve
+// all four products and only the 64 x 64 state is rescaled per chunk.
 // The split factors of P lie within 2^{+-M}, M = max_i max(-A_mid, A_mid - A_last)
-// (log2 units).  M <= 12: Q^, K^ are fp16 (kind::f16); M <= 100: tf32 (fp32
+// (log2 units).  M <= 8: Q^, K^ are fp16 (kind::f16); M <= 100: tf32 (fp32
 // range, kind::tf32); larger (extreme decay, gamma -> 0) or non-finite gates: the
 // chunk's scores and log-decays are computed exactly by CUDA cores.  All other
 // operands carry factors <= 1 and are fp16; bf16 values become fp16 operands.
@@ -62,7 +66,7 @@ constexpr int kThreads = 448;
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kGateMinLog2 = -1.0e4f * 1.4426950408889634f;  // g < -1e4 acts as -1e4
-constexpr float kMaxRefF16 = 12.0f;       // fp16 score operands: factors within 2^{+-12}
+constexpr float kMaxRefF16 = 8.0f;        // fp16 score operands: factors within 2^{+-8}
 constexpr float kMaxRefTF32 = 100.0f;     // tf32 score operands: factors within 2^{+-100}
 
 enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
@@ -76,8 +80,8 @@ constexpr int kOffS = kOffOp + 2 * kOpBytes;                   // 2 x S_[c] (fp1
 constexpr int kOffO = kOffS + 2 * kTile16;                     // 2 x O staging
 constexpr int kOffL = kOffO + 2 * kTile16;                     // triangle of ones
 constexpr int kRefFloats = 5 * kD;                             // raw mid, raw last, mid*log2e, c1, c2
-constexpr int kOffRef = kOffL + kTile16;                       // 2 x kRefFloats
-constexpr int kOffDecay = kOffRef + 2 * kRefFloats * 4;        // kStages x 64 fp32
+constexpr int kOffRef = kOffL + kTile16;                       // kStages x kRefFloats
+constexpr int kOffDecay = kOffRef + kStages * kRefFloats * 4;  // kStages x 64 fp32
 constexpr int kOffMode = kOffDecay + kStages * kD * 4;         // kStages x u32, 2 x 2 maxima
 constexpr int kOffBar = kOffMode + 64;
 constexpr int kNumBars = 40;
@@ -91,7 +95,7 @@ enum {
     BAR_AFULL = BAR_EMPTY + kStages, // [2] MMA -> gen (A accumulator ready)
     BAR_TFREE_A = BAR_AFULL + 2,     // [2] gen -> MMA (A drained)
     BAR_OPND = BAR_TFREE_A + 2,      // [2] gen -> MMA (operands ready)
-    BAR_OPFREE = BAR_OPND + 2,       // [2] MMA (P done) -> gen (Q^/K^ buffer free)
+    BAR_OPFREE = BAR_OPND + 2,       // [2] MMA -> gen (Q^/K^ buffer free: after P, or after O in fp16 mode)
     BAR_PFULL = BAR_OPFREE + 2,      // [2] MMA -> epi-P
     BAR_UFULL = BAR_PFULL + 2,       // [2] MMA -> epi-P
     BAR_OFULL = BAR_UFULL + 2,       // [2] MMA -> epi-O (and epi-P: S buffer free)
@@ -317,13 +321,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         }
         fence_proxy_async_smem();
     }
-    if (warp >= 6 && warp < 10) {
-        // S_[0] = 0
-        const int te = threadIdx.x - 192;
-        for (int i = te; i < kTile16 / 16; i += 128)
-            reinterpret_cast<uint4 *>(smem + kOffS)[i] = make_uint4(0, 0, 0, 0);
-        fence_proxy_async_smem();
-    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -378,22 +375,24 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             int nA = 0, nPU = 0, nO = 0;
             bool ok = true;
             uint64_t t_idle = global_timer_ns();
-            uint32_t spins = 0;
+            uint32_t idle = 0;
             while (nO < N) {
                 bool did = false;
-                if (nO < nPU) {  // O(c) = Qtil S_[c] + P V
+                if (nO < nPU) {  // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V)
                     const int c = nO, s = c % kStages, bb = c & 1;
                     const uint32_t ph = (c >> 1) & 1;
                     if (mbar_test(&bars[BAR_PREADY + bb], ph) && mbar_test(&bars[BAR_SREADY + bb], ph) &&
                         mbar_test(&bars[BAR_TFREE_O + bb], ph ^ 1)) {
                         tc_fence_after();
+                        const uint32_t mode = mode_s[s];
                         const uint32_t st = sbase + kOffStage + s * kStageBytes;
-                        const uint32_t qt = st, vv = st + 2 * kTile16, pp = st + 3 * kTile16;
+                        const uint32_t qa = (mode == kModeF16) ? (sbase + kOffOp + bb * kOpBytes) : st;
+                        const uint32_t vv = st + 2 * kTile16, pp = st + 3 * kTile16;
                         const uint32_t ss = sbase + kOffS + bb * kTile16;
                         const uint32_t d = tmem + kColO + bb * 64;
 #pragma unroll
                         for (int ks = 0; ks < 4; ++ks)
-                            mma_f16_ss(d, smem_desc(qt + ks * 32, 16, 1024, kLayoutSw128),
+                            mma_f16_ss(d, smem_desc(qa + ks * 32, 16, 1024, kLayoutSw128),
                                        smem_desc(ss + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, ks > 0);
 #pragma unroll
                         for (int ks = 0; ks < 4; ++ks)
@@ -401,11 +400,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                        smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
                         mma_commit(&bars[BAR_OFULL + bb]);
                         mma_commit(&bars[BAR_EMPTY + s]);
+                        if (mode == kModeF16) mma_commit(&bars[BAR_OPFREE + bb]);  // Q^, K^ read by P, U, O
                         ++nO;
                         did = true;
                     }
                 }
-                if (!did && nPU < nA) {  // P(c) = Q^ K^^T and U(c) = Kbar^T V
+                if (!did && nPU < nA) {  // P(c) = Q^ K^^T and U(c) = Kbar^T V  (fp16 mode: K^^T V)
                     const int c = nPU, s = c % kStages, bb = c & 1;
                     const uint32_t ph = (c >> 1) & 1;
                     if (mbar_test(&bars[BAR_OPND + bb], ph) && mbar_test(&bars[BAR_TFREE_P + bb], ph ^ 1) &&
@@ -413,6 +413,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         tc_fence_after();
                         const uint32_t mode = mode_s[s];
                         const uint32_t qh = sbase + kOffOp + bb * kOpBytes, kh = qh + kTile32;
+                        const uint32_t st = sbase + kOffStage + s * kStageBytes;
                         if (mode == kModeTF32) {
 #pragma unroll
                             for (int ks = 0; ks < 8; ++ks) {
@@ -428,16 +429,16 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                 mma_f16_ss(tmem + kColP + bb * 64, smem_desc(qh + ks * 32, 16, 1024, kLayoutSw128),
                                            smem_desc(kh + ks * 32, 16, 1024, kLayoutSw128), idesc_p16, ks > 0);
                             mma_commit(&bars[BAR_PFULL + bb]);
-                            mma_commit(&bars[BAR_OPFREE + bb]);
                         } else {
                             mbar_arrive(&bars[BAR_PFULL + bb]);
                             mbar_arrive(&bars[BAR_OPFREE + bb]);
                         }
-                        const uint32_t st = sbase + kOffStage + s * kStageBytes;
-                        const uint32_t kb = st + 1 * kTile16, vv = st + 2 * kTile16;
+                        // K^ (K-major B of P) read as the MN-major A of U
+                        const uint32_t ka = (mode == kModeF16) ? kh : (st + kTile16);
+                        const uint32_t vv = st + 2 * kTile16;
 #pragma unroll
                         for (int ks = 0; ks < 4; ++ks)
-                            mma_f16_ss(tmem + kColU + bb * 64, smem_desc(kb + ks * 2048, 8192, 1024, kLayoutSw128),
+                            mma_f16_ss(tmem + kColU + bb * 64, smem_desc(ka + ks * 2048, 8192, 1024, kLayoutSw128),
                                        smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_u, ks > 0);
                         mma_commit(&bars[BAR_UFULL + bb]);
                         ++nPU;
@@ -461,10 +462,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     }
                 }
                 if (did) {
-                    spins = 0;
+                    idle = 0;
                     t_idle = global_timer_ns();
-                } else if ((++spins & 127u) == 0u) {
-                    if (*abort_flag || global_timer_ns() - t_idle > kWaitLimitNs) {
+                } else {
+                    // nothing ready: back off instead of spinning on the barriers
+                    if (++idle > 4) __nanosleep(64);
+                    if ((idle & 31u) == 0u && (*abort_flag || global_timer_ns() - t_idle > kWaitLimitNs)) {
                         ok = false;
                         break;
                     }
@@ -495,7 +498,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&ar[0]));
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&ar[16]));
             tmem_ld_wait();
-            float *ref = reinterpret_cast<float *>(smem + kOffRef) + bb * kRefFloats;
+            // per-stage references: [0,64) raw A_mid, [64,128) raw A_last, [128,192) A_mid log2,
+            // [192,256) c1 = 2^{A_mid}, [256,320) c2 = 2^{A_last - A_mid}
+            float *ref = reinterpret_cast<float *>(smem + kOffRef) + s * kRefFloats;
             if (row == rho_mid || row == rho_last) {
                 float *dst = ref + (row == rho_mid ? 0 : kD) + ch0;
 #pragma unroll
@@ -507,7 +512,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_A + bb]);
             named_barrier_sync(1, 128);
-            if (tg < kD) {  // per-channel references (log2 units) and split constants
+            if (tg < kD) {
                 const float am = ref[tg] * kLog2e, al = ref[kD + tg] * kLog2e;
                 float m = fmaxf(-am, am - al);
                 if (!(m <= 3.0e38f)) m = 3.0e38f;  // NaN / inf gates: exact path
@@ -535,13 +540,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     const int cl = ch0 + 8 * g8;
                     const float4 am0 = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl);
                     const float4 am1 = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl + 4);
-                    const float4 c10 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl);
-                    const float4 c11 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl + 4);
-                    const float4 c20 = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl);
-                    const float4 c21 = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl + 4);
                     const float amv[8] = {am0.x, am0.y, am0.z, am0.w, am1.x, am1.y, am1.z, am1.w};
-                    const float c1v[8] = {c10.x, c10.y, c10.z, c10.w, c11.x, c11.y, c11.z, c11.w};
-                    const float c2v[8] = {c20.x, c20.y, c20.z, c20.w, c21.x, c21.y, c21.z, c21.w};
                     const uint32_t o16 = sw128(row, cl * 2);
                     const uint4 qw = *reinterpret_cast<const uint4 *>(tq + o16);
                     const uint4 kw = *reinterpret_cast<const uint4 *>(tk + o16);
@@ -563,6 +562,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         *reinterpret_cast<uint4 *>(kh + o16) =
                             make_uint4(h2bits(ks[0], ks[1]), h2bits(ks[2], ks[3]), h2bits(ks[4], ks[5]), h2bits(ks[6], ks[7]));
                     } else {
+                        const float4 c10 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl);
+                        const float4 c11 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl + 4);
+                        const float4 c20 = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl);
+                        const float4 c21 = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl + 4);
+                        const float c1v[8] = {c10.x, c10.y, c10.z, c10.w, c11.x, c11.y, c11.z, c11.w};
+                        const float c2v[8] = {c20.x, c20.y, c20.z, c20.w, c21.x, c21.y, c21.z, c21.w};
                         *reinterpret_cast<float4 *>(qh + off32(row, cl)) =
                             make_float4(to_tf32(qs[0]), to_tf32(qs[1]), to_tf32(qs[2]), to_tf32(qs[3]));
                         *reinterpret_cast<float4 *>(qh + off32(row, cl + 4)) =
@@ -571,13 +576,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                             make_float4(to_tf32(ks[0]), to_tf32(ks[1]), to_tf32(ks[2]), to_tf32(ks[3]));
                         *reinterpret_cast<float4 *>(kh + off32(row, cl + 4)) =
                             make_float4(to_tf32(ks[4]), to_tf32(ks[5]), to_tf32(ks[6]), to_tf32(ks[7]));
+                        *reinterpret_cast<uint4 *>(tq + o16) =
+                            make_uint4(h2bits(qs[0] * c1v[0], qs[1] * c1v[1]), h2bits(qs[2] * c1v[2], qs[3] * c1v[3]),
+                                       h2bits(qs[4] * c1v[4], qs[5] * c1v[5]), h2bits(qs[6] * c1v[6], qs[7] * c1v[7]));
+                        *reinterpret_cast<uint4 *>(tk + o16) =
+                            make_uint4(h2bits(ks[0] * c2v[0], ks[1] * c2v[1]), h2bits(ks[2] * c2v[2], ks[3] * c2v[3]),
+                                       h2bits(ks[4] * c2v[4], ks[5] * c2v[5]), h2bits(ks[6] * c2v[6], ks[7] * c2v[7]));
                     }
-                    *reinterpret_cast<uint4 *>(tq + o16) =
-                        make_uint4(h2bits(qs[0] * c1v[0], qs[1] * c1v[1]), h2bits(qs[2] * c1v[2], qs[3] * c1v[3]),
-                                   h2bits(qs[4] * c1v[4], qs[5] * c1v[5]), h2bits(qs[6] * c1v[6], qs[7] * c1v[7]));
-                    *reinterpret_cast<uint4 *>(tk + o16) =
-                        make_uint4(h2bits(ks[0] * c2v[0], ks[1] * c2v[1]), h2bits(ks[2] * c2v[2], ks[3] * c2v[3]),
-                                   h2bits(ks[4] * c2v[4], ks[5] * c2v[5]), h2bits(ks[6] * c2v[6], ks[7] * c2v[7]));
                 }
             } else {
                 exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp + bb * kOpBytes),
@@ -608,7 +613,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const int row = 16 * q4 + (lane & 15);   // token rho for P, channel i for U / S
         const int ch0 = 32 * hc;
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
-        if (lane == 0) mbar_arrive(&bars[BAR_SREADY + 0]);  // S_[0] = 0 written before the CTA barrier
+        // causal mask of this thread's 32 P columns as packed fp16-pair masks (scan order)
+        uint32_t pm[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+            const int s0 = ch0 + 2 * e;
+            const bool k0 = rev ? (s0 >= row) : (s0 <= row);
+            const bool k1 = rev ? (s0 + 1 >= row) : (s0 + 1 <= row);
+            pm[e] = (k0 ? 0x0000FFFFu : 0u) | (k1 ? 0xFFFF0000u : 0u);
+        }
         float S[32];
 #pragma unroll
         for (int j = 0; j < 32; ++j) S[j] = 0.f;
@@ -618,7 +631,22 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             const uint32_t ph = (c >> 1) & 1;
             if (!mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs)) { ok = false; break; }
             const uint32_t mode = mode_s[s];
+            const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + s * kRefFloats;
+            const bool fold = (mode == kModeF16);
+            const float c1 = fold ? ref[3 * kD + row] : 1.f;
+            const float c2 = fold ? ref[4 * kD + row] : 1.f;
             const float dc = decay_s[s * kD + row];
+            // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout) into buffer bb,
+            // which O(c-2) read last
+            if (c >= 2 && !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs)) { ok = false; break; }
+            {
+                uint8_t *sb = smem + kOffS + bb * kTile16;
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    *reinterpret_cast<uint4 *>(sb + sw128(row, (ch0 + 8 * u) * 2)) =
+                        make_uint4(h2bits(S[8 * u + 0] * c1, S[8 * u + 1] * c1), h2bits(S[8 * u + 2] * c1, S[8 * u + 3] * c1),
+                                   h2bits(S[8 * u + 4] * c1, S[8 * u + 5] * c1), h2bits(S[8 * u + 6] * c1, S[8 * u + 7] * c1));
+            }
             if (mode != kModeExact) {
                 tc_fence_after();
                 uint32_t r[32];
@@ -627,18 +655,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 tmem_ld_wait();
                 uint8_t *pt = smem + kOffStage + s * kStageBytes + 3 * kTile16;
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    uint32_t w[4];
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int s0 = ch0 + 8 * u + 2 * e;
-                        const bool k0 = rev ? (s0 >= row) : (s0 <= row);
-                        const bool k1 = rev ? (s0 + 1 >= row) : (s0 + 1 <= row);
-                        w[e] = h2bits(k0 ? __uint_as_float(r[8 * u + 2 * e]) : 0.f,
-                                      k1 ? __uint_as_float(r[8 * u + 2 * e + 1]) : 0.f);
-                    }
-                    *reinterpret_cast<uint4 *>(pt + sw128(row, (ch0 + 8 * u) * 2)) = make_uint4(w[0], w[1], w[2], w[3]);
-                }
+                for (int u = 0; u < 4; ++u)
+                    *reinterpret_cast<uint4 *>(pt + sw128(row, (ch0 + 8 * u) * 2)) = make_uint4(
+                        h2bits(__uint_as_float(r[8 * u + 0]), __uint_as_float(r[8 * u + 1])) & pm[4 * u + 0],
+                        h2bits(__uint_as_float(r[8 * u + 2]), __uint_as_float(r[8 * u + 3])) & pm[4 * u + 1],
+                        h2bits(__uint_as_float(r[8 * u + 4]), __uint_as_float(r[8 * u + 5])) & pm[4 * u + 2],
+                        h2bits(__uint_as_float(r[8 * u + 6]), __uint_as_float(r[8 * u + 7])) & pm[4 * u + 3]);
             }
             tc_fence_before();
             fence_proxy_async_smem();
@@ -646,8 +668,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (lane == 0) {
                 mbar_arrive(&bars[BAR_TFREE_P + bb]);
                 mbar_arrive(&bars[BAR_PREADY + bb]);
+                mbar_arrive(&bars[BAR_SREADY + bb]);
             }
-            // state carry: S_[c+1] = Diag(d_c) S_[c] + U_c
+            // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
             if (!mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs)) { ok = false; break; }
             tc_fence_after();
             {
@@ -656,28 +679,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
 #pragma unroll
-                for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], __uint_as_float(r[j]));
+                for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_U + bb]);
-            if (c + 1 < N) {
-                const int nb = (c + 1) & 1;
-                // buffer nb was last read by O(c-1)
-                if (c >= 1 && !mbar_wait(&bars[BAR_OFULL + nb], ((c - 1) >> 1) & 1, abort_flag, kWaitLimitNs)) {
-                    ok = false;
-                    break;
-                }
-                uint8_t *sb = smem + kOffS + nb * kTile16;
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    *reinterpret_cast<uint4 *>(sb + sw128(row, (ch0 + 8 * u) * 2)) =
-                        make_uint4(h2bits(S[8 * u + 0], S[8 * u + 1]), h2bits(S[8 * u + 2], S[8 * u + 3]),
-                                   h2bits(S[8 * u + 4], S[8 * u + 5]), h2bits(S[8 * u + 6], S[8 * u + 7]));
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&bars[BAR_SREADY + nb]);
-            }
         }
         if (!ok) record_timeout(abort_flag);
         if (ok && p.final_state != nullptr) {
