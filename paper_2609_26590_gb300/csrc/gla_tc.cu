@@ -9,32 +9,34 @@
 // One CTA walks all chunks of one (b, h) sequence (single pass: q, k, v, g are
 // read once, o and S_final written once; S stays on chip between chunks).
 //
-// Per chunk, five tensor-core products (tcgen05.mma, fp32 accumulators in TMEM):
+// Per chunk, tensor-core products (tcgen05.mma, fp32 accumulators in TMEM):
 //   A = L G          in-chunk cumulative log-decay: L is the 64x64 triangle of
 //                    ones in scan order, G the gate tile as loaded (exact products)
 //   P = Q^ K^^T      intra-chunk scores with e^{A_r - A_j} split at the mid-chunk
 //                    reference: Q^ = q e^{A_r - A_mid}, K^ = k e^{A_mid - A_j}
 //   U = Kbar^T V     chunk summary, Kbar = k e^{A_last - A}
 //   O = Qtil S_[c] + P V   outputs, Qtil = q e^{A}
-// With fp16 score operands the per-channel constants c1 = e^{A_mid} and
-// c2 = e^{A_last - A_mid} are folded into the state instead of the tiles:
-// Qtil S = Q^ (Diag(c1) S) and Kbar^T V = Diag(c2) K^^T V, so Q^ and K^ serve
-// all four products and only the 64 x 64 state is rescaled per chunk.
 // The split factors of P lie within 2^{+-M}, M = max_i max(-A_mid, A_mid - A_last)
-// (log2 units).  M <= 8: Q^, K^ are fp16 (kind::f16); M <= 100: tf32 (fp32
-// range, kind::tf32); larger (extreme decay, gamma -> 0) or non-finite gates: the
-// chunk's scores and log-decays are computed exactly by CUDA cores.  All other
-// operands carry factors <= 1 and are fp16; bf16 values become fp16 operands.
+// (log2 units).  M <= 8 ("fp16 mode"): Q^, K^ are fp16 and serve all products,
+// because the per-channel constants c1 = e^{A_mid}, c2 = e^{A_last - A_mid} fold
+// into the state: Qtil S = Q^ (Diag(c1) S) and Kbar^T V = Diag(c2) K^^T V.
+// M <= 100 ("tf32 mode"): Q^, K^ are tf32 (fp32 range) for P, and Qtil, Kbar are
+// written as fp16 operands.  Larger M or non-finite gates ("exact mode"): the
+// chunk's log-decays and scores are computed exactly by CUDA cores.
 //
-// Warp roles (448 threads, one CTA per SM):
-//   warp 0       TMA producer: q, k, v, g tiles gathered in scan order (64-row
-//                boxes for row orders, 8-row boxes down a column for column
-//                orders); the scan permutation lives in the box coordinates.
-//   warp 1       TMEM allocator + single-thread MMA issuer (issues in data-flow
-//                order: whichever product has its inputs ready).
-//   warps 2-5    gen: reads A from TMEM, builds the decay-scaled operands.
-//   warps 6-9    epi-P: masks P into fp16, carries the fp32 state S in registers.
-//   warps 10-13  epi-O: converts O, TMA-stores it back in spatial order.
+// Memory pipeline: a q/k/g stage ring (freed as soon as the operands are built
+// in fp16 mode) and a separate v ring (freed after the output product).  Row
+// orders move one 64-row TMA box per tensor and chunk; column orders one box per
+// column segment of the chunk, of the segment's exact height (a tensor map per
+// height).  The scan permutation lives entirely in the box coordinates.
+//
+// Warp roles (576 threads, one CTA per SM):
+//   warp 0       TMA producer.
+//   warp 1       TMEM allocator + single-thread MMA issuer (data-flow order).
+//   warps 2-5    gen warpgroup 0 (even chunks)   reads A, builds the operands.
+//   warps 6-9    gen warpgroup 1 (odd chunks)
+//   warps 10-13  epi-P: masks P into fp16, carries the fp32 state S in registers.
+//   warps 14-17  epi-O: converts O, TMA-stores it back in spatial order.
 // A warp reads the TMEM lanes of sub-partition (warp % 4); an M = 64 accumulator
 // keeps rows 16q..16q+15 in lanes 32q..32q+15, and each thread takes one row and
 // 32 of its 64 columns.
@@ -43,6 +45,8 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
+#include <cstring>
+#include <list>
 #include <mutex>
 #include <type_traits>
 
@@ -59,10 +63,12 @@ using namespace ptx;
 
 constexpr int kC = 64;                    // chunk length
 constexpr int kD = 64;                    // Dk = Dv handled by this kernel
-constexpr int kStages = 3;                // input stage ring
+constexpr int kQS = 3;                    // q/k/g ring slots
+constexpr int kVS = 4;                    // v ring slots
 constexpr int kTile16 = kC * kD * 2;      // 64 x 64 16-bit tile (SW128, 128-byte rows)
 constexpr int kTile32 = kC * kD * 4;      // 64 x 64 fp32 tile (two 32-column K-blocks)
-constexpr int kThreads = 448;
+constexpr int kThreads = 576;
+constexpr int kHeights = 8;               // TMA box heights 8, 16, ..., 64
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kGateMinLog2 = -1.0e4f * 1.4426950408889634f;  // g < -1e4 acts as -1e4
@@ -72,39 +78,42 @@ constexpr float kMaxRefTF32 = 100.0f;     // tf32 score operands: factors within
 enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
 
 // Shared-memory map (byte offsets from a 1024-aligned base).
-constexpr int kStageBytes = 4 * kTile16;                       // q, k, v, g
-constexpr int kOffStage = 0;
-constexpr int kOffOp = kOffStage + kStages * kStageBytes;      // 2 x {Q^ | K^} (tf32 size)
-constexpr int kOpBytes = 2 * kTile32;
-constexpr int kOffS = kOffOp + 2 * kOpBytes;                   // 2 x S_[c] (fp16, MN-major)
+constexpr int kQkgBytes = 3 * kTile16;                         // q, k, g of one chunk
+constexpr int kOffQkg = 0;                                     // kQS slots
+constexpr int kOffV = kOffQkg + kQS * kQkgBytes;               // kVS slots
+constexpr int kOffOp = kOffV + kVS * kTile16;                  // 2 x 32 KB operand buffers
+constexpr int kOpBytes = 2 * kTile32;                          //  fp16: Q^ @0, P @8K, K^ @16K
+constexpr int kOffS = kOffOp + 2 * kOpBytes;                   //  tf32: Q^ @0, K^ @16K
 constexpr int kOffO = kOffS + 2 * kTile16;                     // 2 x O staging
 constexpr int kOffL = kOffO + 2 * kTile16;                     // triangle of ones
 constexpr int kRefFloats = 5 * kD;                             // raw mid, raw last, mid*log2e, c1, c2
-constexpr int kOffRef = kOffL + kTile16;                       // kStages x kRefFloats
-constexpr int kOffDecay = kOffRef + kStages * kRefFloats * 4;  // kStages x 64 fp32
-constexpr int kOffMode = kOffDecay + kStages * kD * 4;         // kStages x u32, 2 x 2 maxima
+constexpr int kOffRef = kOffL + kTile16;                       // 3 x kRefFloats (by chunk % 3)
+constexpr int kOffDecay = kOffRef + 3 * kRefFloats * 4;        // 3 x 64 fp32
+constexpr int kOffMode = kOffDecay + 3 * kD * 4;               // 3 x u32 mode, 2 x 2 fp32 maxima
 constexpr int kOffBar = kOffMode + 64;
-constexpr int kNumBars = 40;
+constexpr int kNumBars = 48;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;               // tmem base, abort flag
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;               // + alignment slack
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
 enum {
-    BAR_FULL = 0,                    // [kStages] TMA -> MMA/gen (tiles landed)
-    BAR_EMPTY = BAR_FULL + kStages,  // [kStages] MMA (O done) -> producer
-    BAR_AFULL = BAR_EMPTY + kStages, // [2] MMA -> gen (A accumulator ready)
-    BAR_TFREE_A = BAR_AFULL + 2,     // [2] gen -> MMA (A drained)
-    BAR_OPND = BAR_TFREE_A + 2,      // [2] gen -> MMA (operands ready)
-    BAR_OPFREE = BAR_OPND + 2,       // [2] MMA -> gen (Q^/K^ buffer free: after P, or after O in fp16 mode)
-    BAR_PFULL = BAR_OPFREE + 2,      // [2] MMA -> epi-P
-    BAR_UFULL = BAR_PFULL + 2,       // [2] MMA -> epi-P
-    BAR_OFULL = BAR_UFULL + 2,       // [2] MMA -> epi-O (and epi-P: S buffer free)
-    BAR_PREADY = BAR_OFULL + 2,      // [2] epi-P -> MMA (masked fp16 P in smem)
-    BAR_SREADY = BAR_PREADY + 2,     // [2] epi-P -> MMA (S_[c] fp16 in smem)
-    BAR_TFREE_P = BAR_SREADY + 2,    // [2] epi-P -> MMA
-    BAR_TFREE_U = BAR_TFREE_P + 2,   // [2] epi-P -> MMA
-    BAR_TFREE_O = BAR_TFREE_U + 2,   // [2] epi-O -> MMA
-    BAR_DONE = BAR_TFREE_O + 2,      // MMA: every issued MMA completed
+    BAR_QFULL = 0,                     // [kQS] TMA -> MMA/gen
+    BAR_QEMPTY = BAR_QFULL + kQS,      // [kQS] 4 arrivals: gen (fp16 mode) or MMA after O
+    BAR_VFULL = BAR_QEMPTY + kQS,      // [kVS] TMA -> gen
+    BAR_VEMPTY = BAR_VFULL + kVS,      // [kVS] MMA (O done) -> producer
+    BAR_AFULL = BAR_VEMPTY + kVS,      // [2] MMA -> gen (A accumulator ready)
+    BAR_TFREE_A = BAR_AFULL + 2,       // [2] gen -> MMA (A drained)
+    BAR_OPND = BAR_TFREE_A + 2,        // [2] gen -> MMA (operands ready)
+    BAR_OPFREE = BAR_OPND + 2,         // [2] MMA -> gen (operand buffer free)
+    BAR_PFULL = BAR_OPFREE + 2,        // [2] MMA -> epi-P
+    BAR_UFULL = BAR_PFULL + 2,         // [2] MMA -> epi-P
+    BAR_OFULL = BAR_UFULL + 2,         // [2] MMA -> epi-O (and epi-P: S buffer free)
+    BAR_PREADY = BAR_OFULL + 2,        // [2] epi-P -> MMA (masked fp16 P in smem)
+    BAR_SREADY = BAR_PREADY + 2,       // [2] epi-P -> MMA (S'_[c] fp16 in smem)
+    BAR_TFREE_P = BAR_SREADY + 2,      // [2] epi-P -> MMA
+    BAR_TFREE_U = BAR_TFREE_P + 2,     // [2] epi-P -> MMA
+    BAR_TFREE_O = BAR_TFREE_U + 2,     // [2] epi-O -> MMA
+    BAR_DONE = BAR_TFREE_O + 2,        // MMA: every issued MMA completed
     BAR_COUNT
 };
 static_assert(BAR_COUNT <= kNumBars, "barrier space");
@@ -112,12 +121,10 @@ static_assert(BAR_COUNT <= kNumBars, "barrier space");
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColA = 0, kColP = 128, kColU = 256, kColO = 384;
 
-struct TmaMaps {
-    CUtensorMap q, k, v, g, o, o8;  // o8: 8-row store boxes (row orders, ragged reversed chunk)
-};
+enum { T_Q = 0, T_K = 1, T_V = 2, T_G = 3, T_O = 4, kTensors = 5 };
 
 struct TcParams {
-    TmaMaps maps;
+    CUtensorMap maps[kTensors][kHeights];  // box height 8 (i + 1)
     float *final_state;
     int H, grid_h, grid_w, order, n_chunks, T;
 };
@@ -170,28 +177,44 @@ __device__ __forceinline__ void record_timeout(volatile uint32_t *abort_flag) {
     atomicOr(&g_device_status, kStatusTimeout);
 }
 
-// Scan positions 64c + 8grp .. +7 (smem rows 8grp .. 8grp+7) as 8-row box
-// coordinates.  Row orders address dims (D, H, T, 1, B), column orders
-// (D, H, W, Hg, B).  Reverse orders address the mirrored range, so smem row
-// rho holds scan position 64c + 63 - rho.  Returns false when the group lies
-// entirely outside the sequence (loads then read zero fill, stores are skipped).
-__device__ __forceinline__ bool group_coords(int order, int T, int grid_h, int c, int grp,
-                                             int &x2, int &x3) {
-    const int rev = order & 1;
-    const int u0 = rev ? (T - kC * (c + 1) + 8 * grp) : (kC * c + 8 * grp);
+// Smem row rho of chunk c holds walk position w0 + rho, where the walk is the
+// forward scan (row-major for row orders, down the columns for column orders)
+// and w0 mirrors the range for reverse orders (scan position 64c + 63 - rho).
+__device__ __forceinline__ int chunk_w0(int order, int T, int c) {
+    return (order & 1) ? (T - kC * (c + 1)) : kC * c;
+}
+
+// Visit the TMA boxes of one chunk: calls f(map height index, smem row, c2, c3)
+// for each box.  Row orders: one 64-row box at token w0 (rows outside the
+// sequence are zero-filled on loads; on stores the box is clipped past the end
+// and starts at token 0 when w0 < 0).  Column orders: one box per column
+// segment, of the segment's exact height; with `cover_invalid`, rows outside
+// the sequence get zero-fill boxes placed past the last column (loads only).
+// All heights and offsets are multiples of 8 (T and grid_h are).
+template <typename F>
+__device__ __forceinline__ void chunk_boxes(int order, int T, int grid_h, int grid_w, int c,
+                                            bool cover_invalid, F &&f) {
+    const int w0 = chunk_w0(order, T, c);
     if ((order >> 1) == 0) {
-        x2 = u0;
-        x3 = 0;
-        return u0 >= 0 && u0 < T;
+        if (cover_invalid || w0 >= 0) {
+            f(kHeights - 1, 0, w0, 0);
+        } else {
+            f((kC + w0) / 8 - 1, -w0, 0, 0);
+        }
+        return;
     }
-    if (u0 < 0 || u0 >= T) {
-        x2 = T / grid_h;  // one past the last column: zero fill
-        x3 = 0;
-        return false;
+    const int lo = w0 < 0 ? 0 : w0, hi = (w0 + kC > T) ? T : w0 + kC;
+    if (cover_invalid) {
+        if (lo > w0) f((lo - w0) / 8 - 1, 0, grid_w, 0);
+        if (hi < w0 + kC) f((w0 + kC - hi) / 8 - 1, hi - w0, grid_w, 0);
     }
-    x2 = u0 / grid_h;
-    x3 = u0 % grid_h;
-    return true;
+    for (int w = lo; w < hi;) {
+        const int x = w / grid_h, y = w - x * grid_h;
+        int len = grid_h - y;
+        if (len > hi - w) len = hi - w;
+        f(len / 8 - 1, w - w0, x, y);
+        w += len;
+    }
 }
 
 // Exact scores for one chunk (extreme or non-finite log-decays): serial prefix
@@ -199,7 +222,7 @@ __device__ __forceinline__ bool group_coords(int order, int T, int grid_h, int c
 // CUDA cores, Qtil = q 2^{a}, Kbar = k 2^{a_last - a}, and the chunk decay.
 template <typename E>
 __device__ __noinline__ void exact_chunk(uint8_t *tq, uint8_t *tk, uint8_t *tgate, float *as,
-                                         float *decay, int rev, int tg) {
+                                         float *decay, int rev, int tg, int bar_id) {
     if (tg < kD) {
         float run = 0.f;
         for (int r = 0; r < kC; ++r) {
@@ -212,7 +235,7 @@ __device__ __noinline__ void exact_chunk(uint8_t *tq, uint8_t *tk, uint8_t *tgat
         }
         decay[tg] = ex2(run);
     }
-    named_barrier_sync(1, 128);
+    named_barrier_sync(bar_id, 128);
     const int rho = tg >> 1, half = tg & 1;
     const int r = rev ? kC - 1 - rho : rho;
     uint32_t packed[16];
@@ -235,7 +258,7 @@ __device__ __noinline__ void exact_chunk(uint8_t *tq, uint8_t *tk, uint8_t *tgat
         packed[jj] = h2bits(pv[0], pv[1]);
     }
     const int rho_last = rev ? 0 : kC - 1;
-    named_barrier_sync(1, 128);  // every q/k/gate read of this chunk is done
+    named_barrier_sync(bar_id, 128);  // every q/k/gate read of this chunk is done
     for (int jj = 0; jj < 16; ++jj)
         *reinterpret_cast<uint32_t *>(tgate + sw128(rho, (half * 32 + 2 * jj) * 2)) = packed[jj];
     for (int i = half * 32; i < half * 32 + 32; i += 2) {
@@ -266,13 +289,16 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     const int b = bh / p.H, h = bh % p.H;
     const int N = p.n_chunks;
     const int rev = p.order & 1;
-    const bool col_order = (p.order >> 1) != 0;
 
     if (threadIdx.x == 0) {
         *abort_flag = 0u;
-        for (int i = 0; i < kStages; ++i) {
-            mbar_init(&bars[BAR_FULL + i], 1);
-            mbar_init(&bars[BAR_EMPTY + i], 1);
+        for (int i = 0; i < kQS; ++i) {
+            mbar_init(&bars[BAR_QFULL + i], 1);
+            mbar_init(&bars[BAR_QEMPTY + i], 4);
+        }
+        for (int i = 0; i < kVS; ++i) {
+            mbar_init(&bars[BAR_VFULL + i], 1);
+            mbar_init(&bars[BAR_VEMPTY + i], 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&bars[BAR_AFULL + i], 1);
@@ -294,13 +320,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     if (warp == 1) {
         tmem_alloc(const_cast<uint32_t *>(tmem_base_s), kTmemCols);
         tmem_relinquish();
-    }
-    if (warp == 0 && lane == 0) {
-        tma_prefetch_desc(&p.maps.q);
-        tma_prefetch_desc(&p.maps.k);
-        tma_prefetch_desc(&p.maps.v);
-        tma_prefetch_desc(&p.maps.g);
-        tma_prefetch_desc(&p.maps.o);
     }
     if (warp >= 2 && warp < 6) {
         // triangle of ones in scan order: L[rho][sigma] = 1 when sigma is at or before rho
@@ -329,38 +348,39 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     if (warp == 0) {
         // ======================================================= TMA producer
         if (lane == 0) {
-            int issued = 0;
+            int issued_q = 0, issued_v = 0;
             for (int c = 0; c < N; ++c) {
-                const int s = c % kStages;
-                if (!mbar_wait(&bars[BAR_EMPTY + s], ((c / kStages) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                const int sq = c % kQS, sv = c % kVS;
+                if (!mbar_wait(&bars[BAR_QEMPTY + sq], ((c / kQS) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
                     record_timeout(abort_flag);
                     break;
                 }
-                uint8_t *st = smem + kOffStage + s * kStageBytes;
-                uint64_t *fb = &bars[BAR_FULL + s];
-                mbar_arrive_expect_tx(fb, kStageBytes);
-                if (!col_order) {
-                    const int t0 = rev ? (p.T - kC * (c + 1)) : kC * c;
-                    tma_load_5d(st + 0 * kTile16, &p.maps.q, fb, 0, h, t0, 0, b);
-                    tma_load_5d(st + 1 * kTile16, &p.maps.k, fb, 0, h, t0, 0, b);
-                    tma_load_5d(st + 2 * kTile16, &p.maps.v, fb, 0, h, t0, 0, b);
-                    tma_load_5d(st + 3 * kTile16, &p.maps.g, fb, 0, h, t0, 0, b);
-                } else {
-                    for (int grp = 0; grp < 8; ++grp) {
-                        int x2, x3;
-                        group_coords(p.order, p.T, p.grid_h, c, grp, x2, x3);
-                        const uint32_t o = grp * 1024;
-                        tma_load_5d(st + 0 * kTile16 + o, &p.maps.q, fb, 0, h, x2, x3, b);
-                        tma_load_5d(st + 1 * kTile16 + o, &p.maps.k, fb, 0, h, x2, x3, b);
-                        tma_load_5d(st + 2 * kTile16 + o, &p.maps.v, fb, 0, h, x2, x3, b);
-                        tma_load_5d(st + 3 * kTile16 + o, &p.maps.g, fb, 0, h, x2, x3, b);
-                    }
+                uint8_t *qkg = smem + kOffQkg + sq * kQkgBytes;
+                uint64_t *fq = &bars[BAR_QFULL + sq];
+                mbar_arrive_expect_tx(fq, kQkgBytes);
+                chunk_boxes(p.order, p.T, p.grid_h, p.grid_w, c, true, [&](int hi, int row, int c2, int c3) {
+                    tma_load_5d(qkg + 0 * kTile16 + row * 128, &p.maps[T_Q][hi], fq, 0, h, c2, c3, b);
+                    tma_load_5d(qkg + 1 * kTile16 + row * 128, &p.maps[T_K][hi], fq, 0, h, c2, c3, b);
+                    tma_load_5d(qkg + 2 * kTile16 + row * 128, &p.maps[T_G][hi], fq, 0, h, c2, c3, b);
+                });
+                ++issued_q;
+                if (!mbar_wait(&bars[BAR_VEMPTY + sv], ((c / kVS) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                    record_timeout(abort_flag);
+                    break;
                 }
-                ++issued;
+                uint8_t *vt = smem + kOffV + sv * kTile16;
+                uint64_t *fv = &bars[BAR_VFULL + sv];
+                mbar_arrive_expect_tx(fv, kTile16);
+                chunk_boxes(p.order, p.T, p.grid_h, p.grid_w, c, true, [&](int hi, int row, int c2, int c3) {
+                    tma_load_5d(vt + row * 128, &p.maps[T_V][hi], fv, 0, h, c2, c3, b);
+                });
+                ++issued_v;
             }
             if (*abort_flag) {  // never leave while copies are still landing in shared memory
-                for (int c = (issued > kStages ? issued - kStages : 0); c < issued; ++c)
-                    mbar_wait(&bars[BAR_FULL + c % kStages], (c / kStages) & 1, nullptr, kWaitLimitNs);
+                for (int c = (issued_q > kQS ? issued_q - kQS : 0); c < issued_q; ++c)
+                    mbar_wait(&bars[BAR_QFULL + c % kQS], (c / kQS) & 1, nullptr, kWaitLimitNs);
+                for (int c = (issued_v > kVS ? issued_v - kVS : 0); c < issued_v; ++c)
+                    mbar_wait(&bars[BAR_VFULL + c % kVS], (c / kVS) & 1, nullptr, kWaitLimitNs);
             }
         }
     } else if (warp == 1) {
@@ -379,15 +399,17 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             while (nO < N) {
                 bool did = false;
                 if (nO < nPU) {  // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V)
-                    const int c = nO, s = c % kStages, bb = c & 1;
+                    const int c = nO, bb = c & 1;
                     const uint32_t ph = (c >> 1) & 1;
                     if (mbar_test(&bars[BAR_PREADY + bb], ph) && mbar_test(&bars[BAR_SREADY + bb], ph) &&
                         mbar_test(&bars[BAR_TFREE_O + bb], ph ^ 1)) {
                         tc_fence_after();
-                        const uint32_t mode = mode_s[s];
-                        const uint32_t st = sbase + kOffStage + s * kStageBytes;
-                        const uint32_t qa = (mode == kModeF16) ? (sbase + kOffOp + bb * kOpBytes) : st;
-                        const uint32_t vv = st + 2 * kTile16, pp = st + 3 * kTile16;
+                        const uint32_t mode = mode_s[c % 3];
+                        const uint32_t qkg = sbase + kOffQkg + (c % kQS) * kQkgBytes;
+                        const uint32_t op = sbase + kOffOp + bb * kOpBytes;
+                        const uint32_t qa = (mode == kModeF16) ? op : qkg;
+                        const uint32_t pp = (mode == kModeF16) ? op + kTile16 : qkg + 2 * kTile16;
+                        const uint32_t vv = sbase + kOffV + (c % kVS) * kTile16;
                         const uint32_t ss = sbase + kOffS + bb * kTile16;
                         const uint32_t d = tmem + kColO + bb * 64;
 #pragma unroll
@@ -399,21 +421,26 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                             mma_f16_ss(d, smem_desc(pp + ks * 32, 16, 1024, kLayoutSw128),
                                        smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
                         mma_commit(&bars[BAR_OFULL + bb]);
-                        mma_commit(&bars[BAR_EMPTY + s]);
-                        if (mode == kModeF16) mma_commit(&bars[BAR_OPFREE + bb]);  // Q^, K^ read by P, U, O
+                        mma_commit(&bars[BAR_VEMPTY + c % kVS]);
+                        if (mode == kModeF16) {
+                            mma_commit(&bars[BAR_OPFREE + bb]);  // Q^, K^, P read by P, U, O
+                        } else {
+                            // Qtil / Kbar / P lived in the q/k/g slot: four arrivals free it
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) mma_commit(&bars[BAR_QEMPTY + c % kQS]);
+                        }
                         ++nO;
                         did = true;
                     }
                 }
                 if (!did && nPU < nA) {  // P(c) = Q^ K^^T and U(c) = Kbar^T V  (fp16 mode: K^^T V)
-                    const int c = nPU, s = c % kStages, bb = c & 1;
+                    const int c = nPU, bb = c & 1;
                     const uint32_t ph = (c >> 1) & 1;
                     if (mbar_test(&bars[BAR_OPND + bb], ph) && mbar_test(&bars[BAR_TFREE_P + bb], ph ^ 1) &&
                         mbar_test(&bars[BAR_TFREE_U + bb], ph ^ 1)) {
                         tc_fence_after();
-                        const uint32_t mode = mode_s[s];
+                        const uint32_t mode = mode_s[c % 3];
                         const uint32_t qh = sbase + kOffOp + bb * kOpBytes, kh = qh + kTile32;
-                        const uint32_t st = sbase + kOffStage + s * kStageBytes;
                         if (mode == kModeTF32) {
 #pragma unroll
                             for (int ks = 0; ks < 8; ++ks) {
@@ -433,9 +460,10 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                             mbar_arrive(&bars[BAR_PFULL + bb]);
                             mbar_arrive(&bars[BAR_OPFREE + bb]);
                         }
-                        // K^ (K-major B of P) read as the MN-major A of U
-                        const uint32_t ka = (mode == kModeF16) ? kh : (st + kTile16);
-                        const uint32_t vv = st + 2 * kTile16;
+                        // K^ (K-major B of P) is read as the MN-major A of U in fp16 mode
+                        const uint32_t ka =
+                            (mode == kModeF16) ? kh : (sbase + kOffQkg + (c % kQS) * kQkgBytes + kTile16);
+                        const uint32_t vv = sbase + kOffV + (c % kVS) * kTile16;
 #pragma unroll
                         for (int ks = 0; ks < 4; ++ks)
                             mma_f16_ss(tmem + kColU + bb * 64, smem_desc(ka + ks * 2048, 8192, 1024, kLayoutSw128),
@@ -446,12 +474,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     }
                 }
                 if (!did && nA < N) {  // A(c) = L G
-                    const int c = nA, s = c % kStages, bb = c & 1;
-                    if (mbar_test(&bars[BAR_FULL + s], (c / kStages) & 1) &&
+                    const int c = nA, bb = c & 1;
+                    if (mbar_test(&bars[BAR_QFULL + c % kQS], (c / kQS) & 1) &&
                         mbar_test(&bars[BAR_TFREE_A + bb], ((c >> 1) & 1) ^ 1)) {
                         tc_fence_after();
                         const uint32_t L = sbase + kOffL;
-                        const uint32_t gt = sbase + kOffStage + s * kStageBytes + 3 * kTile16;
+                        const uint32_t gt = sbase + kOffQkg + (c % kQS) * kQkgBytes + 2 * kTile16;
 #pragma unroll
                         for (int ks = 0; ks < 4; ++ks)
                             mma_f16_ss(tmem + kColA + bb * 64, smem_desc(L + ks * 32, 16, 1024, kLayoutSw128),
@@ -466,7 +494,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     t_idle = global_timer_ns();
                 } else {
                     // nothing ready: back off instead of spinning on the barriers
-                    if (++idle > 4) __nanosleep(64);
+                    if (++idle > 4) __nanosleep(32);
                     if ((idle & 31u) == 0u && (*abort_flag || global_timer_ns() - t_idle > kWaitLimitNs)) {
                         ok = false;
                         break;
@@ -477,19 +505,22 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             mma_commit(&bars[BAR_DONE]);  // TMEM is released only after every MMA completed
             mbar_wait(&bars[BAR_DONE], 0, nullptr, kWaitLimitNs);
         }
-    } else if (warp < 6) {
-        // ======================================================= gen warpgroup
+    } else if (warp < 10) {
+        // ======================================================= gen warpgroups (chunks c = gw mod 2)
+        const int gw = (warp - 2) >> 2;          // 0: even chunks, 1: odd chunks
+        const int bar_id = 1 + gw;
         const int q4 = warp & 3, hc = lane >> 4;
         const int row = 16 * q4 + (lane & 15);   // smem row rho of this thread's accumulator row
         const int ch0 = 32 * hc;                 // its 32 key channels
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
-        const int tg = threadIdx.x - 64;
+        const int tg = threadIdx.x - 64 - 128 * gw;
         const int rho_mid = rev ? 32 : 31, rho_last = rev ? 0 : 63;
-        for (int c = 0; c < N; ++c) {
-            const int s = c % kStages, bb = c & 1;
+        for (int c = gw; c < N; c += 2) {
+            const int s3 = c % 3, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
             if (!mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs) ||
-                !mbar_wait(&bars[BAR_OPFREE + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
+                !mbar_wait(&bars[BAR_OPFREE + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
+                !mbar_wait(&bars[BAR_VFULL + c % kVS], (c / kVS) & 1, abort_flag, kWaitLimitNs)) {
                 record_timeout(abort_flag);
                 break;
             }
@@ -498,9 +529,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&ar[0]));
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&ar[16]));
             tmem_ld_wait();
-            // per-stage references: [0,64) raw A_mid, [64,128) raw A_last, [128,192) A_mid log2,
+            // references of chunk c: [0,64) raw A_mid, [64,128) raw A_last, [128,192) A_mid log2,
             // [192,256) c1 = 2^{A_mid}, [256,320) c2 = 2^{A_last - A_mid}
-            float *ref = reinterpret_cast<float *>(smem + kOffRef) + s * kRefFloats;
+            float *ref = reinterpret_cast<float *>(smem + kOffRef) + s3 * kRefFloats;
             if (row == rho_mid || row == rho_last) {
                 float *dst = ref + (row == rho_mid ? 0 : kD) + ch0;
 #pragma unroll
@@ -511,7 +542,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_A + bb]);
-            named_barrier_sync(1, 128);
+            named_barrier_sync(bar_id, 128);
             if (tg < kD) {
                 const float am = ref[tg] * kLog2e, al = ref[kD + tg] * kLog2e;
                 float m = fmaxf(-am, am - al);
@@ -519,7 +550,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 ref[2 * kD + tg] = am;
                 ref[3 * kD + tg] = ex2(am);
                 ref[4 * kD + tg] = ex2(al - am);
-                decay_s[s * kD + tg] = ex2(al);
+                decay_s[s3 * kD + tg] = ex2(al);
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 16));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 8));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 4));
@@ -527,12 +558,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
                 if (lane == 0) mx_s[bb * 2 + (tg >> 5)] = m;
             }
-            named_barrier_sync(1, 128);
+            named_barrier_sync(bar_id, 128);
             const float mmax = fmaxf(mx_s[bb * 2], mx_s[bb * 2 + 1]);
             const uint32_t mode = mmax <= kMaxRefF16 ? kModeF16 : (mmax <= kMaxRefTF32 ? kModeTF32 : kModeExact);
-            if (tg == 0) mode_s[s] = mode;
-            uint8_t *st = smem + kOffStage + s * kStageBytes;
-            uint8_t *tq = st, *tk = st + kTile16, *tv = st + 2 * kTile16, *tgt = st + 3 * kTile16;
+            if (tg == 0) mode_s[s3] = mode;
+            uint8_t *qkg = smem + kOffQkg + (c % kQS) * kQkgBytes;
+            uint8_t *tq = qkg, *tk = qkg + kTile16, *tgt = qkg + 2 * kTile16;
+            uint8_t *tv = smem + kOffV + (c % kVS) * kTile16;
             if (mode != kModeExact) {
                 uint8_t *qh = smem + kOffOp + bb * kOpBytes, *kh = qh + kTile32;
 #pragma unroll
@@ -586,7 +618,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
             } else {
                 exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp + bb * kOpBytes),
-                               decay_s + s * kD, rev, tg);
+                               decay_s + s3 * kD, rev, tg, bar_id);
             }
             if constexpr (std::is_same<E, __nv_bfloat16>::value) {
                 // bf16 values become fp16 MMA operands (exact for |v| in the fp16 normal range)
@@ -605,9 +637,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             }
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_OPND + bb]);
+            if (lane == 0) {
+                mbar_arrive(&bars[BAR_OPND + bb]);
+                // fp16 mode: q, k, g of this chunk are no longer read by anyone
+                if (mode == kModeF16) mbar_arrive(&bars[BAR_QEMPTY + c % kQS]);
+            }
         }
-    } else if (warp < 10) {
+    } else if (warp < 14) {
         // ======================================================= epi-P warpgroup
         const int q4 = warp & 3, hc = lane >> 4;
         const int row = 16 * q4 + (lane & 15);   // token rho for P, channel i for U / S
@@ -627,15 +663,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         for (int j = 0; j < 32; ++j) S[j] = 0.f;
         bool ok = true;
         for (int c = 0; c < N; ++c) {
-            const int s = c % kStages, bb = c & 1;
+            const int s3 = c % 3, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
             if (!mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs)) { ok = false; break; }
-            const uint32_t mode = mode_s[s];
-            const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + s * kRefFloats;
+            const uint32_t mode = mode_s[s3];
+            const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + s3 * kRefFloats;
             const bool fold = (mode == kModeF16);
             const float c1 = fold ? ref[3 * kD + row] : 1.f;
             const float c2 = fold ? ref[4 * kD + row] : 1.f;
-            const float dc = decay_s[s * kD + row];
+            const float dc = decay_s[s3 * kD + row];
             // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout) into buffer bb,
             // which O(c-2) read last
             if (c >= 2 && !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs)) { ok = false; break; }
@@ -653,7 +689,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColP + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColP + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
-                uint8_t *pt = smem + kOffStage + s * kStageBytes + 3 * kTile16;
+                uint8_t *pt = fold ? (smem + kOffOp + bb * kOpBytes + kTile16)
+                                   : (smem + kOffQkg + (c % kQS) * kQkgBytes + 2 * kTile16);
 #pragma unroll
                 for (int u = 0; u < 4; ++u)
                     *reinterpret_cast<uint4 *>(pt + sw128(row, (ch0 + 8 * u) * 2)) = make_uint4(
@@ -697,7 +734,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const int row = 16 * q4 + (lane & 15);
         const int ch0 = 32 * hc;
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
-        const bool elected = (warp == 10 && lane == 0);
+        const bool elected = (warp == 14 && lane == 0);
         bool ok = true;
         for (int c = 0; c < N; ++c) {
             const int bb = c & 1;
@@ -724,21 +761,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_O + bb]);
             named_barrier_sync(3, 128);
             if (elected) {
-                if (!col_order) {
-                    const int t0 = rev ? (p.T - kC * (c + 1)) : kC * c;
-                    if (t0 >= 0) {
-                        tma_store_5d(&p.maps.o, ob, 0, h, t0, 0, b);
-                    } else {  // ragged first-in-memory chunk of a reverse scan: 8-row boxes from t = 0
-                        for (int grp = 0; grp < 8; ++grp)
-                            if (t0 + 8 * grp >= 0) tma_store_5d(&p.maps.o8, ob + grp * 1024, 0, h, t0 + 8 * grp, 0, b);
-                    }
-                } else {
-                    for (int grp = 0; grp < 8; ++grp) {
-                        int x2, x3;
-                        if (group_coords(p.order, p.T, p.grid_h, c, grp, x2, x3))
-                            tma_store_5d(&p.maps.o, ob + grp * 1024, 0, h, x2, x3, b);
-                    }
-                }
+                chunk_boxes(p.order, p.T, p.grid_h, p.grid_w, c, false, [&](int hi, int rw, int c2, int c3) {
+                    tma_store_5d(&p.maps[T_O][hi], ob + rw * 128, 0, h, c2, c3, b);
+                });
                 tma_store_commit();
             }
         }
@@ -770,7 +795,7 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 }
 
 // Row orders: dims (D, H, T, 1, B), box (64, 1, rows, 1, 1).
-// Column orders: dims (D, H, W, Hg, B), box (64, 1, 1, 8, 1).
+// Column orders: dims (D, H, W, Hg, B), box (64, 1, 1, rows, 1).
 bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int rows) {
     auto enc = get_encode();
     if (!enc) return false;
@@ -788,7 +813,7 @@ bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int rows) {
         dims[2] = (cuuint64_t)p.grid_w;
         dims[3] = (cuuint64_t)p.grid_h;
         strides[2] = (cuuint64_t)p.grid_w * p.H * D * es;
-        box[3] = 8;
+        box[3] = (cuuint32_t)rows;
     }
     const CUtensorMapDataType dt = p.dtype == 1 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     return enc(m, dt, 5, const_cast<void *>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -796,25 +821,68 @@ bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int rows) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Encoded maps are cached per (pointers, shape, order, dtype): a repeated call
+// reuses them instead of encoding 40 maps again.
+struct MapKey {
+    const void *ptr[kTensors];
+    int B, H, grid_h, grid_w, order, dtype;
+    bool operator==(const MapKey &o) const { return std::memcmp(this, &o, sizeof(MapKey)) == 0; }
+};
+struct MapEntry {
+    MapKey key;
+    CUtensorMap maps[kTensors][kHeights];
+};
+std::mutex g_map_mutex;
+std::list<MapEntry> g_map_cache;  // most recent first
+constexpr size_t kMapCacheSize = 32;
+
+bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
+    MapKey key;
+    std::memset(&key, 0, sizeof(key));
+    key.ptr[T_Q] = p.q;
+    key.ptr[T_K] = p.k;
+    key.ptr[T_V] = p.v;
+    key.ptr[T_G] = p.g;
+    key.ptr[T_O] = p.out;
+    key.B = p.B;
+    key.H = p.H;
+    key.grid_h = p.grid_h;
+    key.grid_w = p.grid_w;
+    key.order = p.order;
+    key.dtype = p.dtype;
+    std::lock_guard<std::mutex> lock(g_map_mutex);
+    for (auto it = g_map_cache.begin(); it != g_map_cache.end(); ++it) {
+        if (it->key == key) {
+            std::memcpy(out, it->maps, sizeof(out));
+            g_map_cache.splice(g_map_cache.begin(), g_map_cache, it);
+            return true;
+        }
+    }
+    MapEntry e;
+    e.key = key;
+    for (int t = 0; t < kTensors; ++t)
+        for (int hi = 0; hi < kHeights; ++hi)
+            if (!encode_map(&e.maps[t][hi], key.ptr[t], p, 8 * (hi + 1))) return false;
+    std::memcpy(out, e.maps, sizeof(out));
+    g_map_cache.push_front(e);
+    if (g_map_cache.size() > kMapCacheSize) g_map_cache.pop_back();
+    return true;
+}
+
 }  // namespace
 
 bool tc_supported(const Problem &p) {
     if (p.dtype != 1 && p.dtype != 2) return false;       // fp16 / bf16 operands only
     if (p.Dk != kD || p.Dv != kD) return false;
-    if (p.T % 8 != 0) return false;                        // 8-row store boxes never straddle the end
-    if ((p.order >> 1) != 0 && p.grid_h % 8 != 0) return false;  // 8-row groups stay in one column
+    if (p.T % 8 != 0) return false;                        // box heights are multiples of 8
+    if ((p.order >> 1) != 0 && p.grid_h % 8 != 0) return false;  // column segments are too
     if (p.T > (1 << 30)) return false;
     return get_encode() != nullptr;
 }
 
 cudaError_t launch_tc(const Problem &p, cudaStream_t stream) {
     TcParams tp;
-    const bool col = (p.order >> 1) != 0;
-    const int rows = col ? 8 : 64;
-    if (!encode_map(&tp.maps.q, p.q, p, rows) || !encode_map(&tp.maps.k, p.k, p, rows) ||
-        !encode_map(&tp.maps.v, p.v, p, rows) || !encode_map(&tp.maps.g, p.g, p, rows) ||
-        !encode_map(&tp.maps.o, p.out, p, rows) || !encode_map(&tp.maps.o8, p.out, p, 8))
-        return cudaErrorInvalidValue;
+    if (!get_maps(p, tp.maps)) return cudaErrorInvalidValue;
     tp.final_state = p.final_state;
     tp.H = p.H;
     tp.grid_h = p.grid_h;
