@@ -30,12 +30,14 @@
 // column segment of the chunk, of the segment's exact height (a tensor map per
 // height).  The scan permutation lives entirely in the box coordinates.
 //
-// Warp roles (576 threads, one CTA per SM):
+// Warp roles (576 threads, one CTA per SM).  Each MMA is issued by one elected
+// thread of the role that produced its last operand, as soon as it is ready:
 //   warp 0       TMA producer.
-//   warp 1       TMEM allocator + single-thread MMA issuer (data-flow order).
-//   warps 2-5    gen warpgroup 0 (even chunks)   reads A, builds the operands.
-//   warps 6-9    gen warpgroup 1 (odd chunks)
-//   warps 10-13  epi-P: masks P into fp16, carries the fp32 state S in registers.
+//   warp 1       TMEM allocator; issues A = L G when a q/k/g stage lands.
+//   warps 2-5    gen warpgroup 0 (even chunks): reads A, builds the operands,
+//   warps 6-9    gen warpgroup 1 (odd chunks)    issues P and U.
+//   warps 10-13  epi-P: masks P into fp16, writes Diag(c1) S, issues O, carries
+//                the fp32 state S in registers.
 //   warps 14-17  epi-O: converts O, TMA-stores it back in spatial order.
 // A warp reads the TMEM lanes of sub-partition (warp % 4); an M = 64 accumulator
 // keeps rows 16q..16q+15 in lanes 32q..32q+15, and each thread takes one row and
@@ -97,24 +99,21 @@ constexpr int kSmemBytes = kOffMisc + 64 + 1024;               // + alignment sl
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
 enum {
-    BAR_QFULL = 0,                     // [kQS] TMA -> MMA/gen
-    BAR_QEMPTY = BAR_QFULL + kQS,      // [kQS] 4 arrivals: gen (fp16 mode) or MMA after O
+    BAR_QFULL = 0,                     // [kQS] TMA -> A issuer / gen
+    BAR_QEMPTY = BAR_QFULL + kQS,      // [kQS] gen (fp16 mode) or O issuer -> producer
     BAR_VFULL = BAR_QEMPTY + kQS,      // [kVS] TMA -> gen
-    BAR_VEMPTY = BAR_VFULL + kVS,      // [kVS] MMA (O done) -> producer
-    BAR_AFULL = BAR_VEMPTY + kVS,      // [2] MMA -> gen (A accumulator ready)
-    BAR_TFREE_A = BAR_AFULL + 2,       // [2] gen -> MMA (A drained)
-    BAR_OPND = BAR_TFREE_A + 2,        // [2] gen -> MMA (operands ready)
-    BAR_OPFREE = BAR_OPND + 2,         // [2] MMA -> gen (operand buffer free)
-    BAR_PFULL = BAR_OPFREE + 2,        // [2] MMA -> epi-P
-    BAR_UFULL = BAR_PFULL + 2,         // [2] MMA -> epi-P
-    BAR_OFULL = BAR_UFULL + 2,         // [2] MMA -> epi-O (and epi-P: S buffer free)
-    BAR_PREADY = BAR_OFULL + 2,        // [2] epi-P -> MMA (masked fp16 P in smem)
-    BAR_SREADY = BAR_PREADY + 2,       // [2] epi-P -> MMA (S'_[c] fp16 in smem)
-    BAR_TFREE_P = BAR_SREADY + 2,      // [2] epi-P -> MMA
-    BAR_TFREE_U = BAR_TFREE_P + 2,     // [2] epi-P -> MMA
-    BAR_TFREE_O = BAR_TFREE_U + 2,     // [2] epi-O -> MMA
-    BAR_DONE = BAR_TFREE_O + 2,        // MMA: every issued MMA completed
-    BAR_COUNT
+    BAR_VEMPTY = BAR_VFULL + kVS,      // [kVS] O done -> producer
+    BAR_AFULL = BAR_VEMPTY + kVS,      // [2] A done -> gen
+    BAR_TFREE_A = BAR_AFULL + 2,       // [2] gen drained A -> A issuer
+    BAR_OPFREE = BAR_TFREE_A + 2,      // [2] operand buffer free (after P, or after O in fp16 mode)
+    BAR_PFULL = BAR_OPFREE + 2,        // [2] P done -> epi-P
+    BAR_UFULL = BAR_PFULL + 2,         // [2] U done -> epi-P
+    BAR_OFULL = BAR_UFULL + 2,         // [2] O done -> epi-O (and epi-P: S buffer free)
+    BAR_TFREE_P = BAR_OFULL + 2,       // [2] epi-P drained P -> gen (P issuer)
+    BAR_TFREE_U = BAR_TFREE_P + 2,     // [2] epi-P drained U -> gen (U issuer)
+    BAR_TFREE_O = BAR_TFREE_U + 2,     // [2] epi-O drained O -> epi-P (O issuer)
+    BAR_DONE = BAR_TFREE_O + 2,        // [4] per issuing thread: its MMAs completed
+    BAR_COUNT = BAR_DONE + 4
 };
 static_assert(BAR_COUNT <= kNumBars, "barrier space");
 
@@ -294,7 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         *abort_flag = 0u;
         for (int i = 0; i < kQS; ++i) {
             mbar_init(&bars[BAR_QFULL + i], 1);
-            mbar_init(&bars[BAR_QEMPTY + i], 4);
+            mbar_init(&bars[BAR_QEMPTY + i], 1);
         }
         for (int i = 0; i < kVS; ++i) {
             mbar_init(&bars[BAR_VFULL + i], 1);
@@ -303,18 +302,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         for (int i = 0; i < 2; ++i) {
             mbar_init(&bars[BAR_AFULL + i], 1);
             mbar_init(&bars[BAR_TFREE_A + i], 4);
-            mbar_init(&bars[BAR_OPND + i], 4);
             mbar_init(&bars[BAR_OPFREE + i], 1);
             mbar_init(&bars[BAR_PFULL + i], 1);
             mbar_init(&bars[BAR_UFULL + i], 1);
             mbar_init(&bars[BAR_OFULL + i], 1);
-            mbar_init(&bars[BAR_PREADY + i], 4);
-            mbar_init(&bars[BAR_SREADY + i], 4);
             mbar_init(&bars[BAR_TFREE_P + i], 4);
             mbar_init(&bars[BAR_TFREE_U + i], 4);
             mbar_init(&bars[BAR_TFREE_O + i], 4);
         }
-        mbar_init(&bars[BAR_DONE], 1);
+        for (int i = 0; i < 4; ++i) mbar_init(&bars[BAR_DONE + i], 1);
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -384,126 +380,27 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             }
         }
     } else if (warp == 1) {
-        // ======================================================= MMA issuer (data-flow order)
+        // ======================================================= A issuer: A(c) = L G
         if (lane == 0) {
             const uint32_t idesc_a = instr_desc(Elem<E>::fmt, 64, 64, 0, 1);
-            const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
-            const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
-            const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
-            const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
-            const uint32_t sbase = smem_u32(smem);
-            int nA = 0, nPU = 0, nO = 0;
-            bool ok = true;
-            uint64_t t_idle = global_timer_ns();
-            uint32_t idle = 0;
-            while (nO < N) {
-                bool did = false;
-                if (nO < nPU) {  // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V)
-                    const int c = nO, bb = c & 1;
-                    const uint32_t ph = (c >> 1) & 1;
-                    if (mbar_test(&bars[BAR_PREADY + bb], ph) && mbar_test(&bars[BAR_SREADY + bb], ph) &&
-                        mbar_test(&bars[BAR_TFREE_O + bb], ph ^ 1)) {
-                        tc_fence_after();
-                        const uint32_t mode = mode_s[c % 3];
-                        const uint32_t qkg = sbase + kOffQkg + (c % kQS) * kQkgBytes;
-                        const uint32_t op = sbase + kOffOp + bb * kOpBytes;
-                        const uint32_t qa = (mode == kModeF16) ? op : qkg;
-                        const uint32_t pp = (mode == kModeF16) ? op + kTile16 : qkg + 2 * kTile16;
-                        const uint32_t vv = sbase + kOffV + (c % kVS) * kTile16;
-                        const uint32_t ss = sbase + kOffS + bb * kTile16;
-                        const uint32_t d = tmem + kColO + bb * 64;
-#pragma unroll
-                        for (int ks = 0; ks < 4; ++ks)
-                            mma_f16_ss(d, smem_desc(qa + ks * 32, 16, 1024, kLayoutSw128),
-                                       smem_desc(ss + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, ks > 0);
-#pragma unroll
-                        for (int ks = 0; ks < 4; ++ks)
-                            mma_f16_ss(d, smem_desc(pp + ks * 32, 16, 1024, kLayoutSw128),
-                                       smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
-                        mma_commit(&bars[BAR_OFULL + bb]);
-                        mma_commit(&bars[BAR_VEMPTY + c % kVS]);
-                        if (mode == kModeF16) {
-                            mma_commit(&bars[BAR_OPFREE + bb]);  // Q^, K^, P read by P, U, O
-                        } else {
-                            // Qtil / Kbar / P lived in the q/k/g slot: four arrivals free it
-#pragma unroll
-                            for (int i = 0; i < 4; ++i) mma_commit(&bars[BAR_QEMPTY + c % kQS]);
-                        }
-                        ++nO;
-                        did = true;
-                    }
+            const uint32_t L = smem_u32(smem + kOffL);
+            for (int c = 0; c < N; ++c) {
+                const int bb = c & 1;
+                if (!mbar_wait(&bars[BAR_QFULL + c % kQS], (c / kQS) & 1, abort_flag, kWaitLimitNs) ||
+                    !mbar_wait(&bars[BAR_TFREE_A + bb], ((c >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                    record_timeout(abort_flag);
+                    break;
                 }
-                if (!did && nPU < nA) {  // P(c) = Q^ K^^T and U(c) = Kbar^T V  (fp16 mode: K^^T V)
-                    const int c = nPU, bb = c & 1;
-                    const uint32_t ph = (c >> 1) & 1;
-                    if (mbar_test(&bars[BAR_OPND + bb], ph) && mbar_test(&bars[BAR_TFREE_P + bb], ph ^ 1) &&
-                        mbar_test(&bars[BAR_TFREE_U + bb], ph ^ 1)) {
-                        tc_fence_after();
-                        const uint32_t mode = mode_s[c % 3];
-                        const uint32_t qh = sbase + kOffOp + bb * kOpBytes, kh = qh + kTile32;
-                        if (mode == kModeTF32) {
+                tc_fence_after();
+                const uint32_t gt = smem_u32(smem + kOffQkg + (c % kQS) * kQkgBytes + 2 * kTile16);
 #pragma unroll
-                            for (int ks = 0; ks < 8; ++ks) {
-                                const uint32_t o = (ks >> 2) * 8192 + (ks & 3) * 32;
-                                mma_tf32_ss(tmem + kColP + bb * 64, smem_desc(qh + o, 16, 1024, kLayoutSw128),
-                                            smem_desc(kh + o, 16, 1024, kLayoutSw128), idesc_p32, ks > 0);
-                            }
-                            mma_commit(&bars[BAR_PFULL + bb]);
-                            mma_commit(&bars[BAR_OPFREE + bb]);
-                        } else if (mode == kModeF16) {
-#pragma unroll
-                            for (int ks = 0; ks < 4; ++ks)
-                                mma_f16_ss(tmem + kColP + bb * 64, smem_desc(qh + ks * 32, 16, 1024, kLayoutSw128),
-                                           smem_desc(kh + ks * 32, 16, 1024, kLayoutSw128), idesc_p16, ks > 0);
-                            mma_commit(&bars[BAR_PFULL + bb]);
-                        } else {
-                            mbar_arrive(&bars[BAR_PFULL + bb]);
-                            mbar_arrive(&bars[BAR_OPFREE + bb]);
-                        }
-                        // K^ (K-major B of P) is read as the MN-major A of U in fp16 mode
-                        const uint32_t ka =
-                            (mode == kModeF16) ? kh : (sbase + kOffQkg + (c % kQS) * kQkgBytes + kTile16);
-                        const uint32_t vv = sbase + kOffV + (c % kVS) * kTile16;
-#pragma unroll
-                        for (int ks = 0; ks < 4; ++ks)
-                            mma_f16_ss(tmem + kColU + bb * 64, smem_desc(ka + ks * 2048, 8192, 1024, kLayoutSw128),
-                                       smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_u, ks > 0);
-                        mma_commit(&bars[BAR_UFULL + bb]);
-                        ++nPU;
-                        did = true;
-                    }
-                }
-                if (!did && nA < N) {  // A(c) = L G
-                    const int c = nA, bb = c & 1;
-                    if (mbar_test(&bars[BAR_QFULL + c % kQS], (c / kQS) & 1) &&
-                        mbar_test(&bars[BAR_TFREE_A + bb], ((c >> 1) & 1) ^ 1)) {
-                        tc_fence_after();
-                        const uint32_t L = sbase + kOffL;
-                        const uint32_t gt = sbase + kOffQkg + (c % kQS) * kQkgBytes + 2 * kTile16;
-#pragma unroll
-                        for (int ks = 0; ks < 4; ++ks)
-                            mma_f16_ss(tmem + kColA + bb * 64, smem_desc(L + ks * 32, 16, 1024, kLayoutSw128),
-                                       smem_desc(gt + ks * 2048, 8192, 1024, kLayoutSw128), idesc_a, ks > 0);
-                        mma_commit(&bars[BAR_AFULL + bb]);
-                        ++nA;
-                        did = true;
-                    }
-                }
-                if (did) {
-                    idle = 0;
-                    t_idle = global_timer_ns();
-                } else {
-                    // nothing ready: back off instead of spinning on the barriers
-                    if (++idle > 4) __nanosleep(32);
-                    if ((idle & 31u) == 0u && (*abort_flag || global_timer_ns() - t_idle > kWaitLimitNs)) {
-                        ok = false;
-                        break;
-                    }
-                }
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_f16_ss(tmem + kColA + bb * 64, smem_desc(L + ks * 32, 16, 1024, kLayoutSw128),
+                               smem_desc(gt + ks * 2048, 8192, 1024, kLayoutSw128), idesc_a, ks > 0);
+                mma_commit(&bars[BAR_AFULL + bb]);
             }
-            if (!ok) record_timeout(abort_flag);
-            mma_commit(&bars[BAR_DONE]);  // TMEM is released only after every MMA completed
-            mbar_wait(&bars[BAR_DONE], 0, nullptr, kWaitLimitNs);
+            mma_commit(&bars[BAR_DONE + 0]);  // TMEM is released only after these MMAs completed
+            mbar_wait(&bars[BAR_DONE + 0], 0, nullptr, kWaitLimitNs);
         }
     } else if (warp < 10) {
         // ======================================================= gen warpgroups (chunks c = gw mod 2)
@@ -515,15 +412,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
         const int tg = threadIdx.x - 64 - 128 * gw;
         const int rho_mid = rev ? 32 : 31, rho_last = rev ? 0 : 63;
+        const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
+        const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
+        const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
         for (int c = gw; c < N; c += 2) {
             const int s3 = c % 3, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
-            if (!mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs) ||
-                !mbar_wait(&bars[BAR_OPFREE + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
-                !mbar_wait(&bars[BAR_VFULL + c % kVS], (c / kVS) & 1, abort_flag, kWaitLimitNs)) {
-                record_timeout(abort_flag);
-                break;
-            }
+            const bool fail = !mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs) ||
+                              !mbar_wait(&bars[BAR_OPFREE + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
+                              !mbar_wait(&bars[BAR_VFULL + c % kVS], (c / kVS) & 1, abort_flag, kWaitLimitNs);
             tc_fence_after();
             uint32_t ar[32];
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&ar[0]));
@@ -532,7 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             // references of chunk c: [0,64) raw A_mid, [64,128) raw A_last, [128,192) A_mid log2,
             // [192,256) c1 = 2^{A_mid}, [256,320) c2 = 2^{A_last - A_mid}
             float *ref = reinterpret_cast<float *>(smem + kOffRef) + s3 * kRefFloats;
-            if (row == rho_mid || row == rho_last) {
+            if (!fail && (row == rho_mid || row == rho_last)) {
                 float *dst = ref + (row == rho_mid ? 0 : kD) + ch0;
 #pragma unroll
                 for (int u = 0; u < 8; ++u)
@@ -540,9 +437,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                                                      __uint_as_float(ar[4 * u + 2]), __uint_as_float(ar[4 * u + 3]));
             }
             tc_fence_before();
+            if (named_barrier_or(bar_id, 128, fail || *abort_flag != 0u)) {  // the whole warpgroup gives up together
+                record_timeout(abort_flag);
+                break;
+            }
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_A + bb]);
-            named_barrier_sync(bar_id, 128);
             if (tg < kD) {
                 const float am = ref[tg] * kLog2e, al = ref[kD + tg] * kLog2e;
                 float m = fmaxf(-am, am - al);
@@ -636,12 +536,50 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
             }
             fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&bars[BAR_OPND + bb]);
+            named_barrier_sync(bar_id, 128);  // every operand of chunk c is in shared memory
+            if (tg == 0) {
                 // fp16 mode: q, k, g of this chunk are no longer read by anyone
                 if (mode == kModeF16) mbar_arrive(&bars[BAR_QEMPTY + c % kQS]);
+                if (!mbar_wait(&bars[BAR_TFREE_P + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
+                    !mbar_wait(&bars[BAR_TFREE_U + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
+                    record_timeout(abort_flag);
+                } else {
+                    tc_fence_after();
+                    // P(c) = Q^ K^^T
+                    const uint32_t qh = smem_u32(smem + kOffOp + bb * kOpBytes), kh = qh + kTile32;
+                    if (mode == kModeTF32) {
+#pragma unroll
+                        for (int ks = 0; ks < 8; ++ks) {
+                            const uint32_t o = (ks >> 2) * 8192 + (ks & 3) * 32;
+                            mma_tf32_ss(tmem + kColP + bb * 64, smem_desc(qh + o, 16, 1024, kLayoutSw128),
+                                        smem_desc(kh + o, 16, 1024, kLayoutSw128), idesc_p32, ks > 0);
+                        }
+                        mma_commit(&bars[BAR_PFULL + bb]);
+                        mma_commit(&bars[BAR_OPFREE + bb]);
+                    } else if (mode == kModeF16) {
+#pragma unroll
+                        for (int ks = 0; ks < 4; ++ks)
+                            mma_f16_ss(tmem + kColP + bb * 64, smem_desc(qh + ks * 32, 16, 1024, kLayoutSw128),
+                                       smem_desc(kh + ks * 32, 16, 1024, kLayoutSw128), idesc_p16, ks > 0);
+                        mma_commit(&bars[BAR_PFULL + bb]);
+                    } else {
+                        mbar_arrive(&bars[BAR_PFULL + bb]);
+                        mbar_arrive(&bars[BAR_OPFREE + bb]);
+                    }
+                    // U(c) = Kbar^T V; in fp16 mode K^ (K-major B of P) is read as the MN-major A
+                    const uint32_t ka = (mode == kModeF16) ? kh : smem_u32(tk);
+                    const uint32_t vv = smem_u32(tv);
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_f16_ss(tmem + kColU + bb * 64, smem_desc(ka + ks * 2048, 8192, 1024, kLayoutSw128),
+                                   smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_u, ks > 0);
+                    mma_commit(&bars[BAR_UFULL + bb]);
+                }
             }
+        }
+        if (tg == 0) {
+            mma_commit(&bars[BAR_DONE + 1 + gw]);
+            mbar_wait(&bars[BAR_DONE + 1 + gw], 0, nullptr, kWaitLimitNs);
         }
     } else if (warp < 14) {
         // ======================================================= epi-P warpgroup
@@ -649,6 +587,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const int row = 16 * q4 + (lane & 15);   // token rho for P, channel i for U / S
         const int ch0 = 32 * hc;
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
+        const bool elected = (warp == 10 && lane == 0);
+        const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
         // causal mask of this thread's 32 P columns as packed fp16-pair masks (scan order)
         uint32_t pm[16];
 #pragma unroll
@@ -661,20 +601,24 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         float S[32];
 #pragma unroll
         for (int j = 0; j < 32; ++j) S[j] = 0.f;
-        bool ok = true;
+        bool ok = true, fail = false;
         for (int c = 0; c < N; ++c) {
             const int s3 = c % 3, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
-            if (!mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs)) { ok = false; break; }
+            fail = fail || !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
+            // S'_[c] goes to buffer bb, which O(c-2) read last
+            if (c >= 2) fail = fail || !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs);
+            if (named_barrier_or(4, 128, fail || *abort_flag != 0u)) {  // the whole warpgroup gives up together
+                ok = false;
+                break;
+            }
             const uint32_t mode = mode_s[s3];
             const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + s3 * kRefFloats;
             const bool fold = (mode == kModeF16);
             const float c1 = fold ? ref[3 * kD + row] : 1.f;
             const float c2 = fold ? ref[4 * kD + row] : 1.f;
             const float dc = decay_s[s3 * kD + row];
-            // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout) into buffer bb,
-            // which O(c-2) read last
-            if (c >= 2 && !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs)) { ok = false; break; }
+            // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout)
             {
                 uint8_t *sb = smem + kOffS + bb * kTile16;
 #pragma unroll
@@ -702,13 +646,38 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tc_fence_before();
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&bars[BAR_TFREE_P + bb]);
-                mbar_arrive(&bars[BAR_PREADY + bb]);
-                mbar_arrive(&bars[BAR_SREADY + bb]);
+            if (lane == 0) mbar_arrive(&bars[BAR_TFREE_P + bb]);
+            named_barrier_sync(4, 128);  // masked P and S'_[c] of every thread are in shared memory
+            if (elected) {
+                // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V)
+                if (!mbar_wait(&bars[BAR_TFREE_O + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
+                    fail = true;  // stops the group at the next chunk's barrier
+                } else {
+                    tc_fence_after();
+                    const uint32_t qkg = smem_u32(smem + kOffQkg + (c % kQS) * kQkgBytes);
+                    const uint32_t op = smem_u32(smem + kOffOp + bb * kOpBytes);
+                    const uint32_t qa = fold ? op : qkg;
+                    const uint32_t pp = fold ? op + kTile16 : qkg + 2 * kTile16;
+                    const uint32_t vv = smem_u32(smem + kOffV + (c % kVS) * kTile16);
+                    const uint32_t ss = smem_u32(smem + kOffS + bb * kTile16);
+                    const uint32_t d = tmem + kColO + bb * 64;
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_f16_ss(d, smem_desc(qa + ks * 32, 16, 1024, kLayoutSw128),
+                                   smem_desc(ss + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, ks > 0);
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_f16_ss(d, smem_desc(pp + ks * 32, 16, 1024, kLayoutSw128),
+                                   smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
+                    mma_commit(&bars[BAR_OFULL + bb]);
+                    mma_commit(&bars[BAR_VEMPTY + c % kVS]);
+                    // fp16 mode: Q^, K^, P lived in the operand buffer; otherwise Qtil, Kbar, P
+                    // lived in the q/k/g slot
+                    mma_commit(fold ? &bars[BAR_OPFREE + bb] : &bars[BAR_QEMPTY + c % kQS]);
+                }
             }
             // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
-            if (!mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs)) { ok = false; break; }
+            fail = fail || !mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs);
             tc_fence_after();
             {
                 uint32_t r[32];
@@ -722,8 +691,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_U + bb]);
         }
-        if (!ok) record_timeout(abort_flag);
-        if (ok && p.final_state != nullptr) {
+        if (!ok || fail) record_timeout(abort_flag);
+        if (elected) {
+            mma_commit(&bars[BAR_DONE + 3]);
+            mbar_wait(&bars[BAR_DONE + 3], 0, nullptr, kWaitLimitNs);
+        }
+        if (ok && !fail && p.final_state != nullptr) {
             float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)bh * kD + row) * kD + ch0);
 #pragma unroll
             for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
@@ -739,9 +712,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         for (int c = 0; c < N; ++c) {
             const int bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
-            if (!mbar_wait(&bars[BAR_OFULL + bb], ph, abort_flag, kWaitLimitNs)) { ok = false; break; }
+            const bool fail = !mbar_wait(&bars[BAR_OFULL + bb], ph, abort_flag, kWaitLimitNs);
             if (elected) tma_store_wait_read<1>();
-            named_barrier_sync(3, 128);
+            if (named_barrier_or(3, 128, fail || *abort_flag != 0u)) {  // the whole warpgroup gives up together
+                ok = false;
+                break;
+            }
             tc_fence_after();
             uint32_t r[32];
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
