@@ -24,21 +24,25 @@
 // written as fp16 operands.  Larger M or non-finite gates ("exact mode"): the
 // chunk's log-decays and scores are computed exactly by CUDA cores.
 //
-// Memory pipeline: a q/k/g stage ring (freed as soon as the operands are built
-// in fp16 mode) and a separate v ring (freed after the output product).  Row
-// orders move one 64-row TMA box per tensor and chunk; column orders one box per
-// column segment of the chunk, of the segment's exact height (a tensor map per
-// height).  The scan permutation lives entirely in the box coordinates.
+// Memory: each chunk owns a 32 KB stage slot (q, k, v, g tiles) from its TMA
+// load until its output product completes; the derived fp16 operands are
+// written in place (Q^ or Qtil over q, K^ or Kbar over k, the masked scores P
+// over g, bf16 v converted to fp16 in place), so five chunks can be in flight.
+// Only the tf32 score operands use a separate buffer, freed as soon as P is
+// done.  Row orders load one 64-row TMA box per tensor and chunk; column orders
+// one box per column segment of the chunk, of the segment's exact height (a
+// tensor map per height).  The scan permutation lives in the box coordinates of
+// the loads and in the addresses of the output stores.
 //
 // Warp roles (576 threads, one CTA per SM).  Each MMA is issued by one elected
 // thread of the role that produced its last operand, as soon as it is ready:
 //   warp 0       TMA producer.
-//   warp 1       TMEM allocator; issues A = L G when a q/k/g stage lands.
+//   warp 1       TMEM allocator; issues A = L G when a stage lands.
 //   warps 2-5    gen warpgroup 0 (even chunks): reads A, builds the operands,
 //   warps 6-9    gen warpgroup 1 (odd chunks)    issues P and U.
 //   warps 10-13  epi-P: masks P into fp16, writes Diag(c1) S, issues O, carries
 //                the fp32 state S in registers.
-//   warps 14-17  epi-O: converts O, TMA-stores it back in spatial order.
+//   warps 14-17  epi-O: converts O and stores it at the tokens' spatial positions.
 // A warp reads the TMEM lanes of sub-partition (warp % 4); an M = 64 accumulator
 // keeps rows 16q..16q+15 in lanes 32q..32q+15, and each thread takes one row and
 // 32 of its 64 columns.
@@ -65,8 +69,7 @@ using namespace ptx;
 
 constexpr int kC = 64;                    // chunk length
 constexpr int kD = 64;                    // Dk = Dv handled by this kernel
-constexpr int kQS = 3;                    // q/k/g ring slots
-constexpr int kVS = 4;                    // v ring slots
+constexpr int kSlots = 5;                 // stage slots (chunks in flight)
 constexpr int kTile16 = kC * kD * 2;      // 64 x 64 16-bit tile (SW128, 128-byte rows)
 constexpr int kTile32 = kC * kD * 4;      // 64 x 64 fp32 tile (two 32-column K-blocks)
 constexpr int kThreads = 576;
@@ -80,33 +83,29 @@ constexpr float kMaxRefTF32 = 100.0f;     // tf32 score operands: factors within
 enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
 
 // Shared-memory map (byte offsets from a 1024-aligned base).
-constexpr int kQkgBytes = 3 * kTile16;                         // q, k, g of one chunk
-constexpr int kOffQkg = 0;                                     // kQS slots
-constexpr int kOffV = kOffQkg + kQS * kQkgBytes;               // kVS slots
-constexpr int kOffOp = kOffV + kVS * kTile16;                  // 2 x 32 KB operand buffers
-constexpr int kOpBytes = 2 * kTile32;                          //  fp16: Q^ @0, P @8K, K^ @16K
-constexpr int kOffS = kOffOp + 2 * kOpBytes;                   //  tf32: Q^ @0, K^ @16K
-constexpr int kOffO = kOffS + 2 * kTile16;                     // 2 x O staging
-constexpr int kOffL = kOffO + 2 * kTile16;                     // triangle of ones
+constexpr int kSlotBytes = 4 * kTile16;                        // q @0, k @8K, v @16K, g @24K
+constexpr int kQ = 0, kK = kTile16, kV = 2 * kTile16, kG = 3 * kTile16;
+constexpr int kOffSlot = 0;
+constexpr int kOffOp = kOffSlot + kSlots * kSlotBytes;         // tf32 Q^ @0, K^ @16K
+constexpr int kOffS = kOffOp + 2 * kTile32;                    // 2 x S'_[c] (fp16, MN-major)
+constexpr int kOffL = kOffS + 2 * kTile16;                     // triangle of ones
 constexpr int kRefFloats = 5 * kD;                             // raw mid, raw last, mid*log2e, c1, c2
-constexpr int kOffRef = kOffL + kTile16;                       // 3 x kRefFloats (by chunk % 3)
-constexpr int kOffDecay = kOffRef + 3 * kRefFloats * 4;        // 3 x 64 fp32
-constexpr int kOffMode = kOffDecay + 3 * kD * 4;               // 3 x u32 mode, 2 x 2 fp32 maxima
+constexpr int kOffRef = kOffL + kTile16;                       // per slot
+constexpr int kOffDecay = kOffRef + kSlots * kRefFloats * 4;   // per slot, 64 fp32
+constexpr int kOffMode = kOffDecay + kSlots * kD * 4;          // per slot u32 mode; 2 x 2 fp32 maxima
 constexpr int kOffBar = kOffMode + 64;
-constexpr int kNumBars = 48;
+constexpr int kNumBars = 40;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;               // tmem base, abort flag
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;               // + alignment slack
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
 enum {
-    BAR_QFULL = 0,                     // [kQS] TMA -> A issuer / gen
-    BAR_QEMPTY = BAR_QFULL + kQS,      // [kQS] gen (fp16 mode) or O issuer -> producer
-    BAR_VFULL = BAR_QEMPTY + kQS,      // [kVS] TMA -> gen
-    BAR_VEMPTY = BAR_VFULL + kVS,      // [kVS] O done -> producer
-    BAR_AFULL = BAR_VEMPTY + kVS,      // [2] A done -> gen
+    BAR_FULL = 0,                      // [kSlots] TMA -> A issuer / gen
+    BAR_EMPTY = BAR_FULL + kSlots,     // [kSlots] U and O done -> producer (two commits)
+    BAR_AFULL = BAR_EMPTY + kSlots,    // [2] A done -> gen
     BAR_TFREE_A = BAR_AFULL + 2,       // [2] gen drained A -> A issuer
-    BAR_OPFREE = BAR_TFREE_A + 2,      // [2] operand buffer free (after P, or after O in fp16 mode)
-    BAR_PFULL = BAR_OPFREE + 2,        // [2] P done -> epi-P
+    BAR_OPFREE = BAR_TFREE_A + 2,      // tf32 operand buffer released (once per chunk)
+    BAR_PFULL = BAR_OPFREE + 1,        // [2] P done -> epi-P
     BAR_UFULL = BAR_PFULL + 2,         // [2] U done -> epi-P
     BAR_OFULL = BAR_UFULL + 2,         // [2] O done -> epi-O (and epi-P: S buffer free)
     BAR_TFREE_P = BAR_OFULL + 2,       // [2] epi-P drained P -> gen (P issuer)
@@ -120,10 +119,11 @@ static_assert(BAR_COUNT <= kNumBars, "barrier space");
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColA = 0, kColP = 128, kColU = 256, kColO = 384;
 
-enum { T_Q = 0, T_K = 1, T_V = 2, T_G = 3, T_O = 4, kTensors = 5 };
+enum { T_Q = 0, T_K = 1, T_V = 2, T_G = 3, kTensors = 4 };
 
 struct TcParams {
     CUtensorMap maps[kTensors][kHeights];  // box height 8 (i + 1)
+    void *out;
     float *final_state;
     int H, grid_h, grid_w, order, n_chunks, T;
 };
@@ -183,30 +183,21 @@ __device__ __forceinline__ int chunk_w0(int order, int T, int c) {
     return (order & 1) ? (T - kC * (c + 1)) : kC * c;
 }
 
-// Visit the TMA boxes of one chunk: calls f(map height index, smem row, c2, c3)
-// for each box.  Row orders: one 64-row box at token w0 (rows outside the
-// sequence are zero-filled on loads; on stores the box is clipped past the end
-// and starts at token 0 when w0 < 0).  Column orders: one box per column
-// segment, of the segment's exact height; with `cover_invalid`, rows outside
-// the sequence get zero-fill boxes placed past the last column (loads only).
-// All heights and offsets are multiples of 8 (T and grid_h are).
+// Visit the TMA load boxes of one chunk: calls f(map height index, smem row, c2, c3).
+// Row orders: one 64-row box at token w0 (rows outside the sequence are
+// zero-filled).  Column orders: one box per column segment, of the segment's
+// exact height, plus zero-fill boxes placed past the last column for rows
+// outside the sequence.  Heights and offsets are multiples of 8 (T and grid_h are).
 template <typename F>
-__device__ __forceinline__ void chunk_boxes(int order, int T, int grid_h, int grid_w, int c,
-                                            bool cover_invalid, F &&f) {
+__device__ __forceinline__ void chunk_load_boxes(int order, int T, int grid_h, int grid_w, int c, F &&f) {
     const int w0 = chunk_w0(order, T, c);
     if ((order >> 1) == 0) {
-        if (cover_invalid || w0 >= 0) {
-            f(kHeights - 1, 0, w0, 0);
-        } else {
-            f((kC + w0) / 8 - 1, -w0, 0, 0);
-        }
+        f(kHeights - 1, 0, w0, 0);
         return;
     }
     const int lo = w0 < 0 ? 0 : w0, hi = (w0 + kC > T) ? T : w0 + kC;
-    if (cover_invalid) {
-        if (lo > w0) f((lo - w0) / 8 - 1, 0, grid_w, 0);
-        if (hi < w0 + kC) f((w0 + kC - hi) / 8 - 1, hi - w0, grid_w, 0);
-    }
+    if (lo > w0) f((lo - w0) / 8 - 1, 0, grid_w, 0);
+    if (hi < w0 + kC) f((w0 + kC - hi) / 8 - 1, hi - w0, grid_w, 0);
     for (int w = lo; w < hi;) {
         const int x = w / grid_h, y = w - x * grid_h;
         int len = grid_h - y;
@@ -214,6 +205,14 @@ __device__ __forceinline__ void chunk_boxes(int order, int T, int grid_h, int gr
         f(len / 8 - 1, w - w0, x, y);
         w += len;
     }
+}
+
+// Spatial token of walk position w (-1 outside the sequence).
+__device__ __forceinline__ int walk_token(int order, int T, int grid_h, int grid_w, int w) {
+    if (w < 0 || w >= T) return -1;
+    if ((order >> 1) == 0) return w;
+    const int x = w / grid_h;
+    return (w - x * grid_h) * grid_w + x;
 }
 
 // Exact scores for one chunk (extreme or non-finite log-decays): serial prefix
@@ -281,7 +280,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     volatile uint32_t *abort_flag = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc + 4);
     float *decay_s = reinterpret_cast<float *>(smem + kOffDecay);
     volatile uint32_t *mode_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMode);
-    float *mx_s = reinterpret_cast<float *>(smem + kOffMode + 16);   // [2][2] partial maxima
+    float *mx_s = reinterpret_cast<float *>(smem + kOffMode + 32);   // [2][2] partial maxima
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int bh = blockIdx.x;
@@ -291,18 +290,14 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 
     if (threadIdx.x == 0) {
         *abort_flag = 0u;
-        for (int i = 0; i < kQS; ++i) {
-            mbar_init(&bars[BAR_QFULL + i], 1);
-            mbar_init(&bars[BAR_QEMPTY + i], 1);
+        for (int i = 0; i < kSlots; ++i) {
+            mbar_init(&bars[BAR_FULL + i], 1);
+            mbar_init(&bars[BAR_EMPTY + i], 2);  // U(c) and O(c) both done (issued by two threads)
         }
-        for (int i = 0; i < kVS; ++i) {
-            mbar_init(&bars[BAR_VFULL + i], 1);
-            mbar_init(&bars[BAR_VEMPTY + i], 1);
-        }
+        mbar_init(&bars[BAR_OPFREE], 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&bars[BAR_AFULL + i], 1);
             mbar_init(&bars[BAR_TFREE_A + i], 4);
-            mbar_init(&bars[BAR_OPFREE + i], 1);
             mbar_init(&bars[BAR_PFULL + i], 1);
             mbar_init(&bars[BAR_UFULL + i], 1);
             mbar_init(&bars[BAR_OFULL + i], 1);
@@ -344,39 +339,27 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     if (warp == 0) {
         // ======================================================= TMA producer
         if (lane == 0) {
-            int issued_q = 0, issued_v = 0;
+            int issued = 0;
             for (int c = 0; c < N; ++c) {
-                const int sq = c % kQS, sv = c % kVS;
-                if (!mbar_wait(&bars[BAR_QEMPTY + sq], ((c / kQS) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                const int sl = c % kSlots;
+                if (!mbar_wait(&bars[BAR_EMPTY + sl], ((c / kSlots) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
                     record_timeout(abort_flag);
                     break;
                 }
-                uint8_t *qkg = smem + kOffQkg + sq * kQkgBytes;
-                uint64_t *fq = &bars[BAR_QFULL + sq];
-                mbar_arrive_expect_tx(fq, kQkgBytes);
-                chunk_boxes(p.order, p.T, p.grid_h, p.grid_w, c, true, [&](int hi, int row, int c2, int c3) {
-                    tma_load_5d(qkg + 0 * kTile16 + row * 128, &p.maps[T_Q][hi], fq, 0, h, c2, c3, b);
-                    tma_load_5d(qkg + 1 * kTile16 + row * 128, &p.maps[T_K][hi], fq, 0, h, c2, c3, b);
-                    tma_load_5d(qkg + 2 * kTile16 + row * 128, &p.maps[T_G][hi], fq, 0, h, c2, c3, b);
+                uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
+                uint64_t *fb = &bars[BAR_FULL + sl];
+                mbar_arrive_expect_tx(fb, kSlotBytes);
+                chunk_load_boxes(p.order, p.T, p.grid_h, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
+                    tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, 0, h, c2, c3, b);
+                    tma_load_5d(st + kK + row * 128, &p.maps[T_K][hi], fb, 0, h, c2, c3, b);
+                    tma_load_5d(st + kV + row * 128, &p.maps[T_V][hi], fb, 0, h, c2, c3, b);
+                    tma_load_5d(st + kG + row * 128, &p.maps[T_G][hi], fb, 0, h, c2, c3, b);
                 });
-                ++issued_q;
-                if (!mbar_wait(&bars[BAR_VEMPTY + sv], ((c / kVS) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
-                    record_timeout(abort_flag);
-                    break;
-                }
-                uint8_t *vt = smem + kOffV + sv * kTile16;
-                uint64_t *fv = &bars[BAR_VFULL + sv];
-                mbar_arrive_expect_tx(fv, kTile16);
-                chunk_boxes(p.order, p.T, p.grid_h, p.grid_w, c, true, [&](int hi, int row, int c2, int c3) {
-                    tma_load_5d(vt + row * 128, &p.maps[T_V][hi], fv, 0, h, c2, c3, b);
-                });
-                ++issued_v;
+                ++issued;
             }
             if (*abort_flag) {  // never leave while copies are still landing in shared memory
-                for (int c = (issued_q > kQS ? issued_q - kQS : 0); c < issued_q; ++c)
-                    mbar_wait(&bars[BAR_QFULL + c % kQS], (c / kQS) & 1, nullptr, kWaitLimitNs);
-                for (int c = (issued_v > kVS ? issued_v - kVS : 0); c < issued_v; ++c)
-                    mbar_wait(&bars[BAR_VFULL + c % kVS], (c / kVS) & 1, nullptr, kWaitLimitNs);
+                for (int c = (issued > kSlots ? issued - kSlots : 0); c < issued; ++c)
+                    mbar_wait(&bars[BAR_FULL + c % kSlots], (c / kSlots) & 1, nullptr, kWaitLimitNs);
             }
         }
     } else if (warp == 1) {
@@ -386,13 +369,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             const uint32_t L = smem_u32(smem + kOffL);
             for (int c = 0; c < N; ++c) {
                 const int bb = c & 1;
-                if (!mbar_wait(&bars[BAR_QFULL + c % kQS], (c / kQS) & 1, abort_flag, kWaitLimitNs) ||
+                if (!mbar_wait(&bars[BAR_FULL + c % kSlots], (c / kSlots) & 1, abort_flag, kWaitLimitNs) ||
                     !mbar_wait(&bars[BAR_TFREE_A + bb], ((c >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
                     record_timeout(abort_flag);
                     break;
                 }
                 tc_fence_after();
-                const uint32_t gt = smem_u32(smem + kOffQkg + (c % kQS) * kQkgBytes + 2 * kTile16);
+                const uint32_t gt = smem_u32(smem + kOffSlot + (c % kSlots) * kSlotBytes + kG);
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
                     mma_f16_ss(tmem + kColA + bb * 64, smem_desc(L + ks * 32, 16, 1024, kLayoutSw128),
@@ -416,11 +399,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
         const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
         for (int c = gw; c < N; c += 2) {
-            const int s3 = c % 3, bb = c & 1;
+            const int sl = c % kSlots, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
-            const bool fail = !mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs) ||
-                              !mbar_wait(&bars[BAR_OPFREE + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
-                              !mbar_wait(&bars[BAR_VFULL + c % kVS], (c / kVS) & 1, abort_flag, kWaitLimitNs);
+            const bool fail = !mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs);
             tc_fence_after();
             uint32_t ar[32];
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&ar[0]));
@@ -428,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tmem_ld_wait();
             // references of chunk c: [0,64) raw A_mid, [64,128) raw A_last, [128,192) A_mid log2,
             // [192,256) c1 = 2^{A_mid}, [256,320) c2 = 2^{A_last - A_mid}
-            float *ref = reinterpret_cast<float *>(smem + kOffRef) + s3 * kRefFloats;
+            float *ref = reinterpret_cast<float *>(smem + kOffRef) + sl * kRefFloats;
             if (!fail && (row == rho_mid || row == rho_last)) {
                 float *dst = ref + (row == rho_mid ? 0 : kD) + ch0;
 #pragma unroll
@@ -437,7 +418,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                                                      __uint_as_float(ar[4 * u + 2]), __uint_as_float(ar[4 * u + 3]));
             }
             tc_fence_before();
-            if (named_barrier_or(bar_id, 128, fail || *abort_flag != 0u)) {  // the whole warpgroup gives up together
+            if (named_barrier_or(bar_id, 128, fail || *abort_flag != 0u)) {  // the group gives up together
                 record_timeout(abort_flag);
                 break;
             }
@@ -450,23 +431,28 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 ref[2 * kD + tg] = am;
                 ref[3 * kD + tg] = ex2(am);
                 ref[4 * kD + tg] = ex2(al - am);
-                decay_s[s3 * kD + tg] = ex2(al);
+                decay_s[sl * kD + tg] = ex2(al);
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 16));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 8));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 4));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
-                if (lane == 0) mx_s[bb * 2 + (tg >> 5)] = m;
+                if (lane == 0) mx_s[gw * 2 + (tg >> 5)] = m;
             }
             named_barrier_sync(bar_id, 128);
-            const float mmax = fmaxf(mx_s[bb * 2], mx_s[bb * 2 + 1]);
+            const float mmax = fmaxf(mx_s[gw * 2], mx_s[gw * 2 + 1]);
             const uint32_t mode = mmax <= kMaxRefF16 ? kModeF16 : (mmax <= kMaxRefTF32 ? kModeTF32 : kModeExact);
-            if (tg == 0) mode_s[s3] = mode;
-            uint8_t *qkg = smem + kOffQkg + (c % kQS) * kQkgBytes;
-            uint8_t *tq = qkg, *tk = qkg + kTile16, *tgt = qkg + 2 * kTile16;
-            uint8_t *tv = smem + kOffV + (c % kVS) * kTile16;
+            if (tg == 0) mode_s[sl] = mode;
+            uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
+            uint8_t *tq = st + kQ, *tk = st + kK, *tv = st + kV, *tgt = st + kG;
+            bool opfail = false;
+            if (mode != kModeF16) {
+                // the tf32 / scratch buffer is shared by consecutive chunks: wait for the previous
+                // release; the decision is uniform because the exact path has named barriers
+                opfail = named_barrier_or(bar_id, 128, !mbar_wait(&bars[BAR_OPFREE], (c & 1) ^ 1, abort_flag, kWaitLimitNs));
+            }
             if (mode != kModeExact) {
-                uint8_t *qh = smem + kOffOp + bb * kOpBytes, *kh = qh + kTile32;
+                uint8_t *qh = smem + kOffOp, *kh = qh + kTile32;
 #pragma unroll
                 for (int g8 = 0; g8 < 4; ++g8) {
                     const int cl = ch0 + 8 * g8;
@@ -489,11 +475,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         ks[2 * e + 1] = k2.y * ex2(-e1);
                     }
                     if (mode == kModeF16) {
-                        *reinterpret_cast<uint4 *>(qh + o16) =
+                        // Q^ over q, K^ over k (each thread rewrites exactly what it read)
+                        *reinterpret_cast<uint4 *>(tq + o16) =
                             make_uint4(h2bits(qs[0], qs[1]), h2bits(qs[2], qs[3]), h2bits(qs[4], qs[5]), h2bits(qs[6], qs[7]));
-                        *reinterpret_cast<uint4 *>(kh + o16) =
+                        *reinterpret_cast<uint4 *>(tk + o16) =
                             make_uint4(h2bits(ks[0], ks[1]), h2bits(ks[2], ks[3]), h2bits(ks[4], ks[5]), h2bits(ks[6], ks[7]));
-                    } else {
+                    } else if (!opfail) {
                         const float4 c10 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl);
                         const float4 c11 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl + 4);
                         const float4 c20 = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl);
@@ -508,6 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                             make_float4(to_tf32(ks[0]), to_tf32(ks[1]), to_tf32(ks[2]), to_tf32(ks[3]));
                         *reinterpret_cast<float4 *>(kh + off32(row, cl + 4)) =
                             make_float4(to_tf32(ks[4]), to_tf32(ks[5]), to_tf32(ks[6]), to_tf32(ks[7]));
+                        // Qtil over q, Kbar over k
                         *reinterpret_cast<uint4 *>(tq + o16) =
                             make_uint4(h2bits(qs[0] * c1v[0], qs[1] * c1v[1]), h2bits(qs[2] * c1v[2], qs[3] * c1v[3]),
                                        h2bits(qs[4] * c1v[4], qs[5] * c1v[5]), h2bits(qs[6] * c1v[6], qs[7] * c1v[7]));
@@ -516,9 +504,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                        h2bits(ks[4] * c2v[4], ks[5] * c2v[5]), h2bits(ks[6] * c2v[6], ks[7] * c2v[7]));
                     }
                 }
-            } else {
-                exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp + bb * kOpBytes),
-                               decay_s + s3 * kD, rev, tg, bar_id);
+            } else if (!opfail) {
+                exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp), decay_s + sl * kD, rev, tg,
+                               bar_id);
             }
             if constexpr (std::is_same<E, __nv_bfloat16>::value) {
                 // bf16 values become fp16 MMA operands (exact for |v| in the fp16 normal range)
@@ -536,18 +524,26 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
             }
             fence_proxy_async_smem();
-            named_barrier_sync(bar_id, 128);  // every operand of chunk c is in shared memory
+            if (named_barrier_or(bar_id, 128, opfail)) {  // every operand of chunk c is in shared memory
+                record_timeout(abort_flag);
+                break;
+            }
             if (tg == 0) {
-                // fp16 mode: q, k, g of this chunk are no longer read by anyone
-                if (mode == kModeF16) mbar_arrive(&bars[BAR_QEMPTY + c % kQS]);
+                if (mode == kModeF16) {
+                    // pass the shared tf32 buffer on: this chunk does not use it
+                    if (!mbar_wait(&bars[BAR_OPFREE], (c & 1) ^ 1, abort_flag, kWaitLimitNs)) record_timeout(abort_flag);
+                    mbar_arrive(&bars[BAR_OPFREE]);
+                } else if (mode == kModeExact) {
+                    mbar_arrive(&bars[BAR_OPFREE]);  // the exact path's scratch use is over
+                }
                 if (!mbar_wait(&bars[BAR_TFREE_P + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
                     !mbar_wait(&bars[BAR_TFREE_U + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
                     record_timeout(abort_flag);
                 } else {
                     tc_fence_after();
                     // P(c) = Q^ K^^T
-                    const uint32_t qh = smem_u32(smem + kOffOp + bb * kOpBytes), kh = qh + kTile32;
                     if (mode == kModeTF32) {
+                        const uint32_t qh = smem_u32(smem + kOffOp), kh = qh + kTile32;
 #pragma unroll
                         for (int ks = 0; ks < 8; ++ks) {
                             const uint32_t o = (ks >> 2) * 8192 + (ks & 3) * 32;
@@ -555,8 +551,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                         smem_desc(kh + o, 16, 1024, kLayoutSw128), idesc_p32, ks > 0);
                         }
                         mma_commit(&bars[BAR_PFULL + bb]);
-                        mma_commit(&bars[BAR_OPFREE + bb]);
+                        mma_commit(&bars[BAR_OPFREE]);
                     } else if (mode == kModeF16) {
+                        const uint32_t qh = smem_u32(tq), kh = smem_u32(tk);
 #pragma unroll
                         for (int ks = 0; ks < 4; ++ks)
                             mma_f16_ss(tmem + kColP + bb * 64, smem_desc(qh + ks * 32, 16, 1024, kLayoutSw128),
@@ -564,16 +561,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         mma_commit(&bars[BAR_PFULL + bb]);
                     } else {
                         mbar_arrive(&bars[BAR_PFULL + bb]);
-                        mbar_arrive(&bars[BAR_OPFREE + bb]);
                     }
-                    // U(c) = Kbar^T V; in fp16 mode K^ (K-major B of P) is read as the MN-major A
-                    const uint32_t ka = (mode == kModeF16) ? kh : smem_u32(tk);
-                    const uint32_t vv = smem_u32(tv);
+                    // U(c) = Kbar^T V (fp16 mode: K^^T V): the k slot read as the MN-major A
+                    const uint32_t ka = smem_u32(tk), vv = smem_u32(tv);
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks)
                         mma_f16_ss(tmem + kColU + bb * 64, smem_desc(ka + ks * 2048, 8192, 1024, kLayoutSw128),
                                    smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_u, ks > 0);
                     mma_commit(&bars[BAR_UFULL + bb]);
+                    mma_commit(&bars[BAR_EMPTY + sl]);  // with O(c)'s commit, frees the slot
                 }
             }
         }
@@ -603,21 +599,21 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         for (int j = 0; j < 32; ++j) S[j] = 0.f;
         bool ok = true, fail = false;
         for (int c = 0; c < N; ++c) {
-            const int s3 = c % 3, bb = c & 1;
+            const int sl = c % kSlots, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
             fail = fail || !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
             // S'_[c] goes to buffer bb, which O(c-2) read last
             if (c >= 2) fail = fail || !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs);
-            if (named_barrier_or(4, 128, fail || *abort_flag != 0u)) {  // the whole warpgroup gives up together
+            if (named_barrier_or(4, 128, fail || *abort_flag != 0u)) {  // the group gives up together
                 ok = false;
                 break;
             }
-            const uint32_t mode = mode_s[s3];
-            const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + s3 * kRefFloats;
+            const uint32_t mode = mode_s[sl];
+            const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + sl * kRefFloats;
             const bool fold = (mode == kModeF16);
             const float c1 = fold ? ref[3 * kD + row] : 1.f;
             const float c2 = fold ? ref[4 * kD + row] : 1.f;
-            const float dc = decay_s[s3 * kD + row];
+            const float dc = decay_s[sl * kD + row];
             // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout)
             {
                 uint8_t *sb = smem + kOffS + bb * kTile16;
@@ -627,17 +623,17 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         make_uint4(h2bits(S[8 * u + 0] * c1, S[8 * u + 1] * c1), h2bits(S[8 * u + 2] * c1, S[8 * u + 3] * c1),
                                    h2bits(S[8 * u + 4] * c1, S[8 * u + 5] * c1), h2bits(S[8 * u + 6] * c1, S[8 * u + 7] * c1));
             }
+            uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
             if (mode != kModeExact) {
                 tc_fence_after();
                 uint32_t r[32];
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColP + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColP + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
-                uint8_t *pt = fold ? (smem + kOffOp + bb * kOpBytes + kTile16)
-                                   : (smem + kOffQkg + (c % kQS) * kQkgBytes + 2 * kTile16);
+                // masked P over the gate tile (consumed by A(c) long ago)
 #pragma unroll
                 for (int u = 0; u < 4; ++u)
-                    *reinterpret_cast<uint4 *>(pt + sw128(row, (ch0 + 8 * u) * 2)) = make_uint4(
+                    *reinterpret_cast<uint4 *>(st + kG + sw128(row, (ch0 + 8 * u) * 2)) = make_uint4(
                         h2bits(__uint_as_float(r[8 * u + 0]), __uint_as_float(r[8 * u + 1])) & pm[4 * u + 0],
                         h2bits(__uint_as_float(r[8 * u + 2]), __uint_as_float(r[8 * u + 3])) & pm[4 * u + 1],
                         h2bits(__uint_as_float(r[8 * u + 4]), __uint_as_float(r[8 * u + 5])) & pm[4 * u + 2],
@@ -649,31 +645,24 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_P + bb]);
             named_barrier_sync(4, 128);  // masked P and S'_[c] of every thread are in shared memory
             if (elected) {
-                // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V)
+                // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V), all from the slot
                 if (!mbar_wait(&bars[BAR_TFREE_O + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
                     fail = true;  // stops the group at the next chunk's barrier
                 } else {
                     tc_fence_after();
-                    const uint32_t qkg = smem_u32(smem + kOffQkg + (c % kQS) * kQkgBytes);
-                    const uint32_t op = smem_u32(smem + kOffOp + bb * kOpBytes);
-                    const uint32_t qa = fold ? op : qkg;
-                    const uint32_t pp = fold ? op + kTile16 : qkg + 2 * kTile16;
-                    const uint32_t vv = smem_u32(smem + kOffV + (c % kVS) * kTile16);
+                    const uint32_t sa = smem_u32(st);
                     const uint32_t ss = smem_u32(smem + kOffS + bb * kTile16);
                     const uint32_t d = tmem + kColO + bb * 64;
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks)
-                        mma_f16_ss(d, smem_desc(qa + ks * 32, 16, 1024, kLayoutSw128),
+                        mma_f16_ss(d, smem_desc(sa + kQ + ks * 32, 16, 1024, kLayoutSw128),
                                    smem_desc(ss + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, ks > 0);
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks)
-                        mma_f16_ss(d, smem_desc(pp + ks * 32, 16, 1024, kLayoutSw128),
-                                   smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
+                        mma_f16_ss(d, smem_desc(sa + kG + ks * 32, 16, 1024, kLayoutSw128),
+                                   smem_desc(sa + kV + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
                     mma_commit(&bars[BAR_OFULL + bb]);
-                    mma_commit(&bars[BAR_VEMPTY + c % kVS]);
-                    // fp16 mode: Q^, K^, P lived in the operand buffer; otherwise Qtil, Kbar, P
-                    // lived in the q/k/g slot
-                    mma_commit(fold ? &bars[BAR_OPFREE + bb] : &bars[BAR_QEMPTY + c % kQS]);
+                    mma_commit(&bars[BAR_EMPTY + sl]);  // with U(c)'s commit, frees the slot
                 }
             }
             // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
@@ -707,14 +696,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const int row = 16 * q4 + (lane & 15);
         const int ch0 = 32 * hc;
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
-        const bool elected = (warp == 14 && lane == 0);
+        E *out = static_cast<E *>(p.out);
         bool ok = true;
         for (int c = 0; c < N; ++c) {
             const int bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
             const bool fail = !mbar_wait(&bars[BAR_OFULL + bb], ph, abort_flag, kWaitLimitNs);
-            if (elected) tma_store_wait_read<1>();
-            if (named_barrier_or(3, 128, fail || *abort_flag != 0u)) {  // the whole warpgroup gives up together
+            if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
                 ok = false;
                 break;
             }
@@ -723,28 +711,22 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
             tmem_ld_wait();
-            uint8_t *ob = smem + kOffO + bb * kTile16;
-#pragma unroll
-            for (int u = 0; u < 4; ++u)
-                *reinterpret_cast<uint4 *>(ob + sw128(row, (ch0 + 8 * u) * 2)) = make_uint4(
-                    Elem<E>::pack(__uint_as_float(r[8 * u + 0]), __uint_as_float(r[8 * u + 1])),
-                    Elem<E>::pack(__uint_as_float(r[8 * u + 2]), __uint_as_float(r[8 * u + 3])),
-                    Elem<E>::pack(__uint_as_float(r[8 * u + 4]), __uint_as_float(r[8 * u + 5])),
-                    Elem<E>::pack(__uint_as_float(r[8 * u + 6]), __uint_as_float(r[8 * u + 7])));
             tc_fence_before();
-            fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_O + bb]);
-            named_barrier_sync(3, 128);
-            if (elected) {
-                chunk_boxes(p.order, p.T, p.grid_h, p.grid_w, c, false, [&](int hi, int rw, int c2, int c3) {
-                    tma_store_5d(&p.maps[T_O][hi], ob + rw * 128, 0, h, c2, c3, b);
-                });
-                tma_store_commit();
+            // o row rho -> its token's spatial position
+            const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, c) + row);
+            if (t >= 0) {
+                uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * kD + ch0);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    dst[u] = make_uint4(Elem<E>::pack(__uint_as_float(r[8 * u + 0]), __uint_as_float(r[8 * u + 1])),
+                                        Elem<E>::pack(__uint_as_float(r[8 * u + 2]), __uint_as_float(r[8 * u + 3])),
+                                        Elem<E>::pack(__uint_as_float(r[8 * u + 4]), __uint_as_float(r[8 * u + 5])),
+                                        Elem<E>::pack(__uint_as_float(r[8 * u + 6]), __uint_as_float(r[8 * u + 7])));
             }
         }
         if (!ok) record_timeout(abort_flag);
-        if (elected) tma_store_wait_all<0>();
     }
 
     tc_fence_before();
@@ -798,7 +780,7 @@ bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int rows) {
 }
 
 // Encoded maps are cached per (pointers, shape, order, dtype): a repeated call
-// reuses them instead of encoding 40 maps again.
+// reuses them instead of encoding 32 maps again.
 struct MapKey {
     const void *ptr[kTensors];
     int B, H, grid_h, grid_w, order, dtype;
@@ -819,7 +801,6 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     key.ptr[T_K] = p.k;
     key.ptr[T_V] = p.v;
     key.ptr[T_G] = p.g;
-    key.ptr[T_O] = p.out;
     key.B = p.B;
     key.H = p.H;
     key.grid_h = p.grid_h;
@@ -859,6 +840,7 @@ bool tc_supported(const Problem &p) {
 cudaError_t launch_tc(const Problem &p, cudaStream_t stream) {
     TcParams tp;
     if (!get_maps(p, tp.maps)) return cudaErrorInvalidValue;
+    tp.out = p.out;
     tp.final_state = p.final_state;
     tp.H = p.H;
     tp.grid_h = p.grid_h;
