@@ -34,15 +34,17 @@
 // tensor map per height).  The scan permutation lives in the box coordinates of
 // the loads and in the addresses of the output stores.
 //
-// Warp roles (576 threads, one CTA per SM).  Each MMA is issued by one elected
-// thread of the role that produced its last operand, as soon as it is ready:
+// Warp roles (640 threads, one CTA per SM).  MMAs are issued by dedicated
+// single-thread issuers, so no compute warp ever waits on MMA issue:
 //   warp 0       TMA producer.
 //   warp 1       TMEM allocator; issues A = L G when a stage lands.
-//   warps 2-5    gen warpgroup 0 (even chunks): reads A, builds the operands,
-//   warps 6-9    gen warpgroup 1 (odd chunks)    issues P and U.
-//   warps 10-13  epi-P: masks P into fp16, writes Diag(c1) S, issues O, carries
-//                the fp32 state S in registers.
+//   warps 2-5    gen warpgroup 0 (even chunks): reads A, builds the operands.
+//   warps 6-9    gen warpgroup 1 (odd chunks)
+//   warps 10-13  epi-P: masks P into fp16, writes Diag(c1) S, carries the fp32
+//                state S in registers.
 //   warps 14-17  epi-O: converts O and stores it at the tokens' spatial positions.
+//   warp 18      issues P and U when a chunk's operands are ready.
+//   warp 19      issues O when a chunk's masked P and scaled state are ready.
 // A warp reads the TMEM lanes of sub-partition (warp % 4); an M = 64 accumulator
 // keeps rows 16q..16q+15 in lanes 32q..32q+15, and each thread takes one row and
 // 32 of its 64 columns.
@@ -72,7 +74,7 @@ constexpr int kD = 64;                    // Dk = Dv handled by this kernel
 constexpr int kSlots = 5;                 // stage slots (chunks in flight)
 constexpr int kTile16 = kC * kD * 2;      // 64 x 64 16-bit tile (SW128, 128-byte rows)
 constexpr int kTile32 = kC * kD * 4;      // 64 x 64 fp32 tile (two 32-column K-blocks)
-constexpr int kThreads = 576;
+constexpr int kThreads = 640;
 constexpr int kHeights = 8;               // TMA box heights 8, 16, ..., 64
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
 constexpr float kLog2e = 1.4426950408889634f;
@@ -105,14 +107,16 @@ enum {
     BAR_AFULL = BAR_EMPTY + kSlots,    // [2] A done -> gen
     BAR_TFREE_A = BAR_AFULL + 2,       // [2] gen drained A -> A issuer
     BAR_OPFREE = BAR_TFREE_A + 2,      // tf32 operand buffer released (once per chunk)
-    BAR_PFULL = BAR_OPFREE + 1,        // [2] P done -> epi-P
+    BAR_OPND = BAR_OPFREE + 1,         // [2] gen -> P/U issuer (operands in smem), 4 arrivals
+    BAR_PREADY = BAR_OPND + 2,         // [2] epi-P -> O issuer (P and S' in smem), 4 arrivals
+    BAR_PFULL = BAR_PREADY + 2,        // [2] P done -> epi-P
     BAR_UFULL = BAR_PFULL + 2,         // [2] U done -> epi-P
     BAR_OFULL = BAR_UFULL + 2,         // [2] O done -> epi-O (and epi-P: S buffer free)
-    BAR_TFREE_P = BAR_OFULL + 2,       // [2] epi-P drained P -> gen (P issuer)
-    BAR_TFREE_U = BAR_TFREE_P + 2,     // [2] epi-P drained U -> gen (U issuer)
-    BAR_TFREE_O = BAR_TFREE_U + 2,     // [2] epi-O drained O -> epi-P (O issuer)
-    BAR_DONE = BAR_TFREE_O + 2,        // [4] per issuing thread: its MMAs completed
-    BAR_COUNT = BAR_DONE + 4
+    BAR_TFREE_P = BAR_OFULL + 2,       // [2] epi-P drained P -> P/U issuer
+    BAR_TFREE_U = BAR_TFREE_P + 2,     // [2] epi-P drained U -> P/U issuer
+    BAR_TFREE_O = BAR_TFREE_U + 2,     // [2] epi-O drained O -> O issuer
+    BAR_DONE = BAR_TFREE_O + 2,        // [3] per issuing thread: its MMAs completed
+    BAR_COUNT = BAR_DONE + 3
 };
 static_assert(BAR_COUNT <= kNumBars, "barrier space");
 
@@ -298,6 +302,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         for (int i = 0; i < 2; ++i) {
             mbar_init(&bars[BAR_AFULL + i], 1);
             mbar_init(&bars[BAR_TFREE_A + i], 4);
+            mbar_init(&bars[BAR_OPND + i], 4);
+            mbar_init(&bars[BAR_PREADY + i], 4);
             mbar_init(&bars[BAR_PFULL + i], 1);
             mbar_init(&bars[BAR_UFULL + i], 1);
             mbar_init(&bars[BAR_OFULL + i], 1);
@@ -305,7 +311,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             mbar_init(&bars[BAR_TFREE_U + i], 4);
             mbar_init(&bars[BAR_TFREE_O + i], 4);
         }
-        for (int i = 0; i < 4; ++i) mbar_init(&bars[BAR_DONE + i], 1);
+        for (int i = 0; i < 3; ++i) mbar_init(&bars[BAR_DONE + i], 1);
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -395,9 +401,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
         const int tg = threadIdx.x - 64 - 128 * gw;
         const int rho_mid = rev ? 32 : 31, rho_last = rev ? 0 : 63;
-        const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
-        const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
-        const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
         for (int c = gw; c < N; c += 2) {
             const int sl = c % kSlots, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
@@ -524,58 +527,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
             }
             fence_proxy_async_smem();
-            if (named_barrier_or(bar_id, 128, opfail)) {  // every operand of chunk c is in shared memory
+            if (named_barrier_or(bar_id, 128, opfail)) {
                 record_timeout(abort_flag);
                 break;
             }
-            if (tg == 0) {
-                if (mode == kModeF16) {
-                    // pass the shared tf32 buffer on: this chunk does not use it
-                    if (!mbar_wait(&bars[BAR_OPFREE], (c & 1) ^ 1, abort_flag, kWaitLimitNs)) record_timeout(abort_flag);
-                    mbar_arrive(&bars[BAR_OPFREE]);
-                } else if (mode == kModeExact) {
-                    mbar_arrive(&bars[BAR_OPFREE]);  // the exact path's scratch use is over
-                }
-                if (!mbar_wait(&bars[BAR_TFREE_P + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
-                    !mbar_wait(&bars[BAR_TFREE_U + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
-                    record_timeout(abort_flag);
-                } else {
-                    tc_fence_after();
-                    // P(c) = Q^ K^^T
-                    if (mode == kModeTF32) {
-                        const uint32_t qh = smem_u32(smem + kOffOp), kh = qh + kTile32;
-#pragma unroll
-                        for (int ks = 0; ks < 8; ++ks) {
-                            const uint32_t o = (ks >> 2) * 8192 + (ks & 3) * 32;
-                            mma_tf32_ss(tmem + kColP + bb * 64, smem_desc(qh + o, 16, 1024, kLayoutSw128),
-                                        smem_desc(kh + o, 16, 1024, kLayoutSw128), idesc_p32, ks > 0);
-                        }
-                        mma_commit(&bars[BAR_PFULL + bb]);
-                        mma_commit(&bars[BAR_OPFREE]);
-                    } else if (mode == kModeF16) {
-                        const uint32_t qh = smem_u32(tq), kh = smem_u32(tk);
-#pragma unroll
-                        for (int ks = 0; ks < 4; ++ks)
-                            mma_f16_ss(tmem + kColP + bb * 64, smem_desc(qh + ks * 32, 16, 1024, kLayoutSw128),
-                                       smem_desc(kh + ks * 32, 16, 1024, kLayoutSw128), idesc_p16, ks > 0);
-                        mma_commit(&bars[BAR_PFULL + bb]);
-                    } else {
-                        mbar_arrive(&bars[BAR_PFULL + bb]);
-                    }
-                    // U(c) = Kbar^T V (fp16 mode: K^^T V): the k slot read as the MN-major A
-                    const uint32_t ka = smem_u32(tk), vv = smem_u32(tv);
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks)
-                        mma_f16_ss(tmem + kColU + bb * 64, smem_desc(ka + ks * 2048, 8192, 1024, kLayoutSw128),
-                                   smem_desc(vv + ks * 2048, 8192, 1024, kLayoutSw128), idesc_u, ks > 0);
-                    mma_commit(&bars[BAR_UFULL + bb]);
-                    mma_commit(&bars[BAR_EMPTY + sl]);  // with O(c)'s commit, frees the slot
-                }
-            }
-        }
-        if (tg == 0) {
-            mma_commit(&bars[BAR_DONE + 1 + gw]);
-            mbar_wait(&bars[BAR_DONE + 1 + gw], 0, nullptr, kWaitLimitNs);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bars[BAR_OPND + bb]);  // operands of chunk c are in smem
         }
     } else if (warp < 14) {
         // ======================================================= epi-P warpgroup
@@ -583,8 +540,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const int row = 16 * q4 + (lane & 15);   // token rho for P, channel i for U / S
         const int ch0 = 32 * hc;
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
-        const bool elected = (warp == 10 && lane == 0);
-        const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
         // causal mask of this thread's 32 P columns as packed fp16-pair masks (scan order)
         uint32_t pm[16];
 #pragma unroll
@@ -604,7 +559,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             fail = fail || !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
             // S'_[c] goes to buffer bb, which O(c-2) read last
             if (c >= 2) fail = fail || !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs);
-            if (named_barrier_or(4, 128, fail || *abort_flag != 0u)) {  // the group gives up together
+            if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
                 ok = false;
                 break;
             }
@@ -642,28 +597,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tc_fence_before();
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_TFREE_P + bb]);
-            named_barrier_sync(4, 128);  // masked P and S'_[c] of every thread are in shared memory
-            if (elected) {
-                // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V), all from the slot
-                if (!mbar_wait(&bars[BAR_TFREE_O + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
-                    fail = true;  // stops the group at the next chunk's barrier
-                } else {
-                    tc_fence_after();
-                    const uint32_t sa = smem_u32(st);
-                    const uint32_t ss = smem_u32(smem + kOffS + bb * kTile16);
-                    const uint32_t d = tmem + kColO + bb * 64;
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks)
-                        mma_f16_ss(d, smem_desc(sa + kQ + ks * 32, 16, 1024, kLayoutSw128),
-                                   smem_desc(ss + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, ks > 0);
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks)
-                        mma_f16_ss(d, smem_desc(sa + kG + ks * 32, 16, 1024, kLayoutSw128),
-                                   smem_desc(sa + kV + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
-                    mma_commit(&bars[BAR_OFULL + bb]);
-                    mma_commit(&bars[BAR_EMPTY + sl]);  // with U(c)'s commit, frees the slot
-                }
+            if (lane == 0) {
+                mbar_arrive(&bars[BAR_TFREE_P + bb]);
+                mbar_arrive(&bars[BAR_PREADY + bb]);  // this warp's rows of P and S'_[c] are in smem
             }
             // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
             fail = fail || !mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs);
@@ -681,16 +617,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (lane == 0) mbar_arrive(&bars[BAR_TFREE_U + bb]);
         }
         if (!ok || fail) record_timeout(abort_flag);
-        if (elected) {
-            mma_commit(&bars[BAR_DONE + 3]);
-            mbar_wait(&bars[BAR_DONE + 3], 0, nullptr, kWaitLimitNs);
-        }
         if (ok && !fail && p.final_state != nullptr) {
             float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)bh * kD + row) * kD + ch0);
 #pragma unroll
             for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
         }
-    } else {
+    } else if (warp < 18) {
         // ======================================================= epi-O warpgroup
         const int q4 = warp & 3, hc = lane >> 4;
         const int row = 16 * q4 + (lane & 15);
@@ -727,6 +659,99 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             }
         }
         if (!ok) record_timeout(abort_flag);
+    } else if (warp == 18) {
+        // ======================================================= P/U issuer
+        if (lane == 0) {
+            const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
+            const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
+            const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
+            for (int c = 0; c < N; ++c) {
+                const int sl = c % kSlots, bb = c & 1;
+                const uint32_t ph = (c >> 1) & 1;
+                if (!mbar_wait(&bars[BAR_OPND + bb], ph, abort_flag, kWaitLimitNs)) {
+                    record_timeout(abort_flag);
+                    break;
+                }
+                const uint32_t mode = mode_s[sl];
+                if (mode == kModeF16) {
+                    // pass the shared tf32 buffer on: this chunk did not use it
+                    if (!mbar_wait(&bars[BAR_OPFREE], (c & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                        record_timeout(abort_flag);
+                        break;
+                    }
+                    mbar_arrive(&bars[BAR_OPFREE]);
+                } else if (mode == kModeExact) {
+                    mbar_arrive(&bars[BAR_OPFREE]);  // the exact path's scratch use is over
+                }
+                if (!mbar_wait(&bars[BAR_TFREE_P + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
+                    !mbar_wait(&bars[BAR_TFREE_U + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
+                    record_timeout(abort_flag);
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t st = smem_u32(smem + kOffSlot + sl * kSlotBytes);
+                // P(c) = Q^ K^^T
+                if (mode == kModeTF32) {
+                    const uint32_t qh = smem_u32(smem + kOffOp), kh = qh + kTile32;
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const uint32_t o = (ks >> 2) * 8192 + (ks & 3) * 32;
+                        mma_tf32_ss(tmem + kColP + bb * 64, smem_desc(qh + o, 16, 1024, kLayoutSw128),
+                                    smem_desc(kh + o, 16, 1024, kLayoutSw128), idesc_p32, ks > 0);
+                    }
+                    mma_commit(&bars[BAR_PFULL + bb]);
+                    mma_commit(&bars[BAR_OPFREE]);
+                } else if (mode == kModeF16) {
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        mma_f16_ss(tmem + kColP + bb * 64, smem_desc(st + kQ + ks * 32, 16, 1024, kLayoutSw128),
+                                   smem_desc(st + kK + ks * 32, 16, 1024, kLayoutSw128), idesc_p16, ks > 0);
+                    mma_commit(&bars[BAR_PFULL + bb]);
+                } else {
+                    mbar_arrive(&bars[BAR_PFULL + bb]);
+                }
+                // U(c) = Kbar^T V (fp16 mode: K^^T V): the k slot read as the MN-major A
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_f16_ss(tmem + kColU + bb * 64, smem_desc(st + kK + ks * 2048, 8192, 1024, kLayoutSw128),
+                               smem_desc(st + kV + ks * 2048, 8192, 1024, kLayoutSw128), idesc_u, ks > 0);
+                mma_commit(&bars[BAR_UFULL + bb]);
+                mma_commit(&bars[BAR_EMPTY + sl]);  // with O(c)'s commit, frees the slot
+            }
+            mma_commit(&bars[BAR_DONE + 1]);
+            mbar_wait(&bars[BAR_DONE + 1], 0, nullptr, kWaitLimitNs);
+        }
+    } else {
+        // ======================================================= O issuer (warp 19)
+        if (lane == 0) {
+            const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
+            for (int c = 0; c < N; ++c) {
+                const int sl = c % kSlots, bb = c & 1;
+                const uint32_t ph = (c >> 1) & 1;
+                if (!mbar_wait(&bars[BAR_PREADY + bb], ph, abort_flag, kWaitLimitNs) ||
+                    !mbar_wait(&bars[BAR_TFREE_O + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
+                    record_timeout(abort_flag);
+                    break;
+                }
+                tc_fence_after();
+                // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V), all from the slot
+                const uint32_t st = smem_u32(smem + kOffSlot + sl * kSlotBytes);
+                const uint32_t ss = smem_u32(smem + kOffS + bb * kTile16);
+                const uint32_t d = tmem + kColO + bb * 64;
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_f16_ss(d, smem_desc(st + kQ + ks * 32, 16, 1024, kLayoutSw128),
+                               smem_desc(ss + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    mma_f16_ss(d, smem_desc(st + kG + ks * 32, 16, 1024, kLayoutSw128),
+                               smem_desc(st + kV + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
+                mma_commit(&bars[BAR_OFULL + bb]);
+                mma_commit(&bars[BAR_EMPTY + sl]);  // with U(c)'s commit, frees the slot
+            }
+            mma_commit(&bars[BAR_DONE + 2]);
+            mbar_wait(&bars[BAR_DONE + 2], 0, nullptr, kWaitLimitNs);
+        }
     }
 
     tc_fence_before();
