@@ -106,8 +106,7 @@ enum {
     BAR_EMPTY = BAR_FULL + kSlots,     // [kSlots] U and O done -> producer (two commits)
     BAR_AFULL = BAR_EMPTY + kSlots,    // [2] A done -> gen
     BAR_TFREE_A = BAR_AFULL + 2,       // [2] gen drained A -> A issuer
-    BAR_OPFREE = BAR_TFREE_A + 2,      // tf32 operand buffer released (once per chunk)
-    BAR_OPND = BAR_OPFREE + 1,         // [2] gen -> P/U issuer (operands in smem), 4 arrivals
+    BAR_OPND = BAR_TFREE_A + 2,        // [2] gen -> P/U issuer (operands in smem), 4 arrivals
     BAR_PREADY = BAR_OPND + 2,         // [2] epi-P -> O issuer (P and S' in smem), 4 arrivals
     BAR_PFULL = BAR_PREADY + 2,        // [2] P done -> epi-P
     BAR_UFULL = BAR_PFULL + 2,         // [2] U done -> epi-P
@@ -178,6 +177,20 @@ template <> struct Elem<__nv_bfloat16> {
 __device__ __forceinline__ void record_timeout(volatile uint32_t *abort_flag) {
     *abort_flag = 1u;
     atomicOr(&g_device_status, kStatusTimeout);
+}
+
+// Bounded wait until *counter >= target (a counter written by one thread of
+// this CTA); false on timeout or when another role gave up.
+__device__ __forceinline__ bool wait_counter(const volatile uint32_t *counter, uint32_t target,
+                                             const volatile uint32_t *abort, uint64_t limit_ns) {
+    if (*counter >= target) return true;
+    const uint64_t t0 = global_timer_ns();
+    while (*counter < target) {
+        if (*abort) return false;
+        if (global_timer_ns() - t0 > limit_ns) return false;
+        __nanosleep(20);
+    }
+    return true;
 }
 
 // Smem row rho of chunk c holds walk position w0 + rho, where the walk is the
@@ -282,6 +295,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBar);
     volatile uint32_t *tmem_base_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc);
     volatile uint32_t *abort_flag = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc + 4);
+    // chunks whose P product is done: the tf32 / exact-path scratch buffer may be
+    // reused by chunk c once op_done >= c (a counter, so no phase can be misread)
+    volatile uint32_t *op_done = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc + 8);
     float *decay_s = reinterpret_cast<float *>(smem + kOffDecay);
     volatile uint32_t *mode_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMode);
     float *mx_s = reinterpret_cast<float *>(smem + kOffMode + 32);   // [2][2] partial maxima
@@ -294,11 +310,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 
     if (threadIdx.x == 0) {
         *abort_flag = 0u;
+        *op_done = 0u;
         for (int i = 0; i < kSlots; ++i) {
             mbar_init(&bars[BAR_FULL + i], 1);
             mbar_init(&bars[BAR_EMPTY + i], 2);  // U(c) and O(c) both done (issued by two threads)
         }
-        mbar_init(&bars[BAR_OPFREE], 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&bars[BAR_AFULL + i], 1);
             mbar_init(&bars[BAR_TFREE_A + i], 4);
@@ -452,7 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (mode != kModeF16) {
                 // the tf32 / scratch buffer is shared by consecutive chunks: wait for the previous
                 // release; the decision is uniform because the exact path has named barriers
-                opfail = named_barrier_or(bar_id, 128, !mbar_wait(&bars[BAR_OPFREE], (c & 1) ^ 1, abort_flag, kWaitLimitNs));
+                opfail = named_barrier_or(bar_id, 128, !wait_counter(op_done, (uint32_t)c, abort_flag, kWaitLimitNs));
             }
             if (mode != kModeExact) {
                 uint8_t *qh = smem + kOffOp, *kh = qh + kTile32;
@@ -532,7 +548,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 break;
             }
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_OPND + bb]);  // operands of chunk c are in smem
+            if (lane == 0) {
+                // OPND[bb] may run at most one phase ahead of its waiter: chunk c-2's P must be
+                // done (so the issuer consumed chunk c-2's arrivals) before chunk c arrives
+                if (c >= 2 && !mbar_wait(&bars[BAR_PFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs))
+                    record_timeout(abort_flag);
+                mbar_arrive(&bars[BAR_OPND + bb]);  // operands of chunk c are in smem
+            }
         }
     } else if (warp < 14) {
         // ======================================================= epi-P warpgroup
@@ -563,6 +585,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 ok = false;
                 break;
             }
+            if (warp == 10 && lane == 0) *op_done = (uint32_t)c + 1u;  // P(c) is done
             const uint32_t mode = mode_s[sl];
             const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + sl * kRefFloats;
             const bool fold = (mode == kModeF16);
@@ -673,16 +696,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     break;
                 }
                 const uint32_t mode = mode_s[sl];
-                if (mode == kModeF16) {
-                    // pass the shared tf32 buffer on: this chunk did not use it
-                    if (!mbar_wait(&bars[BAR_OPFREE], (c & 1) ^ 1, abort_flag, kWaitLimitNs)) {
-                        record_timeout(abort_flag);
-                        break;
-                    }
-                    mbar_arrive(&bars[BAR_OPFREE]);
-                } else if (mode == kModeExact) {
-                    mbar_arrive(&bars[BAR_OPFREE]);  // the exact path's scratch use is over
-                }
                 if (!mbar_wait(&bars[BAR_TFREE_P + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
                     !mbar_wait(&bars[BAR_TFREE_U + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
                     record_timeout(abort_flag);
@@ -700,7 +713,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                     smem_desc(kh + o, 16, 1024, kLayoutSw128), idesc_p32, ks > 0);
                     }
                     mma_commit(&bars[BAR_PFULL + bb]);
-                    mma_commit(&bars[BAR_OPFREE]);
                 } else if (mode == kModeF16) {
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks)
