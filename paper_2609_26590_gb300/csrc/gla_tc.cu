@@ -34,17 +34,16 @@
 // tensor map per height).  The scan permutation lives in the box coordinates of
 // the loads and in the addresses of the output stores.
 //
-// Warp roles (640 threads, one CTA per SM).  MMAs are issued by dedicated
-// single-thread issuers, so no compute warp ever waits on MMA issue:
+// Warp roles (448 threads, one CTA per SM).  Few roles with small loops keep
+// the hot code inside the SM's instruction cache:
 //   warp 0       TMA producer.
-//   warp 1       TMEM allocator; issues A = L G when a stage lands.
-//   warps 2-5    gen warpgroup 0 (even chunks): reads A, builds the operands.
-//   warps 6-9    gen warpgroup 1 (odd chunks)
-//   warps 10-13  epi-P: masks P into fp16, writes Diag(c1) S, carries the fp32
-//                state S in registers.
-//   warps 14-17  epi-O: converts O and stores it at the tokens' spatial positions.
-//   warp 18      issues P and U when a chunk's operands are ready.
-//   warp 19      issues O when a chunk's masked P and scaled state are ready.
+//   warp 1       TMEM allocator; one thread issues every MMA (A, P, U, O) from a
+//                polling loop, whichever stage has its inputs ready.
+//   warps 2-5    gen warpgroup 0 (even chunks): reads A, builds the operands of its
+//                chunk, then masks the chunk's scores P into fp16.
+//   warps 6-9    gen warpgroup 1 (odd chunks).
+//   warps 10-13  epi: carries the fp32 state S in registers, writes Diag(c1) S,
+//                and stores each chunk's outputs at the tokens' spatial positions.
 // A warp reads the TMEM lanes of sub-partition (warp % 4); an M = 64 accumulator
 // keeps rows 16q..16q+15 in lanes 32q..32q+15, and each thread takes one row and
 // 32 of its 64 columns.
@@ -74,7 +73,7 @@ constexpr int kD = 64;                    // Dk = Dv handled by this kernel
 constexpr int kSlots = 5;                 // stage slots (chunks in flight)
 constexpr int kTile16 = kC * kD * 2;      // 64 x 64 16-bit tile (SW128, 128-byte rows)
 constexpr int kTile32 = kC * kD * 4;      // 64 x 64 fp32 tile (two 32-column K-blocks)
-constexpr int kThreads = 640;
+constexpr int kThreads = 448;
 constexpr int kHeights = 8;               // TMA box heights 8, 16, ..., 64
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
 constexpr float kLog2e = 1.4426950408889634f;
@@ -102,20 +101,21 @@ constexpr int kSmemBytes = kOffMisc + 64 + 1024;               // + alignment sl
 static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
 enum {
-    BAR_FULL = 0,                      // [kSlots] TMA -> A issuer / gen
-    BAR_EMPTY = BAR_FULL + kSlots,     // [kSlots] U and O done -> producer (two commits)
-    BAR_AFULL = BAR_EMPTY + kSlots,    // [2] A done -> gen
-    BAR_TFREE_A = BAR_AFULL + 2,       // [2] gen drained A -> A issuer
-    BAR_OPND = BAR_TFREE_A + 2,        // [2] gen -> P/U issuer (operands in smem), 4 arrivals
-    BAR_PREADY = BAR_OPND + 2,         // [2] epi-P -> O issuer (P and S' in smem), 4 arrivals
-    BAR_PFULL = BAR_PREADY + 2,        // [2] P done -> epi-P
-    BAR_UFULL = BAR_PFULL + 2,         // [2] U done -> epi-P
-    BAR_OFULL = BAR_UFULL + 2,         // [2] O done -> epi-O (and epi-P: S buffer free)
-    BAR_TFREE_P = BAR_OFULL + 2,       // [2] epi-P drained P -> P/U issuer
-    BAR_TFREE_U = BAR_TFREE_P + 2,     // [2] epi-P drained U -> P/U issuer
-    BAR_TFREE_O = BAR_TFREE_U + 2,     // [2] epi-O drained O -> O issuer
-    BAR_DONE = BAR_TFREE_O + 2,        // [3] per issuing thread: its MMAs completed
-    BAR_COUNT = BAR_DONE + 3
+    BAR_FULL = 0,                      // [kSlots] TMA -> issuer (A)
+    BAR_EMPTY = BAR_FULL + kSlots,     // [kSlots] O(c) and everything before it done -> producer
+    BAR_REFS = BAR_EMPTY + kSlots,     // [kSlots] gen -> epi: chunk constants and mode
+    BAR_AFULL = BAR_REFS + kSlots,     // [2] A done -> gen
+    BAR_TFREE_A = BAR_AFULL + 2,       // [2] gen drained A -> issuer, 4 arrivals
+    BAR_OPND = BAR_TFREE_A + 2,        // [2] gen -> issuer (operands in smem), 4 arrivals
+    BAR_PFULL = BAR_OPND + 2,          // [2] P done -> gen
+    BAR_PREADY = BAR_PFULL + 2,        // [2] gen -> issuer (masked P in smem, TMEM P drained), 4 arrivals
+    BAR_UFULL = BAR_PREADY + 2,        // [2] U done -> epi
+    BAR_TFREE_U = BAR_UFULL + 2,       // [2] epi drained U -> issuer, 4 arrivals
+    BAR_SREADY = BAR_TFREE_U + 2,      // [2] epi -> issuer (Diag(c1) S in smem), 4 arrivals
+    BAR_OFULL = BAR_SREADY + 2,        // [2] O done -> epi
+    BAR_TFREE_O = BAR_OFULL + 2,       // [2] epi drained O -> issuer, 4 arrivals
+    BAR_DONE = BAR_TFREE_O + 2,        // every MMA completed (teardown)
+    BAR_COUNT = BAR_DONE + 1
 };
 static_assert(BAR_COUNT <= kNumBars, "barrier space");
 
@@ -138,6 +138,12 @@ __device__ __forceinline__ uint32_t sw128(uint32_t row, uint32_t byte) {
 __device__ __forceinline__ uint32_t off32(uint32_t row, uint32_t col) {
     return (col >> 5) * 8192u + sw128(row, (col & 31u) * 4u);
 }
+// SW128 operand descriptors: K-major tiles (8-row groups 1024 B apart) and
+// MN-major tiles (64-element atoms 8192 B apart).  A K step of 16 elements adds
+// 32 B (2 in the address field) to a K-major descriptor and 2048 B (128) to an
+// MN-major one.
+__device__ __forceinline__ uint64_t kdesc(uint32_t saddr) { return smem_desc(saddr, 16, 1024, kLayoutSw128); }
+__device__ __forceinline__ uint64_t mndesc(uint32_t saddr) { return smem_desc(saddr, 8192, 1024, kLayoutSw128); }
 __device__ __forceinline__ float ex2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
@@ -287,6 +293,55 @@ __device__ __noinline__ void exact_chunk(uint8_t *tq, uint8_t *tk, uint8_t *tgat
     }
 }
 
+// Operands of a tf32-mode chunk (split factors beyond the fp16 range): tf32 Q^ and
+// K^ for the score product in the scratch buffer, fp16 Qtil = Q^ c1 over q and
+// Kbar = K^ c2 over k.  Re-reads the thread's 32 log-decays from TMEM (A is kept
+// until the operands are built).
+template <typename E>
+__device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *opbuf, const float *ref,
+                                           uint32_t taddr, int row, int ch0) {
+    uint32_t ar[32];
+    tmem_ld_16x32bx2_x16(taddr + 0, *reinterpret_cast<uint32_t(*)[16]>(&ar[0]));
+    tmem_ld_16x32bx2_x16(taddr + 16, *reinterpret_cast<uint32_t(*)[16]>(&ar[16]));
+    tmem_ld_wait();
+    uint8_t *qh = opbuf, *kh = opbuf + kTile32;
+#pragma unroll
+    for (int g8 = 0; g8 < 4; ++g8) {
+        const int cl = ch0 + 8 * g8;
+        const uint32_t o16 = sw128(row, cl * 2);
+        const uint4 qw = *reinterpret_cast<const uint4 *>(tq + o16);
+        const uint4 kw = *reinterpret_cast<const uint4 *>(tk + o16);
+        const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w}, ka[4] = {kw.x, kw.y, kw.z, kw.w};
+        float qs[8], ks[8];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 q2 = Elem<E>::unpack(qa[e]), k2 = Elem<E>::unpack(ka[e]);
+            const float e0 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e]), kLog2e, -ref[2 * kD + cl + 2 * e]);
+            const float e1 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e + 1]), kLog2e, -ref[2 * kD + cl + 2 * e + 1]);
+            qs[2 * e] = q2.x * ex2(e0);
+            qs[2 * e + 1] = q2.y * ex2(e1);
+            ks[2 * e] = k2.x * ex2(-e0);
+            ks[2 * e + 1] = k2.y * ex2(-e1);
+        }
+        *reinterpret_cast<float4 *>(qh + off32(row, cl)) =
+            make_float4(to_tf32(qs[0]), to_tf32(qs[1]), to_tf32(qs[2]), to_tf32(qs[3]));
+        *reinterpret_cast<float4 *>(qh + off32(row, cl + 4)) =
+            make_float4(to_tf32(qs[4]), to_tf32(qs[5]), to_tf32(qs[6]), to_tf32(qs[7]));
+        *reinterpret_cast<float4 *>(kh + off32(row, cl)) =
+            make_float4(to_tf32(ks[0]), to_tf32(ks[1]), to_tf32(ks[2]), to_tf32(ks[3]));
+        *reinterpret_cast<float4 *>(kh + off32(row, cl + 4)) =
+            make_float4(to_tf32(ks[4]), to_tf32(ks[5]), to_tf32(ks[6]), to_tf32(ks[7]));
+        uint32_t qo[4], ko[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            qo[e] = h2bits(qs[2 * e] * ref[3 * kD + cl + 2 * e], qs[2 * e + 1] * ref[3 * kD + cl + 2 * e + 1]);
+            ko[e] = h2bits(ks[2 * e] * ref[4 * kD + cl + 2 * e], ks[2 * e + 1] * ref[4 * kD + cl + 2 * e + 1]);
+        }
+        *reinterpret_cast<uint4 *>(tq + o16) = make_uint4(qo[0], qo[1], qo[2], qo[3]);
+        *reinterpret_cast<uint4 *>(tk + o16) = make_uint4(ko[0], ko[1], ko[2], ko[3]);
+    }
+}
+
 template <typename E>
 __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_constant__ TcParams p) {
     extern __shared__ uint8_t smem_raw[];
@@ -295,9 +350,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBar);
     volatile uint32_t *tmem_base_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc);
     volatile uint32_t *abort_flag = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc + 4);
-    // chunks whose P product is done: the tf32 / exact-path scratch buffer may be
-    // reused by chunk c once op_done >= c (a counter, so no phase can be misread)
-    volatile uint32_t *op_done = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc + 8);
+    // chunks whose P product is done (a maximum over the two gen groups): the tf32 /
+    // exact-path scratch buffer may be reused by chunk c once op_done >= c
+    uint32_t *op_done = reinterpret_cast<uint32_t *>(smem + kOffMisc + 8);
     float *decay_s = reinterpret_cast<float *>(smem + kOffDecay);
     volatile uint32_t *mode_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMode);
     float *mx_s = reinterpret_cast<float *>(smem + kOffMode + 32);   // [2][2] partial maxima
@@ -313,21 +368,22 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         *op_done = 0u;
         for (int i = 0; i < kSlots; ++i) {
             mbar_init(&bars[BAR_FULL + i], 1);
-            mbar_init(&bars[BAR_EMPTY + i], 2);  // U(c) and O(c) both done (issued by two threads)
+            mbar_init(&bars[BAR_EMPTY + i], 1);
+            mbar_init(&bars[BAR_REFS + i], 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&bars[BAR_AFULL + i], 1);
             mbar_init(&bars[BAR_TFREE_A + i], 4);
             mbar_init(&bars[BAR_OPND + i], 4);
-            mbar_init(&bars[BAR_PREADY + i], 4);
             mbar_init(&bars[BAR_PFULL + i], 1);
+            mbar_init(&bars[BAR_PREADY + i], 4);
             mbar_init(&bars[BAR_UFULL + i], 1);
-            mbar_init(&bars[BAR_OFULL + i], 1);
-            mbar_init(&bars[BAR_TFREE_P + i], 4);
             mbar_init(&bars[BAR_TFREE_U + i], 4);
+            mbar_init(&bars[BAR_SREADY + i], 4);
+            mbar_init(&bars[BAR_OFULL + i], 1);
             mbar_init(&bars[BAR_TFREE_O + i], 4);
         }
-        for (int i = 0; i < 3; ++i) mbar_init(&bars[BAR_DONE + i], 1);
+        mbar_init(&bars[BAR_DONE], 1);
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -385,27 +441,110 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             }
         }
     } else if (warp == 1) {
-        // ======================================================= A issuer: A(c) = L G
-        if (lane == 0) {
+        // ======================================================= MMA issuer
+        // One thread issues every product, in a polling loop over three stages so
+        // that a stage waiting on its inputs never holds back another:
+        //   A(a) = L G               when stage a landed and TMEM A[a%2] was drained
+        //   P(u) = Q^ K^^T, U(u)     when the operands of chunk u are in smem; P(u) waits
+        //                            for O(u-2) to be issued (TMEM P[u%2] drained by then)
+        //   O(o) = Q S'_[o] + P V    when masked P and the scaled state of chunk o are in smem
+        // The ordering o <= u <= a and u <= o + 2 keeps every two-phase barrier at
+        // most one phase ahead of its waiter.
+        {
             const uint32_t idesc_a = instr_desc(Elem<E>::fmt, 64, 64, 0, 1);
-            const uint32_t L = smem_u32(smem + kOffL);
-            for (int c = 0; c < N; ++c) {
-                const int bb = c & 1;
-                if (!mbar_wait(&bars[BAR_FULL + c % kSlots], (c / kSlots) & 1, abort_flag, kWaitLimitNs) ||
-                    !mbar_wait(&bars[BAR_TFREE_A + bb], ((c >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
-                    record_timeout(abort_flag);
+            const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
+            const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
+            const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
+            const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
+            const uint32_t slot0 = smem_u32(smem + kOffSlot);
+            const uint64_t dL = kdesc(smem_u32(smem + kOffL));
+            const uint64_t dqh = kdesc(smem_u32(smem + kOffOp)), dkh = kdesc(smem_u32(smem + kOffOp + kTile32));
+            const uint32_t sbuf = smem_u32(smem + kOffS);
+            int a = 0, u = 0, o = 0;
+            int sa = 0, su = 0, so = 0;  // slots of chunks a, u, o
+            uint32_t idle = 0;
+            uint64_t t_idle = 0;
+            bool ok = true;
+            while (o < N) {
+                bool progress = false;
+                if (a < N && __all_sync(0xffffffffu, mbar_test(&bars[BAR_FULL + sa], (a / kSlots) & 1) &&
+                                                         mbar_test(&bars[BAR_TFREE_A + (a & 1)], ((a >> 1) & 1) ^ 1))) {
+                    tc_fence_after();
+                    const uint64_t dg = mndesc(slot0 + sa * kSlotBytes + kG);
+                    const uint32_t d = tmem + kColA + (a & 1) * 64;
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dL + 2 * ks, dg + 128 * ks, idesc_a, ks > 0);
+                    mma_commit_warp(&bars[BAR_AFULL + (a & 1)]);
+                    ++a;
+                    sa = (sa == kSlots - 1) ? 0 : sa + 1;
+                    progress = true;
+                }
+                if (u < a && u < o + 2 &&
+                    __all_sync(0xffffffffu, mbar_test(&bars[BAR_OPND + (u & 1)], (u >> 1) & 1) &&
+                                                mbar_test(&bars[BAR_TFREE_U + (u & 1)], ((u >> 1) & 1) ^ 1))) {
+                    tc_fence_after();
+                    const uint32_t st = slot0 + su * kSlotBytes;
+                    const uint32_t mode = __shfl_sync(0xffffffffu, mode_s[su], 0);
+                    const uint32_t dp = tmem + kColP + (u & 1) * 64;
+                    if (mode == kModeF16) {
+                        const uint64_t dq = kdesc(st + kQ), dk = kdesc(st + kK);
+#pragma unroll
+                        for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(dp, dq + 2 * ks, dk + 2 * ks, idesc_p16, ks > 0);
+                        mma_commit_warp(&bars[BAR_PFULL + (u & 1)]);
+                    } else if (mode == kModeTF32) {
+#pragma unroll
+                        for (int ks = 0; ks < 8; ++ks) {
+                            const uint32_t off = (ks >> 2) * 512 + (ks & 3) * 2;  // (8192 B, 32 B) >> 4
+                            mma_tf32_ss_warp(dp, dqh + off, dkh + off, idesc_p32, ks > 0);
+                        }
+                        mma_commit_warp(&bars[BAR_PFULL + (u & 1)]);
+                    } else if (lane == 0) {
+                        mbar_arrive(&bars[BAR_PFULL + (u & 1)]);  // exact scores are already in smem
+                    }
+                    __syncwarp();
+                    // U(u) = Kbar^T V (fp16 mode: K^^T V): the k tile read as the MN-major A
+                    const uint64_t dk = mndesc(st + kK), dv = mndesc(st + kV);
+                    const uint32_t du = tmem + kColU + (u & 1) * 64;
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(du, dk + 128 * ks, dv + 128 * ks, idesc_u, ks > 0);
+                    mma_commit_warp(&bars[BAR_UFULL + (u & 1)]);
+                    ++u;
+                    su = (su == kSlots - 1) ? 0 : su + 1;
+                    progress = true;
+                }
+                if (o < u && __all_sync(0xffffffffu, mbar_test(&bars[BAR_PREADY + (o & 1)], (o >> 1) & 1) &&
+                                                         mbar_test(&bars[BAR_SREADY + (o & 1)], (o >> 1) & 1) &&
+                                                         mbar_test(&bars[BAR_TFREE_O + (o & 1)], ((o >> 1) & 1) ^ 1))) {
+                    tc_fence_after();
+                    // O(o) = Qtil S_[o] + P V  (fp16 mode: Q^ (Diag(c1) S_[o]) + P V)
+                    const uint32_t st = slot0 + so * kSlotBytes;
+                    const uint64_t dq = kdesc(st + kQ), ds = mndesc(sbuf + (o & 1) * kTile16);
+                    const uint64_t dpm = kdesc(st + kG), dv = mndesc(st + kV);
+                    const uint32_t d = tmem + kColO + (o & 1) * 64;
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dq + 2 * ks, ds + 128 * ks, idesc_o, ks > 0);
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dpm + 2 * ks, dv + 128 * ks, idesc_o, 1);
+                    mma_commit_warp(&bars[BAR_OFULL + (o & 1)]);
+                    mma_commit_warp(&bars[BAR_EMPTY + so]);  // every product of the slot's chunk is done
+                    ++o;
+                    so = (so == kSlots - 1) ? 0 : so + 1;
+                    progress = true;
+                }
+                if (progress) {
+                    idle = 0;
+                    continue;
+                }
+                if (++idle == 1) t_idle = global_timer_ns();
+                if ((idle & 63u) == 0u &&
+                    __any_sync(0xffffffffu, *abort_flag != 0u || global_timer_ns() - t_idle > kWaitLimitNs)) {
+                    ok = false;
                     break;
                 }
-                tc_fence_after();
-                const uint32_t gt = smem_u32(smem + kOffSlot + (c % kSlots) * kSlotBytes + kG);
-#pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    mma_f16_ss(tmem + kColA + bb * 64, smem_desc(L + ks * 32, 16, 1024, kLayoutSw128),
-                               smem_desc(gt + ks * 2048, 8192, 1024, kLayoutSw128), idesc_a, ks > 0);
-                mma_commit(&bars[BAR_AFULL + bb]);
             }
-            mma_commit(&bars[BAR_DONE + 0]);  // TMEM is released only after these MMAs completed
-            mbar_wait(&bars[BAR_DONE + 0], 0, nullptr, kWaitLimitNs);
+            if (!ok && lane == 0) record_timeout(abort_flag);
+            mma_commit_warp(&bars[BAR_DONE]);  // TMEM is released only after every MMA completed
+            mbar_wait(&bars[BAR_DONE], 0, nullptr, kWaitLimitNs);
         }
     } else if (warp < 10) {
         // ======================================================= gen warpgroups (chunks c = gw mod 2)
@@ -413,10 +552,19 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const int bar_id = 1 + gw;
         const int q4 = warp & 3, hc = lane >> 4;
         const int row = 16 * q4 + (lane & 15);   // smem row rho of this thread's accumulator row
-        const int ch0 = 32 * hc;                 // its 32 key channels
+        const int ch0 = 32 * hc;                 // its 32 key channels (A) / score columns (P)
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
         const int tg = threadIdx.x - 64 - 128 * gw;
         const int rho_mid = rev ? 32 : 31, rho_last = rev ? 0 : 63;
+        // causal mask of this thread's 32 score columns as packed fp16-pair masks (scan order)
+        uint32_t pm[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+            const int s0 = ch0 + 2 * e;
+            const bool k0 = rev ? (s0 >= row) : (s0 <= row);
+            const bool k1 = rev ? (s0 + 1 >= row) : (s0 + 1 <= row);
+            pm[e] = (k0 ? 0x0000FFFFu : 0u) | (k1 ? 0xFFFF0000u : 0u);
+        }
         for (int c = gw; c < N; c += 2) {
             const int sl = c % kSlots, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
@@ -432,17 +580,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (!fail && (row == rho_mid || row == rho_last)) {
                 float *dst = ref + (row == rho_mid ? 0 : kD) + ch0;
 #pragma unroll
-                for (int u = 0; u < 8; ++u)
-                    reinterpret_cast<float4 *>(dst)[u] = make_float4(__uint_as_float(ar[4 * u]), __uint_as_float(ar[4 * u + 1]),
-                                                                     __uint_as_float(ar[4 * u + 2]), __uint_as_float(ar[4 * u + 3]));
+                for (int q = 0; q < 8; ++q)
+                    reinterpret_cast<float4 *>(dst)[q] = make_float4(__uint_as_float(ar[4 * q]), __uint_as_float(ar[4 * q + 1]),
+                                                                     __uint_as_float(ar[4 * q + 2]), __uint_as_float(ar[4 * q + 3]));
             }
             tc_fence_before();
             if (named_barrier_or(bar_id, 128, fail || *abort_flag != 0u)) {  // the group gives up together
                 record_timeout(abort_flag);
                 break;
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_TFREE_A + bb]);
             if (tg < kD) {
                 const float am = ref[tg] * kLog2e, al = ref[kD + tg] * kLog2e;
                 float m = fmaxf(-am, am - al);
@@ -470,8 +616,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 // release; the decision is uniform because the exact path has named barriers
                 opfail = named_barrier_or(bar_id, 128, !wait_counter(op_done, (uint32_t)c, abort_flag, kWaitLimitNs));
             }
-            if (mode != kModeExact) {
-                uint8_t *qh = smem + kOffOp, *kh = qh + kTile32;
+            if (mode == kModeF16) {
 #pragma unroll
                 for (int g8 = 0; g8 < 4; ++g8) {
                     const int cl = ch0 + 8 * g8;
@@ -482,56 +627,31 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     const uint4 qw = *reinterpret_cast<const uint4 *>(tq + o16);
                     const uint4 kw = *reinterpret_cast<const uint4 *>(tk + o16);
                     const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w}, ka[4] = {kw.x, kw.y, kw.z, kw.w};
-                    float qs[8], ks[8];
+                    uint32_t qo[4], ko[4];
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
                         const float2 q2 = Elem<E>::unpack(qa[e]), k2 = Elem<E>::unpack(ka[e]);
                         const float e0 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e]), kLog2e, -amv[2 * e]);
                         const float e1 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e + 1]), kLog2e, -amv[2 * e + 1]);
-                        qs[2 * e] = q2.x * ex2(e0);
-                        qs[2 * e + 1] = q2.y * ex2(e1);
-                        ks[2 * e] = k2.x * ex2(-e0);
-                        ks[2 * e + 1] = k2.y * ex2(-e1);
+                        qo[e] = h2bits(q2.x * ex2(e0), q2.y * ex2(e1));
+                        ko[e] = h2bits(k2.x * ex2(-e0), k2.y * ex2(-e1));
                     }
-                    if (mode == kModeF16) {
-                        // Q^ over q, K^ over k (each thread rewrites exactly what it read)
-                        *reinterpret_cast<uint4 *>(tq + o16) =
-                            make_uint4(h2bits(qs[0], qs[1]), h2bits(qs[2], qs[3]), h2bits(qs[4], qs[5]), h2bits(qs[6], qs[7]));
-                        *reinterpret_cast<uint4 *>(tk + o16) =
-                            make_uint4(h2bits(ks[0], ks[1]), h2bits(ks[2], ks[3]), h2bits(ks[4], ks[5]), h2bits(ks[6], ks[7]));
-                    } else if (!opfail) {
-                        const float4 c10 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl);
-                        const float4 c11 = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl + 4);
-                        const float4 c20 = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl);
-                        const float4 c21 = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl + 4);
-                        const float c1v[8] = {c10.x, c10.y, c10.z, c10.w, c11.x, c11.y, c11.z, c11.w};
-                        const float c2v[8] = {c20.x, c20.y, c20.z, c20.w, c21.x, c21.y, c21.z, c21.w};
-                        *reinterpret_cast<float4 *>(qh + off32(row, cl)) =
-                            make_float4(to_tf32(qs[0]), to_tf32(qs[1]), to_tf32(qs[2]), to_tf32(qs[3]));
-                        *reinterpret_cast<float4 *>(qh + off32(row, cl + 4)) =
-                            make_float4(to_tf32(qs[4]), to_tf32(qs[5]), to_tf32(qs[6]), to_tf32(qs[7]));
-                        *reinterpret_cast<float4 *>(kh + off32(row, cl)) =
-                            make_float4(to_tf32(ks[0]), to_tf32(ks[1]), to_tf32(ks[2]), to_tf32(ks[3]));
-                        *reinterpret_cast<float4 *>(kh + off32(row, cl + 4)) =
-                            make_float4(to_tf32(ks[4]), to_tf32(ks[5]), to_tf32(ks[6]), to_tf32(ks[7]));
-                        // Qtil over q, Kbar over k
-                        *reinterpret_cast<uint4 *>(tq + o16) =
-                            make_uint4(h2bits(qs[0] * c1v[0], qs[1] * c1v[1]), h2bits(qs[2] * c1v[2], qs[3] * c1v[3]),
-                                       h2bits(qs[4] * c1v[4], qs[5] * c1v[5]), h2bits(qs[6] * c1v[6], qs[7] * c1v[7]));
-                        *reinterpret_cast<uint4 *>(tk + o16) =
-                            make_uint4(h2bits(ks[0] * c2v[0], ks[1] * c2v[1]), h2bits(ks[2] * c2v[2], ks[3] * c2v[3]),
-                                       h2bits(ks[4] * c2v[4], ks[5] * c2v[5]), h2bits(ks[6] * c2v[6], ks[7] * c2v[7]));
-                    }
+                    // Q^ over q, K^ over k (each thread rewrites exactly what it read)
+                    *reinterpret_cast<uint4 *>(tq + o16) = make_uint4(qo[0], qo[1], qo[2], qo[3]);
+                    *reinterpret_cast<uint4 *>(tk + o16) = make_uint4(ko[0], ko[1], ko[2], ko[3]);
                 }
             } else if (!opfail) {
-                exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp), decay_s + sl * kD, rev, tg,
-                               bar_id);
+                if (mode == kModeTF32)
+                    tf32_operands<E>(tq, tk, smem + kOffOp, ref, tmem + lane_base + kColA + bb * 64, row, ch0);
+                else
+                    exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp), decay_s + sl * kD, rev, tg,
+                                   bar_id);
             }
             if constexpr (std::is_same<E, __nv_bfloat16>::value) {
                 // bf16 values become fp16 MMA operands (exact for |v| in the fp16 normal range)
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
-                    uint4 *pv = reinterpret_cast<uint4 *>(tv + sw128(row, (ch0 + 8 * u) * 2));
+                for (int q = 0; q < 4; ++q) {
+                    uint4 *pv = reinterpret_cast<uint4 *>(tv + sw128(row, (ch0 + 8 * q) * 2));
                     uint4 w = *pv;
                     uint32_t *wp = reinterpret_cast<uint32_t *>(&w);
 #pragma unroll
@@ -543,226 +663,133 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
             }
             fence_proxy_async_smem();
+            tc_fence_before();
             if (named_barrier_or(bar_id, 128, opfail)) {
                 record_timeout(abort_flag);
                 break;
             }
+            if (tg == 0) mbar_arrive(&bars[BAR_REFS + sl]);  // constants and mode of chunk c -> epi
             __syncwarp();
             if (lane == 0) {
-                // OPND[bb] may run at most one phase ahead of its waiter: chunk c-2's P must be
-                // done (so the issuer consumed chunk c-2's arrivals) before chunk c arrives
-                if (c >= 2 && !mbar_wait(&bars[BAR_PFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs))
-                    record_timeout(abort_flag);
-                mbar_arrive(&bars[BAR_OPND + bb]);  // operands of chunk c are in smem
+                mbar_arrive(&bars[BAR_TFREE_A + bb]);  // A(c) is no longer read
+                mbar_arrive(&bars[BAR_OPND + bb]);     // operands of chunk c are in smem
             }
-        }
-    } else if (warp < 14) {
-        // ======================================================= epi-P warpgroup
-        const int q4 = warp & 3, hc = lane >> 4;
-        const int row = 16 * q4 + (lane & 15);   // token rho for P, channel i for U / S
-        const int ch0 = 32 * hc;
-        const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
-        // causal mask of this thread's 32 P columns as packed fp16-pair masks (scan order)
-        uint32_t pm[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-            const int s0 = ch0 + 2 * e;
-            const bool k0 = rev ? (s0 >= row) : (s0 <= row);
-            const bool k1 = rev ? (s0 + 1 >= row) : (s0 + 1 <= row);
-            pm[e] = (k0 ? 0x0000FFFFu : 0u) | (k1 ? 0xFFFF0000u : 0u);
-        }
-        float S[32];
-#pragma unroll
-        for (int j = 0; j < 32; ++j) S[j] = 0.f;
-        bool ok = true, fail = false;
-        for (int c = 0; c < N; ++c) {
-            const int sl = c % kSlots, bb = c & 1;
-            const uint32_t ph = (c >> 1) & 1;
-            fail = fail || !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
-            // S'_[c] goes to buffer bb, which O(c-2) read last
-            if (c >= 2) fail = fail || !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs);
-            if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
-                ok = false;
+            // ---- masked scores of chunk c over its gate tile (consumed by A(c) long ago)
+            const bool pfail = !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
+            if (named_barrier_or(bar_id, 128, pfail)) {
+                record_timeout(abort_flag);
                 break;
             }
-            if (warp == 10 && lane == 0) *op_done = (uint32_t)c + 1u;  // P(c) is done
-            const uint32_t mode = mode_s[sl];
-            const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + sl * kRefFloats;
-            const bool fold = (mode == kModeF16);
-            const float c1 = fold ? ref[3 * kD + row] : 1.f;
-            const float c2 = fold ? ref[4 * kD + row] : 1.f;
-            const float dc = decay_s[sl * kD + row];
-            // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout)
-            {
-                uint8_t *sb = smem + kOffS + bb * kTile16;
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    *reinterpret_cast<uint4 *>(sb + sw128(row, (ch0 + 8 * u) * 2)) =
-                        make_uint4(h2bits(S[8 * u + 0] * c1, S[8 * u + 1] * c1), h2bits(S[8 * u + 2] * c1, S[8 * u + 3] * c1),
-                                   h2bits(S[8 * u + 4] * c1, S[8 * u + 5] * c1), h2bits(S[8 * u + 6] * c1, S[8 * u + 7] * c1));
-            }
-            uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
+            if (tg == 0) atomicMax(op_done, (uint32_t)c + 1u);  // P(c) is done
             if (mode != kModeExact) {
                 tc_fence_after();
                 uint32_t r[32];
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColP + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColP + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
-                // masked P over the gate tile (consumed by A(c) long ago)
 #pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    *reinterpret_cast<uint4 *>(st + kG + sw128(row, (ch0 + 8 * u) * 2)) = make_uint4(
-                        h2bits(__uint_as_float(r[8 * u + 0]), __uint_as_float(r[8 * u + 1])) & pm[4 * u + 0],
-                        h2bits(__uint_as_float(r[8 * u + 2]), __uint_as_float(r[8 * u + 3])) & pm[4 * u + 1],
-                        h2bits(__uint_as_float(r[8 * u + 4]), __uint_as_float(r[8 * u + 5])) & pm[4 * u + 2],
-                        h2bits(__uint_as_float(r[8 * u + 6]), __uint_as_float(r[8 * u + 7])) & pm[4 * u + 3]);
+                for (int q = 0; q < 4; ++q)
+                    *reinterpret_cast<uint4 *>(tgt + sw128(row, (ch0 + 8 * q) * 2)) = make_uint4(
+                        h2bits(__uint_as_float(r[8 * q + 0]), __uint_as_float(r[8 * q + 1])) & pm[4 * q + 0],
+                        h2bits(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])) & pm[4 * q + 1],
+                        h2bits(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])) & pm[4 * q + 2],
+                        h2bits(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])) & pm[4 * q + 3]);
             }
             tc_fence_before();
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&bars[BAR_TFREE_P + bb]);
-                mbar_arrive(&bars[BAR_PREADY + bb]);  // this warp's rows of P and S'_[c] are in smem
-            }
-            // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
-            fail = fail || !mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs);
-            tc_fence_after();
-            {
+            if (lane == 0) mbar_arrive(&bars[BAR_PREADY + bb]);  // this warp's rows of P are in smem
+        }
+    } else {
+        // ======================================================= epi warpgroup
+        // Carries the fp32 state S in registers (thread: channel row, 32 value
+        // columns), writes Diag(c1) S_[c] for the readout product, folds U_c into
+        // the state, and stores O(c-1) at its tokens' spatial positions.
+        const int q4 = warp & 3, hc = lane >> 4;
+        const int row = 16 * q4 + (lane & 15);   // channel i for U / S, token rho for O
+        const int ch0 = 32 * hc;
+        const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
+        E *out = static_cast<E *>(p.out);
+        float S[32];
+#pragma unroll
+        for (int j = 0; j < 32; ++j) S[j] = 0.f;
+        bool ok = true;
+        for (int c = 0; c <= N; ++c) {
+            if (c < N) {
+                const int sl = c % kSlots, bb = c & 1;
+                const uint32_t ph = (c >> 1) & 1;
+                bool fail = !mbar_wait(&bars[BAR_REFS + sl], (c / kSlots) & 1, abort_flag, kWaitLimitNs);
+                if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
+                    ok = false;
+                    break;
+                }
+                const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + sl * kRefFloats;
+                const bool fold = (mode_s[sl] == kModeF16);
+                const float c1 = fold ? ref[3 * kD + row] : 1.f;
+                const float c2 = fold ? ref[4 * kD + row] : 1.f;
+                const float dc = decay_s[sl * kD + row];
+                // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout); buffer bb was
+                // last read by O(c-2), whose completion was observed one iteration ago
+                uint8_t *sb = smem + kOffS + bb * kTile16;
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    *reinterpret_cast<uint4 *>(sb + sw128(row, (ch0 + 8 * q) * 2)) =
+                        make_uint4(h2bits(S[8 * q + 0] * c1, S[8 * q + 1] * c1), h2bits(S[8 * q + 2] * c1, S[8 * q + 3] * c1),
+                                   h2bits(S[8 * q + 4] * c1, S[8 * q + 5] * c1), h2bits(S[8 * q + 6] * c1, S[8 * q + 7] * c1));
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars[BAR_SREADY + bb]);
+                // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
+                fail = !mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs);
+                if (__any_sync(0xffffffffu, fail)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
                 uint32_t r[32];
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
 #pragma unroll
                 for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars[BAR_TFREE_U + bb]);
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_TFREE_U + bb]);
-        }
-        if (!ok || fail) record_timeout(abort_flag);
-        if (ok && !fail && p.final_state != nullptr) {
-            float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)bh * kD + row) * kD + ch0);
+            if (c >= 1) {
+                // outputs of chunk c-1
+                const int co = c - 1, ob = co & 1;
+                const bool fail = !mbar_wait(&bars[BAR_OFULL + ob], (co >> 1) & 1, abort_flag, kWaitLimitNs);
+                if (__any_sync(0xffffffffu, fail)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                uint32_t r[32];
+                tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+                tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+                tmem_ld_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars[BAR_TFREE_O + ob]);
+                // o row rho -> its token's spatial position
+                const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, co) + row);
+                if (t >= 0) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * kD + ch0);
 #pragma unroll
-            for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
-        }
-    } else if (warp < 18) {
-        // ======================================================= epi-O warpgroup
-        const int q4 = warp & 3, hc = lane >> 4;
-        const int row = 16 * q4 + (lane & 15);
-        const int ch0 = 32 * hc;
-        const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
-        E *out = static_cast<E *>(p.out);
-        bool ok = true;
-        for (int c = 0; c < N; ++c) {
-            const int bb = c & 1;
-            const uint32_t ph = (c >> 1) & 1;
-            const bool fail = !mbar_wait(&bars[BAR_OFULL + bb], ph, abort_flag, kWaitLimitNs);
-            if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
-                ok = false;
-                break;
-            }
-            tc_fence_after();
-            uint32_t r[32];
-            tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-            tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
-            tmem_ld_wait();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_TFREE_O + bb]);
-            // o row rho -> its token's spatial position
-            const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, c) + row);
-            if (t >= 0) {
-                uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * kD + ch0);
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    dst[u] = make_uint4(Elem<E>::pack(__uint_as_float(r[8 * u + 0]), __uint_as_float(r[8 * u + 1])),
-                                        Elem<E>::pack(__uint_as_float(r[8 * u + 2]), __uint_as_float(r[8 * u + 3])),
-                                        Elem<E>::pack(__uint_as_float(r[8 * u + 4]), __uint_as_float(r[8 * u + 5])),
-                                        Elem<E>::pack(__uint_as_float(r[8 * u + 6]), __uint_as_float(r[8 * u + 7])));
+                    for (int q = 0; q < 4; ++q)
+                        dst[q] = make_uint4(Elem<E>::pack(__uint_as_float(r[8 * q + 0]), __uint_as_float(r[8 * q + 1])),
+                                            Elem<E>::pack(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])),
+                                            Elem<E>::pack(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])),
+                                            Elem<E>::pack(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])));
+                }
             }
         }
         if (!ok) record_timeout(abort_flag);
-    } else if (warp == 18) {
-        // ======================================================= P/U issuer
-        if (lane == 0) {
-            const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
-            const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
-            const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
-            for (int c = 0; c < N; ++c) {
-                const int sl = c % kSlots, bb = c & 1;
-                const uint32_t ph = (c >> 1) & 1;
-                if (!mbar_wait(&bars[BAR_OPND + bb], ph, abort_flag, kWaitLimitNs)) {
-                    record_timeout(abort_flag);
-                    break;
-                }
-                const uint32_t mode = mode_s[sl];
-                if (!mbar_wait(&bars[BAR_TFREE_P + bb], ph ^ 1, abort_flag, kWaitLimitNs) ||
-                    !mbar_wait(&bars[BAR_TFREE_U + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
-                    record_timeout(abort_flag);
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t st = smem_u32(smem + kOffSlot + sl * kSlotBytes);
-                // P(c) = Q^ K^^T
-                if (mode == kModeTF32) {
-                    const uint32_t qh = smem_u32(smem + kOffOp), kh = qh + kTile32;
+        if (ok && p.final_state != nullptr) {
+            float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)bh * kD + row) * kD + ch0);
 #pragma unroll
-                    for (int ks = 0; ks < 8; ++ks) {
-                        const uint32_t o = (ks >> 2) * 8192 + (ks & 3) * 32;
-                        mma_tf32_ss(tmem + kColP + bb * 64, smem_desc(qh + o, 16, 1024, kLayoutSw128),
-                                    smem_desc(kh + o, 16, 1024, kLayoutSw128), idesc_p32, ks > 0);
-                    }
-                    mma_commit(&bars[BAR_PFULL + bb]);
-                } else if (mode == kModeF16) {
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks)
-                        mma_f16_ss(tmem + kColP + bb * 64, smem_desc(st + kQ + ks * 32, 16, 1024, kLayoutSw128),
-                                   smem_desc(st + kK + ks * 32, 16, 1024, kLayoutSw128), idesc_p16, ks > 0);
-                    mma_commit(&bars[BAR_PFULL + bb]);
-                } else {
-                    mbar_arrive(&bars[BAR_PFULL + bb]);
-                }
-                // U(c) = Kbar^T V (fp16 mode: K^^T V): the k slot read as the MN-major A
-#pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    mma_f16_ss(tmem + kColU + bb * 64, smem_desc(st + kK + ks * 2048, 8192, 1024, kLayoutSw128),
-                               smem_desc(st + kV + ks * 2048, 8192, 1024, kLayoutSw128), idesc_u, ks > 0);
-                mma_commit(&bars[BAR_UFULL + bb]);
-                mma_commit(&bars[BAR_EMPTY + sl]);  // with O(c)'s commit, frees the slot
-            }
-            mma_commit(&bars[BAR_DONE + 1]);
-            mbar_wait(&bars[BAR_DONE + 1], 0, nullptr, kWaitLimitNs);
-        }
-    } else {
-        // ======================================================= O issuer (warp 19)
-        if (lane == 0) {
-            const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
-            for (int c = 0; c < N; ++c) {
-                const int sl = c % kSlots, bb = c & 1;
-                const uint32_t ph = (c >> 1) & 1;
-                if (!mbar_wait(&bars[BAR_PREADY + bb], ph, abort_flag, kWaitLimitNs) ||
-                    !mbar_wait(&bars[BAR_TFREE_O + bb], ph ^ 1, abort_flag, kWaitLimitNs)) {
-                    record_timeout(abort_flag);
-                    break;
-                }
-                tc_fence_after();
-                // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V), all from the slot
-                const uint32_t st = smem_u32(smem + kOffSlot + sl * kSlotBytes);
-                const uint32_t ss = smem_u32(smem + kOffS + bb * kTile16);
-                const uint32_t d = tmem + kColO + bb * 64;
-#pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    mma_f16_ss(d, smem_desc(st + kQ + ks * 32, 16, 1024, kLayoutSw128),
-                               smem_desc(ss + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, ks > 0);
-#pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    mma_f16_ss(d, smem_desc(st + kG + ks * 32, 16, 1024, kLayoutSw128),
-                               smem_desc(st + kV + ks * 2048, 8192, 1024, kLayoutSw128), idesc_o, 1);
-                mma_commit(&bars[BAR_OFULL + bb]);
-                mma_commit(&bars[BAR_EMPTY + sl]);  // with U(c)'s commit, frees the slot
-            }
-            mma_commit(&bars[BAR_DONE + 2]);
-            mbar_wait(&bars[BAR_DONE + 2], 0, nullptr, kWaitLimitNs);
+            for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
         }
     }
 
