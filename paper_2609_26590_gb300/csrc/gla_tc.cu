@@ -37,8 +37,8 @@
 // Warp roles (448 threads, one CTA per SM).  Few roles with small loops keep
 // the hot code inside the SM's instruction cache:
 //   warp 0       TMA producer.
-//   warp 1       TMEM allocator; one thread issues every MMA (A, P, U, O) from a
-//                polling loop, whichever stage has its inputs ready.
+//   warp 1       TMEM allocator and MMA issuer: issues every product (A, P, U, O)
+//                in a fixed software-pipelined order, one barrier wait per stage.
 //   warps 2-5    gen warpgroup 0 (even chunks): reads A, builds the operands of its
 //                chunk, then masks the chunk's scores P into fp16.
 //   warps 6-9    gen warpgroup 1 (odd chunks).
@@ -105,16 +105,14 @@ enum {
     BAR_EMPTY = BAR_FULL + kSlots,     // [kSlots] O(c) and everything before it done -> producer
     BAR_REFS = BAR_EMPTY + kSlots,     // [kSlots] gen -> epi: chunk constants and mode
     BAR_AFULL = BAR_REFS + kSlots,     // [2] A done -> gen
-    BAR_TFREE_A = BAR_AFULL + 2,       // [2] gen drained A -> issuer, 4 arrivals
-    BAR_OPND = BAR_TFREE_A + 2,        // [2] gen -> issuer (operands in smem), 4 arrivals
-    BAR_PFULL = BAR_OPND + 2,          // [2] P done -> gen
-    BAR_PREADY = BAR_PFULL + 2,        // [2] gen -> issuer (masked P in smem, TMEM P drained), 4 arrivals
-    BAR_UFULL = BAR_PREADY + 2,        // [2] U done -> epi
-    BAR_TFREE_U = BAR_UFULL + 2,       // [2] epi drained U -> issuer, 4 arrivals
-    BAR_SREADY = BAR_TFREE_U + 2,      // [2] epi -> issuer (Diag(c1) S in smem), 4 arrivals
-    BAR_OFULL = BAR_SREADY + 2,        // [2] O done -> epi
-    BAR_TFREE_O = BAR_OFULL + 2,       // [2] epi drained O -> issuer, 4 arrivals
-    BAR_DONE = BAR_TFREE_O + 2,        // every MMA completed (teardown)
+    BAR_PURDY = BAR_AFULL + 2,         // [2] P/U(c) may go: gen(c) operands in smem and A(c) read
+                                       //     (4 arrivals) + epi drained U(c-2) (4 arrivals)
+    BAR_PFULL = BAR_PURDY + 2,         // [2] P done -> gen
+    BAR_UFULL = BAR_PFULL + 2,         // [2] U done -> epi
+    BAR_ORDY = BAR_UFULL + 2,          // [2] O(c) may go: gen(c) masked P in smem and TMEM P read
+                                       //     (4) + epi wrote Diag(c1) S_[c] and read O(c-2) (4)
+    BAR_OFULL = BAR_ORDY + 2,          // [2] O done -> epi
+    BAR_DONE = BAR_OFULL + 2,          // every MMA completed (teardown)
     BAR_COUNT = BAR_DONE + 1
 };
 static_assert(BAR_COUNT <= kNumBars, "barrier space");
@@ -355,7 +353,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     uint32_t *op_done = reinterpret_cast<uint32_t *>(smem + kOffMisc + 8);
     float *decay_s = reinterpret_cast<float *>(smem + kOffDecay);
     volatile uint32_t *mode_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMode);
-    float *mx_s = reinterpret_cast<float *>(smem + kOffMode + 32);   // [2][2] partial maxima
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int bh = blockIdx.x;
@@ -373,15 +370,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&bars[BAR_AFULL + i], 1);
-            mbar_init(&bars[BAR_TFREE_A + i], 4);
-            mbar_init(&bars[BAR_OPND + i], 4);
+            mbar_init(&bars[BAR_PURDY + i], 8);
             mbar_init(&bars[BAR_PFULL + i], 1);
-            mbar_init(&bars[BAR_PREADY + i], 4);
             mbar_init(&bars[BAR_UFULL + i], 1);
-            mbar_init(&bars[BAR_TFREE_U + i], 4);
-            mbar_init(&bars[BAR_SREADY + i], 4);
+            mbar_init(&bars[BAR_ORDY + i], 8);
             mbar_init(&bars[BAR_OFULL + i], 1);
-            mbar_init(&bars[BAR_TFREE_O + i], 4);
         }
         mbar_init(&bars[BAR_DONE], 1);
         fence_mbar_init();
@@ -442,110 +435,101 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         }
     } else if (warp == 1) {
         // ======================================================= MMA issuer
-        // One thread issues every product, in a polling loop over three stages so
-        // that a stage waiting on its inputs never holds back another:
-        //   A(a) = L G               when stage a landed and TMEM A[a%2] was drained
-        //   P(u) = Q^ K^^T, U(u)     when the operands of chunk u are in smem; P(u) waits
-        //                            for O(u-2) to be issued (TMEM P[u%2] drained by then)
-        //   O(o) = Q S'_[o] + P V    when masked P and the scaled state of chunk o are in smem
-        // The ordering o <= u <= a and u <= o + 2 keeps every two-phase barrier at
-        // most one phase ahead of its waiter.
-        {
-            const uint32_t idesc_a = instr_desc(Elem<E>::fmt, 64, 64, 0, 1);
-            const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
-            const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
-            const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
-            const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
-            const uint32_t slot0 = smem_u32(smem + kOffSlot);
-            const uint64_t dL = kdesc(smem_u32(smem + kOffL));
-            const uint64_t dqh = kdesc(smem_u32(smem + kOffOp)), dkh = kdesc(smem_u32(smem + kOffOp + kTile32));
-            const uint32_t sbuf = smem_u32(smem + kOffS);
-            int a = 0, u = 0, o = 0;
-            int sa = 0, su = 0, so = 0;  // slots of chunks a, u, o
-            uint32_t idle = 0;
-            uint64_t t_idle = 0;
-            bool ok = true;
-            while (o < N) {
-                bool progress = false;
-                if (a < N && __all_sync(0xffffffffu, mbar_test(&bars[BAR_FULL + sa], (a / kSlots) & 1) &&
-                                                         mbar_test(&bars[BAR_TFREE_A + (a & 1)], ((a >> 1) & 1) ^ 1))) {
+        // The whole warp runs the issue loop (operands warp-uniform) and one elected
+        // lane issues each MMA.  Fixed software-pipelined order, one wait per stage:
+        //   iteration i:  P(i) = Q^ K^^T, U(i) = Kbar^T V   once PURDY(i)
+        //                 A(i+2) = L G                       once stage i+2 landed
+        //                 O(i-1) = Q S'_[i-1] + P V          once ORDY(i-1)
+        // PURDY(i) also says that gen(i) read A(i) (so A(i+2) may overwrite TMEM A) and
+        // that epi drained U(i-2); ORDY(i-1) says TMEM P and O of the same parity were
+        // read.  P(i) comes after O(i-2), so every two-phase barrier stays at most one
+        // phase ahead of its waiter.
+        const uint32_t idesc_a = instr_desc(Elem<E>::fmt, 64, 64, 0, 1);
+        const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
+        const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
+        const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
+        const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
+        const uint32_t slot0 = smem_u32(smem + kOffSlot);
+        const uint64_t dL = kdesc(smem_u32(smem + kOffL));
+        const uint64_t dqh = kdesc(smem_u32(smem + kOffOp)), dkh = kdesc(smem_u32(smem + kOffOp + kTile32));
+        const uint32_t sbuf = smem_u32(smem + kOffS);
+        bool ok = true;
+        for (int c = 0; c < 2 && c < N; ++c) {  // A(0), A(1)
+            ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + c], 0, abort_flag, kWaitLimitNs));
+            if (!ok) break;
+            tc_fence_after();
+            const uint64_t dg = mndesc(slot0 + c * kSlotBytes + kG);
+#pragma unroll
+            for (int ks = 0; ks < 4; ++ks)
+                mma_f16_ss_warp(tmem + kColA + c * 64, dL + 2 * ks, dg + 128 * ks, idesc_a, ks > 0);
+            mma_commit_warp(&bars[BAR_AFULL + c]);
+        }
+        int su = 0, sa = 2 % kSlots, so = 0;   // slots of chunks i, i + 2 and of the next O
+        for (int i = 0; ok && i <= N; ++i) {
+            if (i < N) {
+                ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_PURDY + (i & 1)], (i >> 1) & 1, abort_flag, kWaitLimitNs));
+                if (!ok) break;
+                tc_fence_after();
+                const uint32_t st = slot0 + su * kSlotBytes;
+                const uint32_t mode = __shfl_sync(0xffffffffu, mode_s[su], 0);
+                const uint32_t dp = tmem + kColP + (i & 1) * 64;
+                if (mode == kModeF16) {
+                    const uint64_t dq = kdesc(st + kQ), dk = kdesc(st + kK);
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(dp, dq + 2 * ks, dk + 2 * ks, idesc_p16, ks > 0);
+                    mma_commit_warp(&bars[BAR_PFULL + (i & 1)]);
+                } else if (mode == kModeTF32) {
+#pragma unroll
+                    for (int ks = 0; ks < 8; ++ks) {
+                        const uint32_t off = (ks >> 2) * 512 + (ks & 3) * 2;  // (8192 B, 32 B) >> 4
+                        mma_tf32_ss_warp(dp, dqh + off, dkh + off, idesc_p32, ks > 0);
+                    }
+                    mma_commit_warp(&bars[BAR_PFULL + (i & 1)]);
+                } else if (lane == 0) {
+                    mbar_arrive(&bars[BAR_PFULL + (i & 1)]);  // exact scores are already in smem
+                }
+                __syncwarp();
+                // U(i) = Kbar^T V (fp16 mode: K^^T V): the k tile read as the MN-major A
+                const uint64_t dk = mndesc(st + kK), dv = mndesc(st + kV);
+                const uint32_t du = tmem + kColU + (i & 1) * 64;
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(du, dk + 128 * ks, dv + 128 * ks, idesc_u, ks > 0);
+                mma_commit_warp(&bars[BAR_UFULL + (i & 1)]);
+                su = (su == kSlots - 1) ? 0 : su + 1;
+                if (i + 2 < N) {
+                    ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + sa], ((i + 2) / kSlots) & 1, abort_flag, kWaitLimitNs));
+                    if (!ok) break;
                     tc_fence_after();
                     const uint64_t dg = mndesc(slot0 + sa * kSlotBytes + kG);
-                    const uint32_t d = tmem + kColA + (a & 1) * 64;
+                    const uint32_t d = tmem + kColA + (i & 1) * 64;
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dL + 2 * ks, dg + 128 * ks, idesc_a, ks > 0);
-                    mma_commit_warp(&bars[BAR_AFULL + (a & 1)]);
-                    ++a;
-                    sa = (sa == kSlots - 1) ? 0 : sa + 1;
-                    progress = true;
+                    mma_commit_warp(&bars[BAR_AFULL + (i & 1)]);
                 }
-                if (u < a && u < o + 2 &&
-                    __all_sync(0xffffffffu, mbar_test(&bars[BAR_OPND + (u & 1)], (u >> 1) & 1) &&
-                                                mbar_test(&bars[BAR_TFREE_U + (u & 1)], ((u >> 1) & 1) ^ 1))) {
-                    tc_fence_after();
-                    const uint32_t st = slot0 + su * kSlotBytes;
-                    const uint32_t mode = __shfl_sync(0xffffffffu, mode_s[su], 0);
-                    const uint32_t dp = tmem + kColP + (u & 1) * 64;
-                    if (mode == kModeF16) {
-                        const uint64_t dq = kdesc(st + kQ), dk = kdesc(st + kK);
-#pragma unroll
-                        for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(dp, dq + 2 * ks, dk + 2 * ks, idesc_p16, ks > 0);
-                        mma_commit_warp(&bars[BAR_PFULL + (u & 1)]);
-                    } else if (mode == kModeTF32) {
-#pragma unroll
-                        for (int ks = 0; ks < 8; ++ks) {
-                            const uint32_t off = (ks >> 2) * 512 + (ks & 3) * 2;  // (8192 B, 32 B) >> 4
-                            mma_tf32_ss_warp(dp, dqh + off, dkh + off, idesc_p32, ks > 0);
-                        }
-                        mma_commit_warp(&bars[BAR_PFULL + (u & 1)]);
-                    } else if (lane == 0) {
-                        mbar_arrive(&bars[BAR_PFULL + (u & 1)]);  // exact scores are already in smem
-                    }
-                    __syncwarp();
-                    // U(u) = Kbar^T V (fp16 mode: K^^T V): the k tile read as the MN-major A
-                    const uint64_t dk = mndesc(st + kK), dv = mndesc(st + kV);
-                    const uint32_t du = tmem + kColU + (u & 1) * 64;
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(du, dk + 128 * ks, dv + 128 * ks, idesc_u, ks > 0);
-                    mma_commit_warp(&bars[BAR_UFULL + (u & 1)]);
-                    ++u;
-                    su = (su == kSlots - 1) ? 0 : su + 1;
-                    progress = true;
-                }
-                if (o < u && __all_sync(0xffffffffu, mbar_test(&bars[BAR_PREADY + (o & 1)], (o >> 1) & 1) &&
-                                                         mbar_test(&bars[BAR_SREADY + (o & 1)], (o >> 1) & 1) &&
-                                                         mbar_test(&bars[BAR_TFREE_O + (o & 1)], ((o >> 1) & 1) ^ 1))) {
-                    tc_fence_after();
-                    // O(o) = Qtil S_[o] + P V  (fp16 mode: Q^ (Diag(c1) S_[o]) + P V)
-                    const uint32_t st = slot0 + so * kSlotBytes;
-                    const uint64_t dq = kdesc(st + kQ), ds = mndesc(sbuf + (o & 1) * kTile16);
-                    const uint64_t dpm = kdesc(st + kG), dv = mndesc(st + kV);
-                    const uint32_t d = tmem + kColO + (o & 1) * 64;
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dq + 2 * ks, ds + 128 * ks, idesc_o, ks > 0);
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dpm + 2 * ks, dv + 128 * ks, idesc_o, 1);
-                    mma_commit_warp(&bars[BAR_OFULL + (o & 1)]);
-                    mma_commit_warp(&bars[BAR_EMPTY + so]);  // every product of the slot's chunk is done
-                    ++o;
-                    so = (so == kSlots - 1) ? 0 : so + 1;
-                    progress = true;
-                }
-                if (progress) {
-                    idle = 0;
-                    continue;
-                }
-                if (++idle == 1) t_idle = global_timer_ns();
-                if ((idle & 63u) == 0u &&
-                    __any_sync(0xffffffffu, *abort_flag != 0u || global_timer_ns() - t_idle > kWaitLimitNs)) {
-                    ok = false;
-                    break;
-                }
+                sa = (sa == kSlots - 1) ? 0 : sa + 1;
             }
-            if (!ok && lane == 0) record_timeout(abort_flag);
-            mma_commit_warp(&bars[BAR_DONE]);  // TMEM is released only after every MMA completed
-            mbar_wait(&bars[BAR_DONE], 0, nullptr, kWaitLimitNs);
+            if (i >= 1) {
+                const int c = i - 1;
+                ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_ORDY + (c & 1)], (c >> 1) & 1, abort_flag, kWaitLimitNs));
+                if (!ok) break;
+                tc_fence_after();
+                // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V)
+                const uint32_t st = slot0 + so * kSlotBytes;
+                const uint64_t dq = kdesc(st + kQ), ds = mndesc(sbuf + (c & 1) * kTile16);
+                const uint64_t dpm = kdesc(st + kG), dv = mndesc(st + kV);
+                const uint32_t d = tmem + kColO + (c & 1) * 64;
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dq + 2 * ks, ds + 128 * ks, idesc_o, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dpm + 2 * ks, dv + 128 * ks, idesc_o, 1);
+                mma_commit_warp(&bars[BAR_OFULL + (c & 1)]);
+                mma_commit_warp(&bars[BAR_EMPTY + so]);  // every product of the slot's chunk is done
+                so = (so == kSlots - 1) ? 0 : so + 1;
+            }
         }
+        if (!ok && lane == 0) record_timeout(abort_flag);
+        mma_commit_warp(&bars[BAR_DONE]);  // TMEM is released only after every MMA completed
+        mbar_wait(&bars[BAR_DONE], 0, nullptr, kWaitLimitNs);
     } else if (warp < 10) {
         // ======================================================= gen warpgroups (chunks c = gw mod 2)
         const int gw = (warp - 2) >> 2;          // 0: even chunks, 1: odd chunks
@@ -569,6 +553,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             const int sl = c % kSlots, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
             const bool fail = !mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs);
+            uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
+            // bf16 values become fp16 MMA operands in place (exact for |v| in the fp16
+            // normal range); the loads go first so that their latency hides behind the
+            // operand build, the converted words are stored with the operands
+            uint4 vw[4];
+            if constexpr (std::is_same<E, __nv_bfloat16>::value) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) vw[q] = *reinterpret_cast<const uint4 *>(st + kV + sw128(row, (ch0 + 8 * q) * 2));
+            }
             tc_fence_after();
             uint32_t ar[32];
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&ar[0]));
@@ -589,27 +582,33 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 record_timeout(abort_flag);
                 break;
             }
-            if (tg < kD) {
-                const float am = ref[tg] * kLog2e, al = ref[kD + tg] * kLog2e;
-                float m = fmaxf(-am, am - al);
+            // every warp reduces the split range M over the 64 channels itself (no second
+            // barrier); warp 0 of the group writes the constants the readout and epi use
+            uint32_t mode;
+            {
+                const float am0 = ref[lane] * kLog2e, al0 = ref[kD + lane] * kLog2e;
+                const float am1 = ref[lane + 32] * kLog2e, al1 = ref[kD + lane + 32] * kLog2e;
+                float m = fmaxf(fmaxf(-am0, am0 - al0), fmaxf(-am1, am1 - al1));
                 if (!(m <= 3.0e38f)) m = 3.0e38f;  // NaN / inf gates: exact path
-                ref[2 * kD + tg] = am;
-                ref[3 * kD + tg] = ex2(am);
-                ref[4 * kD + tg] = ex2(al - am);
-                decay_s[sl * kD + tg] = ex2(al);
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 16));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 8));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 4));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
-                if (lane == 0) mx_s[gw * 2 + (tg >> 5)] = m;
+                mode = m <= kMaxRefF16 ? kModeF16 : (m <= kMaxRefTF32 ? kModeTF32 : kModeExact);
+                if (tg < 32) {
+                    ref[2 * kD + lane] = am0;
+                    ref[2 * kD + lane + 32] = am1;
+                    ref[3 * kD + lane] = ex2(am0);
+                    ref[3 * kD + lane + 32] = ex2(am1);
+                    ref[4 * kD + lane] = ex2(al0 - am0);
+                    ref[4 * kD + lane + 32] = ex2(al1 - am1);
+                    decay_s[sl * kD + lane] = ex2(al0);
+                    decay_s[sl * kD + lane + 32] = ex2(al1);
+                    if (tg == 0) mode_s[sl] = mode;
+                }
             }
-            named_barrier_sync(bar_id, 128);
-            const float mmax = fmaxf(mx_s[gw * 2], mx_s[gw * 2 + 1]);
-            const uint32_t mode = mmax <= kMaxRefF16 ? kModeF16 : (mmax <= kMaxRefTF32 ? kModeTF32 : kModeExact);
-            if (tg == 0) mode_s[sl] = mode;
-            uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
-            uint8_t *tq = st + kQ, *tk = st + kK, *tv = st + kV, *tgt = st + kG;
+            uint8_t *tq = st + kQ, *tk = st + kK, *tgt = st + kG;
             bool opfail = false;
             if (mode != kModeF16) {
                 // the tf32 / scratch buffer is shared by consecutive chunks: wait for the previous
@@ -620,9 +619,10 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 #pragma unroll
                 for (int g8 = 0; g8 < 4; ++g8) {
                     const int cl = ch0 + 8 * g8;
-                    const float4 am0 = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl);
-                    const float4 am1 = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl + 4);
-                    const float amv[8] = {am0.x, am0.y, am0.z, am0.w, am1.x, am1.y, am1.z, am1.w};
+                    const float4 am0 = *reinterpret_cast<const float4 *>(ref + cl);  // raw A_mid
+                    const float4 am1 = *reinterpret_cast<const float4 *>(ref + cl + 4);
+                    const float amv[8] = {am0.x * kLog2e, am0.y * kLog2e, am0.z * kLog2e, am0.w * kLog2e,
+                                          am1.x * kLog2e, am1.y * kLog2e, am1.z * kLog2e, am1.w * kLog2e};
                     const uint32_t o16 = sw128(row, cl * 2);
                     const uint4 qw = *reinterpret_cast<const uint4 *>(tq + o16);
                     const uint4 kw = *reinterpret_cast<const uint4 *>(tk + o16);
@@ -648,18 +648,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                    bar_id);
             }
             if constexpr (std::is_same<E, __nv_bfloat16>::value) {
-                // bf16 values become fp16 MMA operands (exact for |v| in the fp16 normal range)
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
-                    uint4 *pv = reinterpret_cast<uint4 *>(tv + sw128(row, (ch0 + 8 * q) * 2));
-                    uint4 w = *pv;
-                    uint32_t *wp = reinterpret_cast<uint32_t *>(&w);
+                    uint32_t *wp = reinterpret_cast<uint32_t *>(&vw[q]);
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        const float2 f = Elem<E>::unpack(wp[e]);
-                        wp[e] = h2bits(f.x, f.y);
+                        const float2 fv = Elem<E>::unpack(wp[e]);
+                        wp[e] = h2bits(fv.x, fv.y);
                     }
-                    *pv = w;
+                    *reinterpret_cast<uint4 *>(st + kV + sw128(row, (ch0 + 8 * q) * 2)) = vw[q];
                 }
             }
             fence_proxy_async_smem();
@@ -670,10 +667,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             }
             if (tg == 0) mbar_arrive(&bars[BAR_REFS + sl]);  // constants and mode of chunk c -> epi
             __syncwarp();
-            if (lane == 0) {
-                mbar_arrive(&bars[BAR_TFREE_A + bb]);  // A(c) is no longer read
-                mbar_arrive(&bars[BAR_OPND + bb]);     // operands of chunk c are in smem
-            }
+            if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // operands in smem, A(c) read
             // ---- masked scores of chunk c over its gate tile (consumed by A(c) long ago)
             const bool pfail = !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
             if (named_barrier_or(bar_id, 128, pfail)) {
@@ -698,7 +692,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tc_fence_before();
             fence_proxy_async_smem();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bars[BAR_PREADY + bb]);  // this warp's rows of P are in smem
+            if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // this warp's rows of P are in smem
         }
     } else {
         // ======================================================= epi warpgroup
@@ -714,7 +708,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 #pragma unroll
         for (int j = 0; j < 32; ++j) S[j] = 0.f;
         bool ok = true;
-        for (int c = 0; c <= N; ++c) {
+        if (lane == 0) {  // TMEM U buffers start out free: the drains of chunks -2 and -1
+            mbar_arrive(&bars[BAR_PURDY + 0]);
+            mbar_arrive(&bars[BAR_PURDY + 1]);
+        }
+        for (int c = 0; ok && c <= N; ++c) {
             if (c < N) {
                 const int sl = c % kSlots, bb = c & 1;
                 const uint32_t ph = (c >> 1) & 1;
@@ -738,7 +736,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                    h2bits(S[8 * q + 4] * c1, S[8 * q + 5] * c1), h2bits(S[8 * q + 6] * c1, S[8 * q + 7] * c1));
                 fence_proxy_async_smem();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&bars[BAR_SREADY + bb]);
+                if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // with O(c-2) read one iteration ago
                 // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
                 fail = !mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs);
                 if (__any_sync(0xffffffffu, fail)) {
@@ -754,10 +752,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&bars[BAR_TFREE_U + bb]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // U(c) drained: counts for chunk c + 2
             }
             if (c >= 1) {
-                // outputs of chunk c-1
+                // outputs of chunk c-1, stored at their tokens' spatial positions
                 const int co = c - 1, ob = co & 1;
                 const bool fail = !mbar_wait(&bars[BAR_OFULL + ob], (co >> 1) & 1, abort_flag, kWaitLimitNs);
                 if (__any_sync(0xffffffffu, fail)) {
@@ -770,9 +769,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
                 tc_fence_before();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&bars[BAR_TFREE_O + ob]);
-                // o row rho -> its token's spatial position
                 const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, co) + row);
                 if (t >= 0) {
                     uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * kD + ch0);
