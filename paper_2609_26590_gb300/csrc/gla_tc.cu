@@ -6,8 +6,9 @@
 //   o_r      = (q_r . e^{A_r}) S_[c] + sum_{j<=r} (sum_i q_ri k_ji e^{A_ri - A_ji}) v_j
 //   U_c      = sum_r (k_r . e^{A_last - A_r})^T v_r,   d_c = e^{A_last}
 //   S_[c+1]  = Diag(d_c) S_[c] + U_c
-// One CTA walks all chunks of one (b, h) sequence (single pass: q, k, v, g are
-// read once, o and S_final written once; S stays on chip between chunks).
+// A persistent CTA per SM walks all chunks of its (b, h) sequences as one stream
+// (single pass: q, k, v, g are read once, o and S_final written once; S stays on
+// chip between chunks, and the pipeline does not drain between sequences).
 //
 // Per chunk, tensor-core products (tcgen05.mma, fp32 accumulators in TMEM):
 //   A = L G          in-chunk cumulative log-decay: L is the 64x64 triangle of
@@ -127,6 +128,7 @@ struct TcParams {
     void *out;
     float *final_state;
     int H, grid_h, grid_w, order, n_chunks, T;
+    int n_seq;                             // B * H sequences, dealt out round-robin to the CTAs
 };
 
 // ---------------------------------------------------------------- helpers
@@ -202,6 +204,16 @@ __device__ __forceinline__ bool wait_counter(const volatile uint32_t *counter, u
 // and w0 mirrors the range for reverse orders (scan position 64c + 63 - rho).
 __device__ __forceinline__ int chunk_w0(int order, int T, int c) {
     return (order & 1) ? (T - kC * (c + 1)) : kC * c;
+}
+
+// A CTA walks the sequences blockIdx.x, blockIdx.x + gridDim.x, ... as one stream
+// of chunks: stream chunk g is chunk c of sequence bh.
+struct StreamPos {
+    int bh, c;
+};
+__device__ __forceinline__ StreamPos stream_pos(int g, int N) {
+    const int j = g / N;
+    return {static_cast<int>(blockIdx.x) + j * static_cast<int>(gridDim.x), g - j * N};
 }
 
 // Visit the TMA load boxes of one chunk: calls f(map height index, smem row, c2, c3).
@@ -355,9 +367,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     volatile uint32_t *mode_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMode);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int bh = blockIdx.x;
-    const int b = bh / p.H, h = bh % p.H;
-    const int N = p.n_chunks;
+    const int N = p.n_chunks;   // chunks per sequence
+    // this CTA's chunk stream: every barrier phase, stage slot and TMEM buffer below
+    // follows the stream index, so consecutive sequences flow through one pipeline
+    const int G = N * ((p.n_seq - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
+                       static_cast<int>(gridDim.x));
     const int rev = p.order & 1;
 
     if (threadIdx.x == 0) {
@@ -411,9 +425,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         // ======================================================= TMA producer
         if (lane == 0) {
             int issued = 0;
-            for (int c = 0; c < N; ++c) {
-                const int sl = c % kSlots;
-                if (!mbar_wait(&bars[BAR_EMPTY + sl], ((c / kSlots) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+            for (int g = 0; g < G; ++g) {
+                const int sl = g % kSlots;
+                const StreamPos ps = stream_pos(g, N);
+                const int b = ps.bh / p.H, h = ps.bh % p.H, c = ps.c;
+                if (!mbar_wait(&bars[BAR_EMPTY + sl], ((g / kSlots) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
                     record_timeout(abort_flag);
                     break;
                 }
@@ -429,8 +445,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 ++issued;
             }
             if (*abort_flag) {  // never leave while copies are still landing in shared memory
-                for (int c = (issued > kSlots ? issued - kSlots : 0); c < issued; ++c)
-                    mbar_wait(&bars[BAR_FULL + c % kSlots], (c / kSlots) & 1, nullptr, kWaitLimitNs);
+                for (int g = (issued > kSlots ? issued - kSlots : 0); g < issued; ++g)
+                    mbar_wait(&bars[BAR_FULL + g % kSlots], (g / kSlots) & 1, nullptr, kWaitLimitNs);
             }
         }
     } else if (warp == 1) {
@@ -454,7 +470,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const uint64_t dqh = kdesc(smem_u32(smem + kOffOp)), dkh = kdesc(smem_u32(smem + kOffOp + kTile32));
         const uint32_t sbuf = smem_u32(smem + kOffS);
         bool ok = true;
-        for (int c = 0; c < 2 && c < N; ++c) {  // A(0), A(1)
+        for (int c = 0; c < 2 && c < G; ++c) {  // A(0), A(1)
             ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + c], 0, abort_flag, kWaitLimitNs));
             if (!ok) break;
             tc_fence_after();
@@ -465,8 +481,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             mma_commit_warp(&bars[BAR_AFULL + c]);
         }
         int su = 0, sa = 2 % kSlots, so = 0;   // slots of chunks i, i + 2 and of the next O
-        for (int i = 0; ok && i <= N; ++i) {
-            if (i < N) {
+        for (int i = 0; ok && i <= G; ++i) {
+            if (i < G) {
                 ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_PURDY + (i & 1)], (i >> 1) & 1, abort_flag, kWaitLimitNs));
                 if (!ok) break;
                 tc_fence_after();
@@ -496,7 +512,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(du, dk + 128 * ks, dv + 128 * ks, idesc_u, ks > 0);
                 mma_commit_warp(&bars[BAR_UFULL + (i & 1)]);
                 su = (su == kSlots - 1) ? 0 : su + 1;
-                if (i + 2 < N) {
+                if (i + 2 < G) {
                     ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + sa], ((i + 2) / kSlots) & 1, abort_flag, kWaitLimitNs));
                     if (!ok) break;
                     tc_fence_after();
@@ -549,7 +565,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             const bool k1 = rev ? (s0 + 1 >= row) : (s0 + 1 <= row);
             pm[e] = (k0 ? 0x0000FFFFu : 0u) | (k1 ? 0xFFFF0000u : 0u);
         }
-        for (int c = gw; c < N; c += 2) {
+        for (int c = gw; c < G; c += 2) {
             const int sl = c % kSlots, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
             const bool fail = !mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs);
@@ -712,10 +728,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             mbar_arrive(&bars[BAR_PURDY + 0]);
             mbar_arrive(&bars[BAR_PURDY + 1]);
         }
-        for (int c = 0; ok && c <= N; ++c) {
-            if (c < N) {
+        for (int c = 0; ok && c <= G; ++c) {
+            if (c < G) {
                 const int sl = c % kSlots, bb = c & 1;
                 const uint32_t ph = (c >> 1) & 1;
+                const StreamPos ps = stream_pos(c, N);
+                if (ps.c == 0) {  // a new sequence starts from S = 0
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) S[j] = 0.f;
+                }
                 bool fail = !mbar_wait(&bars[BAR_REFS + sl], (c / kSlots) & 1, abort_flag, kWaitLimitNs);
                 if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
                     ok = false;
@@ -751,7 +772,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 #pragma unroll
                 for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
                 tc_fence_before();
-                __syncwarp();
+                if (ps.c == N - 1 && p.final_state != nullptr) {  // the sequence's final state
+                    float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)ps.bh * kD + row) * kD + ch0);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
+                }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // U(c) drained: counts for chunk c + 2
             }
@@ -769,7 +794,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
                 tc_fence_before();
-                const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, co) + row);
+                const StreamPos po = stream_pos(co, N);
+                const int b = po.bh / p.H, h = po.bh % p.H;
+                const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
                 if (t >= 0) {
                     uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * kD + ch0);
 #pragma unroll
@@ -782,11 +809,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             }
         }
         if (!ok) record_timeout(abort_flag);
-        if (ok && p.final_state != nullptr) {
-            float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)bh * kD + row) * kD + ch0);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
-        }
     }
 
     tc_fence_before();
@@ -908,8 +930,15 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream) {
     tp.order = p.order;
     tp.T = static_cast<int>(p.T);
     tp.n_chunks = static_cast<int>((p.T + kC - 1) / kC);
-    const dim3 grid(static_cast<unsigned>(p.B * p.H));
-    cudaError_t e;
+    tp.n_seq = static_cast<int>(p.B * p.H);
+    // persistent: one CTA per SM, each walking its share of the sequences
+    int dev = 0, n_sm = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const int n_cta = tp.n_seq < n_sm ? tp.n_seq : n_sm;
+    const dim3 grid(static_cast<unsigned>(n_cta));
     if (p.dtype == 1) {
         e = cudaFuncSetAttribute(gla_tc_kernel<__half>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
         if (e != cudaSuccess) return e;

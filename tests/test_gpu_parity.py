@@ -115,6 +115,30 @@ def test_small_shapes_all_orders(case, schedule):
         assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, dtype, f"state {order}")
 
 
+# More (b, h) sequences than a GB300 has SMs, so that every persistent CTA of the
+# tensor-core schedule walks two or three sequences back to back through one
+# pipeline (state reset, final state and output positions per sequence).
+STREAM = [
+    (37, 9, 16, 12, "bf16", 16.0, 0.0),   # 333 sequences of 3 full chunks
+    (41, 8, 8, 13, "f16", 1.0, -1.0),     # 328 sequences of 104 tokens (ragged), strong decay
+    (23, 15, 24, 16, "bf16", 1.0, -3.0),  # 345 sequences, decays beyond the fp16 split range
+]
+
+
+@pytest.mark.parametrize("case", STREAM, ids=[f"{c[0]}x{c[1]}-{c[2]}x{c[3]}-{c[4]}" for c in STREAM])
+def test_many_sequences_per_cta(case):
+    B, H, gh, gw, dtype, tau, zm = case
+    assert gla.tc_supported(B, H, gh, gw, 64, 64, 0, TORCH_DT[dtype])
+    inp = wl.make_inputs(B, H, gh, gw, 64, 64, dtype, seed=3000 + STREAM.index(case), tau=tau,
+                         z_mean=zm)
+    f = inputs_f64(inp, dtype)
+    for order in wl.ALL_ORDERS:
+        ref_o, ref_s = oracle.recurrence(f["q"], f["k"], f["v"], f["g"], gh, gw, order)
+        out, fs = _run(inp, dtype, gh, gw, order, "tc")
+        assert_within_bar(_np(out), ref_o, dtype, f"out order {order}")
+        assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, dtype, f"state {order}")
+
+
 @pytest.mark.parametrize("dtype", ["f16", "bf16", "f32"])
 @pytest.mark.parametrize("gate", ["one", "zero"])
 def test_gate_extremes(dtype, gate):
