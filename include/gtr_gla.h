@@ -83,7 +83,7 @@ typedef enum {
 /* Kernel schedule.  AUTO picks the fastest schedule that supports the
  * arguments.  SIMT is the plain fp32 CUDA-core recurrence (any dtype, any
  * shape within the common rules; the float32 path).  TC is the tensor-core
- * chunkwise schedule (tcgen05 MMAs, TMEM accumulators, TMA loads/stores):
+ * chunkwise schedule (tcgen05 MMAs, TMEM accumulators, TMA loads):
  * fp16/bf16 only, with the shape rules of gtr_gla_tc_supported(). */
 typedef enum { GTR_SCHED_AUTO = 0, GTR_SCHED_SIMT = 1, GTR_SCHED_TC = 2 } gtr_schedule_t;
 
@@ -103,7 +103,10 @@ gtr_status_t gtr_gla_fwd_sched(const void *q, const void *k, const void *v,
                                void *out, float *final_state, gtr_schedule_t schedule,
                                cudaStream_t stream);
 
-/* 1 when the tensor-core schedule supports these arguments, else 0. */
+/* 1 when the tensor-core schedule supports these arguments, else 0: fp16 or
+ * bf16, Dk and Dv each 64 or 128 (processed in 64-channel key halves and
+ * 64-column value slices), T = grid_h * grid_w a multiple of 8, and for the
+ * column orders grid_h a multiple of 8. */
 int gtr_gla_tc_supported(int B, int H, int grid_h, int grid_w, int Dk, int Dv,
                          gtr_scan_t scan_order, gtr_dtype_t dtype);
 

@@ -112,7 +112,7 @@ enum {
     BAR_UFULL = BAR_PFULL + 2,         // [2] U done -> epi
     BAR_ORDY = BAR_UFULL + 2,          // [2] O(c) may go: gen(c) masked P in smem and TMEM P read
                                        //     (4) + epi wrote Diag(c1) S_[c] and read O(c-2) (4)
-    BAR_OFULL = BAR_ORDY + 2,          // [2] O done -> epi
+    BAR_OFULL = BAR_ORDY + 2,          // [2] O of a virtual chunk done -> epi
     BAR_DONE = BAR_OFULL + 2,          // every MMA completed (teardown)
     BAR_COUNT = BAR_DONE + 1
 };
@@ -128,7 +128,10 @@ struct TcParams {
     void *out;
     float *final_state;
     int H, grid_h, grid_w, order, n_chunks, T;
-    int n_seq;                             // B * H sequences, dealt out round-robin to the CTAs
+    int Dk, Dv;                            // 64 or 128 each
+    int nh;                                // Dk / 64: 64-channel key halves per chunk
+    int nv;                                // Dv / 64: 64-column value slices, one per CTA work unit
+    int n_units;                           // B * H * nv work units, dealt out round-robin to the CTAs
 };
 
 // ---------------------------------------------------------------- helpers
@@ -206,14 +209,24 @@ __device__ __forceinline__ int chunk_w0(int order, int T, int c) {
     return (order & 1) ? (T - kC * (c + 1)) : kC * c;
 }
 
-// A CTA walks the sequences blockIdx.x, blockIdx.x + gridDim.x, ... as one stream
-// of chunks: stream chunk g is chunk c of sequence bh.
+// Work units are (sequence, 64-column value slice) pairs.  A CTA walks the units
+// blockIdx.x, blockIdx.x + gridDim.x, ... as one stream of "virtual chunks": each
+// 64-token chunk of a unit appears once per 64-channel key half (Dk = 128: twice),
+// carrying that half's q, k, g and the unit's v slice.  The output is linear in the
+// key channels (o = sum over halves of Qtil_a S_a + P_a V), so the halves go through
+// the same per-chunk pipeline and only their O products share one accumulator.
 struct StreamPos {
-    int bh, c;
+    int bh;  // sequence b * H + h
+    int vb;  // value slice
+    int c;   // chunk of the sequence
+    int a;   // key half
 };
-__device__ __forceinline__ StreamPos stream_pos(int g, int N) {
-    const int j = g / N;
-    return {static_cast<int>(blockIdx.x) + j * static_cast<int>(gridDim.x), g - j * N};
+__device__ __forceinline__ StreamPos stream_pos(int v, int N, int nh, int lognv) {
+    const int per = N * nh;
+    const int j = v / per, rem = v - j * per;
+    const int unit = static_cast<int>(blockIdx.x) + j * static_cast<int>(gridDim.x);
+    const int c = rem / nh;
+    return {unit >> lognv, unit & ((1 << lognv) - 1), c, rem - c * nh};
 }
 
 // Visit the TMA load boxes of one chunk: calls f(map height index, smem row, c2, c3).
@@ -352,7 +365,7 @@ __device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *op
     }
 }
 
-template <typename E>
+template <typename E, int NH, int NV>
 __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_constant__ TcParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -368,10 +381,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int N = p.n_chunks;   // chunks per sequence
-    // this CTA's chunk stream: every barrier phase, stage slot and TMEM buffer below
-    // follows the stream index, so consecutive sequences flow through one pipeline
-    const int G = N * ((p.n_seq - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
-                       static_cast<int>(gridDim.x));
+    constexpr int nh = NH;   // 64-channel key halves per chunk (Dk / 64)
+    constexpr int lognv = NV - 1;  // 64-column value slices per sequence (Dv / 64): 1 or 2
+    constexpr int kDk = 64 * NH, kDv = 64 * NV;
+    // this CTA's stream of virtual chunks: every barrier phase, stage slot and TMEM
+    // buffer below follows the stream index (O: the real chunk's index), so
+    // consecutive units flow through one pipeline
+    const int G = N * nh *
+                  ((p.n_units - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
+                   static_cast<int>(gridDim.x));
     const int rev = p.order & 1;
 
     if (threadIdx.x == 0) {
@@ -427,8 +445,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             int issued = 0;
             for (int g = 0; g < G; ++g) {
                 const int sl = g % kSlots;
-                const StreamPos ps = stream_pos(g, N);
+                const StreamPos ps = stream_pos(g, N, nh, lognv);
                 const int b = ps.bh / p.H, h = ps.bh % p.H, c = ps.c;
+                const int xk = 64 * ps.a, xv = 64 * ps.vb;  // channel offsets of the key half, value slice
                 if (!mbar_wait(&bars[BAR_EMPTY + sl], ((g / kSlots) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
                     record_timeout(abort_flag);
                     break;
@@ -437,10 +456,10 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 uint64_t *fb = &bars[BAR_FULL + sl];
                 mbar_arrive_expect_tx(fb, kSlotBytes);
                 chunk_load_boxes(p.order, p.T, p.grid_h, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
-                    tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, 0, h, c2, c3, b);
-                    tma_load_5d(st + kK + row * 128, &p.maps[T_K][hi], fb, 0, h, c2, c3, b);
-                    tma_load_5d(st + kV + row * 128, &p.maps[T_V][hi], fb, 0, h, c2, c3, b);
-                    tma_load_5d(st + kG + row * 128, &p.maps[T_G][hi], fb, 0, h, c2, c3, b);
+                    tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, xk, h, c2, c3, b);
+                    tma_load_5d(st + kK + row * 128, &p.maps[T_K][hi], fb, xk, h, c2, c3, b);
+                    tma_load_5d(st + kV + row * 128, &p.maps[T_V][hi], fb, xv, h, c2, c3, b);
+                    tma_load_5d(st + kG + row * 128, &p.maps[T_G][hi], fb, xk, h, c2, c3, b);
                 });
                 ++issued;
             }
@@ -529,13 +548,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_ORDY + (c & 1)], (c >> 1) & 1, abort_flag, kWaitLimitNs));
                 if (!ok) break;
                 tc_fence_after();
-                // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V)
+                // O(c) = Qtil S_[c] + P V  (fp16 mode: Q^ (Diag(c1) S_[c]) + P V); the key
+                // halves of one real chunk accumulate into the same TMEM buffer
                 const uint32_t st = slot0 + so * kSlotBytes;
                 const uint64_t dq = kdesc(st + kQ), ds = mndesc(sbuf + (c & 1) * kTile16);
                 const uint64_t dpm = kdesc(st + kG), dv = mndesc(st + kV);
-                const uint32_t d = tmem + kColO + (c & 1) * 64;
+                const uint32_t d = tmem + kColO + ((c / nh) & 1) * 64;
+                const uint32_t acc0 = (c % nh) != 0;
 #pragma unroll
-                for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dq + 2 * ks, ds + 128 * ks, idesc_o, ks > 0);
+                for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dq + 2 * ks, ds + 128 * ks, idesc_o, acc0 | (ks > 0));
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dpm + 2 * ks, dv + 128 * ks, idesc_o, 1);
                 mma_commit_warp(&bars[BAR_OFULL + (c & 1)]);
@@ -712,17 +733,23 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         }
     } else {
         // ======================================================= epi warpgroup
-        // Carries the fp32 state S in registers (thread: channel row, 32 value
-        // columns), writes Diag(c1) S_[c] for the readout product, folds U_c into
-        // the state, and stores O(c-1) at its tokens' spatial positions.
+        // Carries the fp32 state of the current key half in registers (thread: channel
+        // row, 32 value columns; with two key halves the other half's state waits in So
+        // and the two swap after every virtual chunk), writes Diag(c1) S for the readout
+        // product, folds U into the state, and stores each real chunk's outputs at its
+        // tokens' spatial positions once the O product of its last key half completed.
         const int q4 = warp & 3, hc = lane >> 4;
         const int row = 16 * q4 + (lane & 15);   // channel i for U / S, token rho for O
         const int ch0 = 32 * hc;
         const uint32_t lane_base = static_cast<uint32_t>(32 * q4) << 16;
         E *out = static_cast<E *>(p.out);
-        float S[32];
+        float S[32], So[NH == 2 ? 32 : 1];
 #pragma unroll
         for (int j = 0; j < 32; ++j) S[j] = 0.f;
+        if constexpr (NH == 2) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) So[j] = 0.f;
+        }
         bool ok = true;
         if (lane == 0) {  // TMEM U buffers start out free: the drains of chunks -2 and -1
             mbar_arrive(&bars[BAR_PURDY + 0]);
@@ -732,12 +759,16 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (c < G) {
                 const int sl = c % kSlots, bb = c & 1;
                 const uint32_t ph = (c >> 1) & 1;
-                const StreamPos ps = stream_pos(c, N);
+                const StreamPos ps = stream_pos(c, N, nh, lognv);
                 if (ps.c == 0) {  // a new sequence starts from S = 0
 #pragma unroll
                     for (int j = 0; j < 32; ++j) S[j] = 0.f;
                 }
                 bool fail = !mbar_wait(&bars[BAR_REFS + sl], (c / kSlots) & 1, abort_flag, kWaitLimitNs);
+                // buffer bb was last read by O(c-2) (one key half: observed by the readout of
+                // the previous iteration already)
+                if (NH == 2 && c >= 2)
+                    fail = fail || !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs);
                 if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
                     ok = false;
                     break;
@@ -747,8 +778,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 const float c1 = fold ? ref[3 * kD + row] : 1.f;
                 const float c2 = fold ? ref[4 * kD + row] : 1.f;
                 const float dc = decay_s[sl * kD + row];
-                // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout); buffer bb was
-                // last read by O(c-2), whose completion was observed one iteration ago
+                // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout)
                 uint8_t *sb = smem + kOffS + bb * kTile16;
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
@@ -757,7 +787,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                                    h2bits(S[8 * q + 4] * c1, S[8 * q + 5] * c1), h2bits(S[8 * q + 6] * c1, S[8 * q + 7] * c1));
                 fence_proxy_async_smem();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // with O(c-2) read one iteration ago
+                if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // with the outputs of c-2 read out
                 // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
                 fail = !mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs);
                 if (__any_sync(0xffffffffu, fail)) {
@@ -773,17 +803,26 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
                 tc_fence_before();
                 if (ps.c == N - 1 && p.final_state != nullptr) {  // the sequence's final state
-                    float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)ps.bh * kD + row) * kD + ch0);
+                    float4 *dst = reinterpret_cast<float4 *>(
+                        p.final_state + ((size_t)ps.bh * kDk + 64 * ps.a + row) * kDv + 64 * ps.vb + ch0);
 #pragma unroll
                     for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // U(c) drained: counts for chunk c + 2
+                if constexpr (NH == 2) {  // the other key half comes next
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const float t = S[j];
+                        S[j] = So[j];
+                        So[j] = t;
+                    }
+                }
             }
-            if (c >= 1) {
-                // outputs of chunk c-1, stored at their tokens' spatial positions
-                const int co = c - 1, ob = co & 1;
-                const bool fail = !mbar_wait(&bars[BAR_OFULL + ob], (co >> 1) & 1, abort_flag, kWaitLimitNs);
+            if (c >= nh && c % nh == 0) {
+                // outputs of the real chunk whose last key half is c-1
+                const int co = c - 1, ob = (co / nh) & 1;
+                const bool fail = !mbar_wait(&bars[BAR_OFULL + (co & 1)], (co >> 1) & 1, abort_flag, kWaitLimitNs);
                 if (__any_sync(0xffffffffu, fail)) {
                     ok = false;
                     break;
@@ -794,11 +833,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
                 tc_fence_before();
-                const StreamPos po = stream_pos(co, N);
+                const StreamPos po = stream_pos(co, N, nh, lognv);
                 const int b = po.bh / p.H, h = po.bh % p.H;
                 const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
                 if (t >= 0) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * kD + ch0);
+                    uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * kDv + 64 * po.vb + ch0);
 #pragma unroll
                     for (int q = 0; q < 4; ++q)
                         dst[q] = make_uint4(Elem<E>::pack(__uint_as_float(r[8 * q + 0]), __uint_as_float(r[8 * q + 1])),
@@ -836,10 +875,11 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
 
 // Row orders: dims (D, H, T, 1, B), box (64, 1, rows, 1, 1).
 // Column orders: dims (D, H, W, Hg, B), box (64, 1, 1, rows, 1).
-bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int rows) {
+// D is the tensor's row width (Dk or Dv); a box covers 64 channels at x = 0 or 64.
+bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int width, int rows) {
     auto enc = get_encode();
     if (!enc) return false;
-    const cuuint64_t es = 2, D = kD;
+    const cuuint64_t es = 2, D = static_cast<cuuint64_t>(width);
     const bool col = (p.order >> 1) != 0;
     cuuint64_t dims[5] = {D, (cuuint64_t)p.H, 0, 0, (cuuint64_t)p.B};
     cuuint64_t strides[4] = {D * es, (cuuint64_t)p.H * D * es, 0, (cuuint64_t)p.T * p.H * D * es};
@@ -865,7 +905,7 @@ bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int rows) {
 // reuses them instead of encoding 32 maps again.
 struct MapKey {
     const void *ptr[kTensors];
-    int B, H, grid_h, grid_w, order, dtype;
+    int B, H, grid_h, grid_w, order, dtype, Dk, Dv;
     bool operator==(const MapKey &o) const { return std::memcmp(this, &o, sizeof(MapKey)) == 0; }
 };
 struct MapEntry {
@@ -889,6 +929,8 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     key.grid_w = p.grid_w;
     key.order = p.order;
     key.dtype = p.dtype;
+    key.Dk = p.Dk;
+    key.Dv = p.Dv;
     std::lock_guard<std::mutex> lock(g_map_mutex);
     for (auto it = g_map_cache.begin(); it != g_map_cache.end(); ++it) {
         if (it->key == key) {
@@ -901,18 +943,34 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     e.key = key;
     for (int t = 0; t < kTensors; ++t)
         for (int hi = 0; hi < kHeights; ++hi)
-            if (!encode_map(&e.maps[t][hi], key.ptr[t], p, 8 * (hi + 1))) return false;
+            if (!encode_map(&e.maps[t][hi], key.ptr[t], p, t == T_V ? p.Dv : p.Dk, 8 * (hi + 1))) return false;
     std::memcpy(out, e.maps, sizeof(out));
     g_map_cache.push_front(e);
     if (g_map_cache.size() > kMapCacheSize) g_map_cache.pop_back();
     return true;
 }
 
+template <typename E, int NH, int NV>
+cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
+    cudaError_t e =
+        cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    if (e != cudaSuccess) return e;
+    gla_tc_kernel<E, NH, NV><<<grid, kThreads, kSmemBytes, stream>>>(tp);
+    return cudaSuccess;
+}
+
+// One instantiation per (element type, key halves, value slices).
+template <typename E>
+cudaError_t launch_shape(dim3 grid, const TcParams &tp, cudaStream_t stream) {
+    if (tp.nh == 1) return tp.nv == 1 ? launch_kernel<E, 1, 1>(grid, tp, stream) : launch_kernel<E, 1, 2>(grid, tp, stream);
+    return tp.nv == 1 ? launch_kernel<E, 2, 1>(grid, tp, stream) : launch_kernel<E, 2, 2>(grid, tp, stream);
+}
+
 }  // namespace
 
 bool tc_supported(const Problem &p) {
     if (p.dtype != 1 && p.dtype != 2) return false;       // fp16 / bf16 operands only
-    if (p.Dk != kD || p.Dv != kD) return false;
+    if ((p.Dk != 64 && p.Dk != 128) || (p.Dv != 64 && p.Dv != 128)) return false;  // 64-wide halves
     if (p.T % 8 != 0) return false;                        // box heights are multiples of 8
     if ((p.order >> 1) != 0 && p.grid_h % 8 != 0) return false;  // column segments are too
     if (p.T > (1 << 30)) return false;
@@ -930,25 +988,21 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream) {
     tp.order = p.order;
     tp.T = static_cast<int>(p.T);
     tp.n_chunks = static_cast<int>((p.T + kC - 1) / kC);
-    tp.n_seq = static_cast<int>(p.B * p.H);
-    // persistent: one CTA per SM, each walking its share of the sequences
+    tp.Dk = p.Dk;
+    tp.Dv = p.Dv;
+    tp.nh = p.Dk / 64;
+    tp.nv = p.Dv / 64;
+    tp.n_units = static_cast<int>(p.B * p.H) * tp.nv;
+    // persistent: one CTA per SM, each walking its share of the work units
     int dev = 0, n_sm = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
-    const int n_cta = tp.n_seq < n_sm ? tp.n_seq : n_sm;
+    const int n_cta = tp.n_units < n_sm ? tp.n_units : n_sm;
     const dim3 grid(static_cast<unsigned>(n_cta));
-    if (p.dtype == 1) {
-        e = cudaFuncSetAttribute(gla_tc_kernel<__half>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-        if (e != cudaSuccess) return e;
-        gla_tc_kernel<__half><<<grid, kThreads, kSmemBytes, stream>>>(tp);
-    } else {
-        e = cudaFuncSetAttribute(gla_tc_kernel<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kSmemBytes);
-        if (e != cudaSuccess) return e;
-        gla_tc_kernel<__nv_bfloat16><<<grid, kThreads, kSmemBytes, stream>>>(tp);
-    }
+    e = p.dtype == 1 ? launch_shape<__half>(grid, tp, stream) : launch_shape<__nv_bfloat16>(grid, tp, stream);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -95,6 +95,9 @@ SMALL = [
     (2, 1, 16, 9, 64, 64, "f16", 1.0, -1.0),
     (3, 2, 8, 24, 64, 64, "f16", 16.0, 0.0),
     (1, 1, 48, 40, 64, 64, "bf16", 1.0, -1.0),
+    (2, 2, 8, 24, 64, 128, "f16", 16.0, 0.0),
+    (1, 3, 16, 12, 128, 64, "bf16", 1.0, -1.0),
+    (1, 2, 24, 8, 128, 128, "f16", 1.0, -3.0),
 ]
 
 
@@ -119,17 +122,19 @@ def test_small_shapes_all_orders(case, schedule):
 # tensor-core schedule walks two or three sequences back to back through one
 # pipeline (state reset, final state and output positions per sequence).
 STREAM = [
-    (37, 9, 16, 12, "bf16", 16.0, 0.0),   # 333 sequences of 3 full chunks
-    (41, 8, 8, 13, "f16", 1.0, -1.0),     # 328 sequences of 104 tokens (ragged), strong decay
-    (23, 15, 24, 16, "bf16", 1.0, -3.0),  # 345 sequences, decays beyond the fp16 split range
+    (37, 9, 16, 12, 64, 64, "bf16", 16.0, 0.0),    # 333 sequences of 3 full chunks
+    (41, 8, 8, 13, 64, 64, "f16", 1.0, -1.0),      # 328 sequences of 104 tokens (ragged), strong decay
+    (23, 15, 24, 16, 64, 64, "bf16", 1.0, -3.0),   # 345 sequences, decays beyond the fp16 split range
+    (20, 9, 16, 8, 128, 128, "bf16", 16.0, 0.0),   # 360 work units: two value slices per sequence
 ]
 
 
-@pytest.mark.parametrize("case", STREAM, ids=[f"{c[0]}x{c[1]}-{c[2]}x{c[3]}-{c[4]}" for c in STREAM])
+@pytest.mark.parametrize("case", STREAM, ids=[f"{c[0]}x{c[1]}-{c[2]}x{c[3]}-d{c[4]}_{c[5]}-{c[6]}"
+                                              for c in STREAM])
 def test_many_sequences_per_cta(case):
-    B, H, gh, gw, dtype, tau, zm = case
-    assert gla.tc_supported(B, H, gh, gw, 64, 64, 0, TORCH_DT[dtype])
-    inp = wl.make_inputs(B, H, gh, gw, 64, 64, dtype, seed=3000 + STREAM.index(case), tau=tau,
+    B, H, gh, gw, Dk, Dv, dtype, tau, zm = case
+    assert gla.tc_supported(B, H, gh, gw, Dk, Dv, 0, TORCH_DT[dtype])
+    inp = wl.make_inputs(B, H, gh, gw, Dk, Dv, dtype, seed=3000 + STREAM.index(case), tau=tau,
                          z_mean=zm)
     f = inputs_f64(inp, dtype)
     for order in wl.ALL_ORDERS:
