@@ -88,7 +88,16 @@ typedef enum {
 typedef enum { GTR_SCHED_AUTO = 0, GTR_SCHED_SIMT = 1, GTR_SCHED_TC = 2 } gtr_schedule_t;
 
 /* Forward of the token mixer with the AUTO schedule (argument rules above).
- * Returns GTR_OK once the work is enqueued on `stream`. */
+ * Returns GTR_OK once the work is enqueued on `stream`.  When few, long
+ * sequences would leave most SMs idle, the tensor-core schedule splits each
+ * sequence into equal segments (a first pass stores every segment's end state
+ * from zero and its total decay, the second pass starts each segment from the
+ * fold of the earlier ones: the state carry of Eq. chunk_boundary_main applied
+ * across segments).  Those summaries live in an internal per-device workspace
+ * that this call allocates (cudaMalloc) the first time a problem needs it and
+ * grows outside stream capture; under capture the call never touches it and
+ * runs the schedule unsplit.  Callers that manage memory themselves use
+ * gtr_gla_fwd_ws. */
 gtr_status_t gtr_gla_fwd(const void *q, const void *k, const void *v, const void *log_gate,
                          int B, int H, int grid_h, int grid_w, int Dk, int Dv,
                          gtr_scan_t scan_order, gtr_dtype_t dtype,
@@ -102,6 +111,25 @@ gtr_status_t gtr_gla_fwd_sched(const void *q, const void *k, const void *v,
                                int Dk, int Dv, gtr_scan_t scan_order, gtr_dtype_t dtype,
                                void *out, float *final_state, gtr_schedule_t schedule,
                                cudaStream_t stream);
+
+/* Bytes of workspace gtr_gla_fwd_ws needs for these arguments on the current
+ * device (segment summaries of the split schedule: B*H*(segments-1)*(Dk*Dv +
+ * Dk) floats); 0 when the call does not split sequences (the SIMT schedule,
+ * or enough sequences to fill the device) or the arguments are invalid.  The
+ * number of segments depends on the device's SM count. */
+size_t gtr_gla_workspace_bytes(int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                               gtr_dtype_t dtype);
+
+/* gtr_gla_fwd with a caller-owned device workspace of workspace_bytes >=
+ * gtr_gla_workspace_bytes() bytes, 256-byte aligned (may be NULL when that is
+ * 0).  The call allocates nothing and does not synchronise.  Returns
+ * GTR_ERR_WORKSPACE when the workspace is missing or too small.  Calls that
+ * overlap on the GPU must not share a workspace. */
+gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const void *log_gate,
+                            int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                            gtr_scan_t scan_order, gtr_dtype_t dtype, void *out,
+                            float *final_state, void *workspace, size_t workspace_bytes,
+                            cudaStream_t stream);
 
 /* 1 when the tensor-core schedule supports these arguments, else 0: fp16 or
  * bf16, Dk and Dv each 64 or 128 (processed in 64-channel key halves and

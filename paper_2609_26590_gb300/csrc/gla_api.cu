@@ -2,6 +2,8 @@
 // dispatch, the host-memory entry point and status reporting.  No kernel code.
 #include <cstdint>
 #include <cstring>
+#include <mutex>
+#include <vector>
 
 #include "gla_internal.h"
 #include "gtr_gla.h"
@@ -74,6 +76,58 @@ gtr_status_t make_problem(const void *q, const void *k, const void *v, const voi
 
 size_t round_up(size_t n, size_t a) { return (n + a - 1) / a * a; }
 
+// Internal per-device workspace of gtr_gla_fwd (segment summaries of the split
+// schedule).  It grows, outside stream capture, to the largest size asked for and
+// is kept until exit.  A call whose stream is being captured never uses it, so no
+// captured graph refers to memory that a later growth frees.
+struct DeviceWorkspace {
+    void *ptr = nullptr;
+    size_t bytes = 0;
+};
+std::mutex g_ws_mutex;
+std::vector<DeviceWorkspace> g_ws;
+
+void *internal_workspace(size_t need, cudaStream_t stream, size_t *got) {
+    *got = 0;
+    if (need == 0) return nullptr;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone) return nullptr;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+    std::lock_guard<std::mutex> lock(g_ws_mutex);
+    if ((size_t)dev >= g_ws.size()) g_ws.resize(dev + 1);
+    DeviceWorkspace &w = g_ws[dev];
+    if (w.bytes < need) {
+        if (w.ptr != nullptr && cudaFree(w.ptr) != cudaSuccess) return nullptr;  // waits for its users
+        w.ptr = nullptr;
+        w.bytes = 0;
+        if (cudaMalloc(&w.ptr, need) != cudaSuccess) {
+            w.ptr = nullptr;
+            cudaGetLastError();  // the schedule runs unsplit instead
+            return nullptr;
+        }
+        w.bytes = need;
+    }
+    *got = w.bytes;
+    return w.ptr;
+}
+
+// Dispatch of one validated, non-empty problem; `ws` null means the internal workspace.
+gtr_status_t dispatch(const gtr::Problem &p, gtr_schedule_t schedule, void *ws, size_t ws_bytes, bool own_ws,
+                      cudaStream_t stream) {
+    cudaError_t e;
+    const bool tc = gtr::tc_supported(p);
+    if (schedule == GTR_SCHED_SIMT || (schedule == GTR_SCHED_AUTO && !tc)) {
+        e = gtr::launch_simt(p, stream);
+    } else {
+        if (!tc) return GTR_ERR_UNSUPPORTED;
+        if (!own_ws) ws = internal_workspace(gtr::tc_workspace_bytes(p), stream, &ws_bytes);
+        e = gtr::launch_tc(p, stream, ws, ws_bytes);
+    }
+    if (e != cudaSuccess) return cuda_fail(e);
+    return GTR_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -88,21 +142,29 @@ gtr_status_t gtr_gla_fwd_sched(const void *q, const void *k, const void *v, cons
     if (st != GTR_OK) return st;
     if (schedule < GTR_SCHED_AUTO || schedule > GTR_SCHED_TC) return GTR_ERR_INVALID_ARG;
     if (B == 0 || H == 0) return GTR_OK;
-    cudaError_t e;
-    switch (schedule) {
-    case GTR_SCHED_SIMT:
-        e = gtr::launch_simt(p, stream);
-        break;
-    case GTR_SCHED_TC:
-        if (!gtr::tc_supported(p)) return GTR_ERR_UNSUPPORTED;
-        e = gtr::launch_tc(p, stream);
-        break;
-    default:
-        e = gtr::tc_supported(p) ? gtr::launch_tc(p, stream) : gtr::launch_simt(p, stream);
-        break;
-    }
-    if (e != cudaSuccess) return cuda_fail(e);
-    return GTR_OK;
+    return dispatch(p, schedule, nullptr, 0, false, stream);
+}
+
+size_t gtr_gla_workspace_bytes(int B, int H, int grid_h, int grid_w, int Dk, int Dv, gtr_dtype_t dtype) {
+    if (check_shape(B, H, grid_h, grid_w, Dk, Dv, 0, dtype) != GTR_OK || B == 0 || H == 0) return 0;
+    gtr::Problem p{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, B, H, grid_h, grid_w,
+                   Dk, Dv, 0, dtype, (long long)grid_h * grid_w};
+    return gtr::tc_supported(p) ? gtr::tc_workspace_bytes(p) : 0;
+}
+
+gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const void *log_gate, int B,
+                            int H, int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
+                            gtr_dtype_t dtype, void *out, float *final_state, void *workspace,
+                            size_t workspace_bytes, cudaStream_t stream) {
+    gtr::Problem p;
+    gtr_status_t st = make_problem(q, k, v, log_gate, B, H, grid_h, grid_w, Dk, Dv, scan_order,
+                                   dtype, out, final_state, &p);
+    if (st != GTR_OK) return st;
+    if ((reinterpret_cast<uintptr_t>(workspace) % 256) != 0) return GTR_ERR_INVALID_ARG;
+    if (B == 0 || H == 0) return GTR_OK;
+    const size_t need = gtr_gla_workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype);
+    if (need > 0 && (workspace == nullptr || workspace_bytes < need)) return GTR_ERR_WORKSPACE;
+    return dispatch(p, GTR_SCHED_AUTO, workspace, workspace_bytes, true, stream);
 }
 
 gtr_status_t gtr_gla_fwd(const void *q, const void *k, const void *v, const void *log_gate, int B,

@@ -23,7 +23,12 @@ cudaError_t launch_simt(const Problem &p, cudaStream_t stream);
 
 // Tensor-core chunkwise schedule (gla_tc.cu).
 bool tc_supported(const Problem &p);
-cudaError_t launch_tc(const Problem &p, cudaStream_t stream);
+// Scratch the tensor-core schedule uses for this problem on the current device:
+// per-segment summaries when it splits sequences (few, long ones), else 0.
+size_t tc_workspace_bytes(const Problem &p);
+// Launches the schedule; it splits sequences only when `workspace` holds at least
+// tc_workspace_bytes(p) bytes (256-byte aligned), else it runs unsplit.
+cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes);
 
 // Device status word of the current device (set by bounded device waits).
 cudaError_t read_and_clear_device_status(unsigned int *status);

@@ -83,6 +83,10 @@ constexpr float kMaxRefF16 = 8.0f;        // fp16 score operands: factors within
 constexpr float kMaxRefTF32 = 100.0f;     // tf32 score operands: factors within 2^{+-100}
 
 enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
+// Kernel passes: kFull (sequences whole), kSplitFull (outputs of segments that
+// start from the fold of the earlier segments' summaries), kSummary (the summaries).
+enum : int { kFull = 0, kSplitFull = 1, kSummary = 2 };
+constexpr int kMinSegChunks = 8;          // a split segment keeps at least this many chunks
 
 // Shared-memory map (byte offsets from a 1024-aligned base).
 constexpr int kSlotBytes = 4 * kTile16;                        // q @0, k @8K, v @16K, g @24K
@@ -131,7 +135,12 @@ struct TcParams {
     int Dk, Dv;                            // 64 or 128 each
     int nh;                                // Dk / 64: 64-channel key halves per chunk
     int nv;                                // Dv / 64: 64-column value slices, one per CTA work unit
-    int n_units;                           // B * H * nv work units, dealt out round-robin to the CTAs
+    int n_units;                           // work units of this launch, dealt out round-robin to the CTAs
+    int seg_len;                           // chunks per segment (a sequence split into nseg equal segments)
+    int nseg;                              // segments per sequence (1: no split)
+    int nsu;                               // segments per (sequence, value slice) among this launch's units
+    float *summary;                        // nseg > 1: per (sequence, segment < nseg - 1) end state from zero
+                                           // [Dk][Dv] and total decay [Dk], fp32
 };
 
 // ---------------------------------------------------------------- helpers
@@ -216,17 +225,24 @@ __device__ __forceinline__ int chunk_w0(int order, int T, int c) {
 // key channels (o = sum over halves of Qtil_a S_a + P_a V), so the halves go through
 // the same per-chunk pipeline and only their O products share one accumulator.
 struct StreamPos {
-    int bh;  // sequence b * H + h
-    int vb;  // value slice
-    int c;   // chunk of the sequence
-    int a;   // key half
+    int bh;   // sequence b * H + h
+    int vb;   // value slice
+    int c;    // chunk of the sequence
+    int a;    // key half
+    int seg;  // segment of the sequence
+    int cl;   // chunk within the segment
 };
-__device__ __forceinline__ StreamPos stream_pos(int v, int N, int nh, int lognv) {
-    const int per = N * nh;
+// Units are (sequence, segment, value slice), the value slice fastest (the two
+// slices of a sequence read the same q, k and gates); a unit covers seg_len chunks.
+__device__ __forceinline__ StreamPos stream_pos(int v, int L, int nh, int lognv, int nsu) {
+    const int per = L * nh;
     const int j = v / per, rem = v - j * per;
     const int unit = static_cast<int>(blockIdx.x) + j * static_cast<int>(gridDim.x);
-    const int c = rem / nh;
-    return {unit >> lognv, unit & ((1 << lognv) - 1), c, rem - c * nh};
+    const int rest = unit >> lognv;
+    const int seg = nsu == 1 ? 0 : rest % nsu;
+    const int bh = nsu == 1 ? rest : rest / nsu;
+    const int cl = rem / nh;
+    return {bh, unit & ((1 << lognv) - 1), seg * L + cl, rem - cl * nh, seg, cl};
 }
 
 // Visit the TMA load boxes of one chunk: calls f(map height index, smem row, c2, c3).
@@ -365,7 +381,7 @@ __device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *op
     }
 }
 
-template <typename E, int NH, int NV>
+template <typename E, int NH, int NV, int MODE>
 __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_constant__ TcParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -380,14 +396,20 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     volatile uint32_t *mode_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMode);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // MODE kFull / kSplitFull: outputs (a split sequence's later segments start from
+    // the state folded from the segment summaries).  MODE kSummary: per segment only
+    // the end state from zero and the total decay (k, v and gates; no scores or outputs).
+    constexpr bool kSum = MODE == kSummary;
+    constexpr bool kSplit = MODE != kFull;
     const int N = p.n_chunks;   // chunks per sequence
+    const int L = p.seg_len;    // chunks per unit
     constexpr int nh = NH;   // 64-channel key halves per chunk (Dk / 64)
     constexpr int lognv = NV - 1;  // 64-column value slices per sequence (Dv / 64): 1 or 2
     constexpr int kDk = 64 * NH, kDv = 64 * NV;
     // this CTA's stream of virtual chunks: every barrier phase, stage slot and TMEM
     // buffer below follows the stream index (O: the real chunk's index), so
     // consecutive units flow through one pipeline
-    const int G = N * nh *
+    const int G = L * nh *
                   ((p.n_units - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
                    static_cast<int>(gridDim.x));
     const int rev = p.order & 1;
@@ -445,7 +467,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             int issued = 0;
             for (int g = 0; g < G; ++g) {
                 const int sl = g % kSlots;
-                const StreamPos ps = stream_pos(g, N, nh, lognv);
+                const StreamPos ps = stream_pos(g, L, nh, lognv, kSplit ? p.nsu : 1);
                 const int b = ps.bh / p.H, h = ps.bh % p.H, c = ps.c;
                 const int xk = 64 * ps.a, xv = 64 * ps.vb;  // channel offsets of the key half, value slice
                 if (!mbar_wait(&bars[BAR_EMPTY + sl], ((g / kSlots) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
@@ -454,9 +476,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
                 uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
                 uint64_t *fb = &bars[BAR_FULL + sl];
-                mbar_arrive_expect_tx(fb, kSlotBytes);
+                mbar_arrive_expect_tx(fb, kSum ? kSlotBytes - kTile16 : kSlotBytes);  // summaries need no q
                 chunk_load_boxes(p.order, p.T, p.grid_h, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
-                    tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, xk, h, c2, c3, b);
+                    if (!kSum) tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, xk, h, c2, c3, b);
                     tma_load_5d(st + kK + row * 128, &p.maps[T_K][hi], fb, xk, h, c2, c3, b);
                     tma_load_5d(st + kV + row * 128, &p.maps[T_V][hi], fb, xv, h, c2, c3, b);
                     tma_load_5d(st + kG + row * 128, &p.maps[T_G][hi], fb, xk, h, c2, c3, b);
@@ -508,7 +530,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 const uint32_t st = slot0 + su * kSlotBytes;
                 const uint32_t mode = __shfl_sync(0xffffffffu, mode_s[su], 0);
                 const uint32_t dp = tmem + kColP + (i & 1) * 64;
-                if (mode == kModeF16) {
+                if (kSum) {
+                    // summaries need no scores
+                } else if (mode == kModeF16) {
                     const uint64_t dq = kdesc(st + kQ), dk = kdesc(st + kK);
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(dp, dq + 2 * ks, dk + 2 * ks, idesc_p16, ks > 0);
@@ -530,6 +554,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(du, dk + 128 * ks, dv + 128 * ks, idesc_u, ks > 0);
                 mma_commit_warp(&bars[BAR_UFULL + (i & 1)]);
+                if (kSum) mma_commit_warp(&bars[BAR_EMPTY + su]);  // U is the stage's last reader
                 su = (su == kSlots - 1) ? 0 : su + 1;
                 if (i + 2 < G) {
                     ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + sa], ((i + 2) / kSlots) & 1, abort_flag, kWaitLimitNs));
@@ -543,7 +568,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
                 sa = (sa == kSlots - 1) ? 0 : sa + 1;
             }
-            if (i >= 1) {
+            if (!kSum && i >= 1) {
                 const int c = i - 1;
                 ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_ORDY + (c & 1)], (c >> 1) & 1, abort_flag, kWaitLimitNs));
                 if (!ok) break;
@@ -661,7 +686,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     const float amv[8] = {am0.x * kLog2e, am0.y * kLog2e, am0.z * kLog2e, am0.w * kLog2e,
                                           am1.x * kLog2e, am1.y * kLog2e, am1.z * kLog2e, am1.w * kLog2e};
                     const uint32_t o16 = sw128(row, cl * 2);
-                    const uint4 qw = *reinterpret_cast<const uint4 *>(tq + o16);
+                    const uint4 qw = kSum ? make_uint4(0u, 0u, 0u, 0u) : *reinterpret_cast<const uint4 *>(tq + o16);
                     const uint4 kw = *reinterpret_cast<const uint4 *>(tk + o16);
                     const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w}, ka[4] = {kw.x, kw.y, kw.z, kw.w};
                     uint32_t qo[4], ko[4];
@@ -674,7 +699,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         ko[e] = h2bits(k2.x * ex2(-e0), k2.y * ex2(-e1));
                     }
                     // Q^ over q, K^ over k (each thread rewrites exactly what it read)
-                    *reinterpret_cast<uint4 *>(tq + o16) = make_uint4(qo[0], qo[1], qo[2], qo[3]);
+                    if (!kSum) *reinterpret_cast<uint4 *>(tq + o16) = make_uint4(qo[0], qo[1], qo[2], qo[3]);
                     *reinterpret_cast<uint4 *>(tk + o16) = make_uint4(ko[0], ko[1], ko[2], ko[3]);
                 }
             } else if (!opfail) {
@@ -705,6 +730,10 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (tg == 0) mbar_arrive(&bars[BAR_REFS + sl]);  // constants and mode of chunk c -> epi
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // operands in smem, A(c) read
+            if (kSum) {  // no scores: the scratch buffer is free once the operands are built
+                if (tg == 0) atomicMax(op_done, (uint32_t)c + 1u);
+                continue;
+            }
             // ---- masked scores of chunk c over its gate tile (consumed by A(c) long ago)
             const bool pfail = !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
             if (named_barrier_or(bar_id, 128, pfail)) {
@@ -750,6 +779,28 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 #pragma unroll
             for (int j = 0; j < 32; ++j) So[j] = 0.f;
         }
+        float dp = 1.f, dpo = 1.f;  // summaries: the segment's decay product per key half
+        // Start state of a split sequence's segment seg > 0 (key half `half`): fold the
+        // end states from zero of segments 0 .. seg-1 with their total decays,
+        // S_start(s + 1) = Diag(D_s) S_start(s) + S_end(s).
+        const size_t sum_stride = (size_t)kDk * kDv + kDk;
+        auto start_state = [&](float(&st)[32], int half, const StreamPos &q) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) st[j] = 0.f;
+            const float *base = p.summary + (size_t)q.bh * (p.nseg - 1) * sum_stride;
+            for (int s2 = 0; s2 < q.seg; ++s2, base += sum_stride) {
+                const float d = base[(size_t)kDk * kDv + 64 * half + row];
+                const float4 *x = reinterpret_cast<const float4 *>(base + (size_t)(64 * half + row) * kDv + 64 * q.vb + ch0);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    const float4 w = x[j];
+                    st[4 * j] = fmaf(d, st[4 * j], w.x);
+                    st[4 * j + 1] = fmaf(d, st[4 * j + 1], w.y);
+                    st[4 * j + 2] = fmaf(d, st[4 * j + 2], w.z);
+                    st[4 * j + 3] = fmaf(d, st[4 * j + 3], w.w);
+                }
+            }
+        };
         bool ok = true;
         if (lane == 0) {  // TMEM U buffers start out free: the drains of chunks -2 and -1
             mbar_arrive(&bars[BAR_PURDY + 0]);
@@ -759,15 +810,25 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (c < G) {
                 const int sl = c % kSlots, bb = c & 1;
                 const uint32_t ph = (c >> 1) & 1;
-                const StreamPos ps = stream_pos(c, N, nh, lognv);
-                if (ps.c == 0) {  // a new sequence starts from S = 0
+                const StreamPos ps = stream_pos(c, L, nh, lognv, kSplit ? p.nsu : 1);
+                if (ps.cl == 0 && ps.a == 0) {  // a unit starts: its state (every key half)
+                    if (!kSplit || kSum || ps.seg == 0) {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) S[j] = 0.f;
+                        for (int j = 0; j < 32; ++j) S[j] = 0.f;
+                        if constexpr (NH == 2) {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) So[j] = 0.f;
+                        }
+                    } else if constexpr (kSplit) {
+                        start_state(S, 0, ps);
+                        if constexpr (NH == 2) start_state(So, 1, ps);
+                    }
+                    dp = dpo = 1.f;
                 }
                 bool fail = !mbar_wait(&bars[BAR_REFS + sl], (c / kSlots) & 1, abort_flag, kWaitLimitNs);
                 // buffer bb was last read by O(c-2) (one key half: observed by the readout of
                 // the previous iteration already)
-                if (NH == 2 && c >= 2)
+                if (!kSum && NH == 2 && c >= 2)
                     fail = fail || !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs);
                 if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
                     ok = false;
@@ -778,16 +839,18 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 const float c1 = fold ? ref[3 * kD + row] : 1.f;
                 const float c2 = fold ? ref[4 * kD + row] : 1.f;
                 const float dc = decay_s[sl * kD + row];
-                // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout)
-                uint8_t *sb = smem + kOffS + bb * kTile16;
+                if (!kSum) {
+                    // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout)
+                    uint8_t *sb = smem + kOffS + bb * kTile16;
 #pragma unroll
-                for (int q = 0; q < 4; ++q)
-                    *reinterpret_cast<uint4 *>(sb + sw128(row, (ch0 + 8 * q) * 2)) =
-                        make_uint4(h2bits(S[8 * q + 0] * c1, S[8 * q + 1] * c1), h2bits(S[8 * q + 2] * c1, S[8 * q + 3] * c1),
-                                   h2bits(S[8 * q + 4] * c1, S[8 * q + 5] * c1), h2bits(S[8 * q + 6] * c1, S[8 * q + 7] * c1));
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // with the outputs of c-2 read out
+                    for (int q = 0; q < 4; ++q)
+                        *reinterpret_cast<uint4 *>(sb + sw128(row, (ch0 + 8 * q) * 2)) = make_uint4(
+                            h2bits(S[8 * q + 0] * c1, S[8 * q + 1] * c1), h2bits(S[8 * q + 2] * c1, S[8 * q + 3] * c1),
+                            h2bits(S[8 * q + 4] * c1, S[8 * q + 5] * c1), h2bits(S[8 * q + 6] * c1, S[8 * q + 7] * c1));
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // with the outputs of c-2 read out
+                }
                 // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
                 fail = !mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs);
                 if (__any_sync(0xffffffffu, fail)) {
@@ -802,7 +865,16 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 #pragma unroll
                 for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
                 tc_fence_before();
-                if (ps.c == N - 1 && p.final_state != nullptr) {  // the sequence's final state
+                if (kSum) {
+                    dp *= dc;
+                    if (ps.cl == L - 1) {  // the segment's summary
+                        float *base = p.summary + ((size_t)ps.bh * (p.nseg - 1) + ps.seg) * sum_stride;
+                        float4 *dst = reinterpret_cast<float4 *>(base + (size_t)(64 * ps.a + row) * kDv + 64 * ps.vb + ch0);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
+                        if (ps.vb == 0 && hc == 0) base[(size_t)kDk * kDv + 64 * ps.a + row] = dp;
+                    }
+                } else if (ps.c == N - 1 && p.final_state != nullptr) {  // the sequence's final state
                     float4 *dst = reinterpret_cast<float4 *>(
                         p.final_state + ((size_t)ps.bh * kDk + 64 * ps.a + row) * kDv + 64 * ps.vb + ch0);
 #pragma unroll
@@ -817,9 +889,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         S[j] = So[j];
                         So[j] = t;
                     }
+                    const float t = dp;
+                    dp = dpo;
+                    dpo = t;
                 }
             }
-            if (c >= nh && c % nh == 0) {
+            if (!kSum && c >= nh && c % nh == 0) {
                 // outputs of the real chunk whose last key half is c-1
                 const int co = c - 1, ob = (co / nh) & 1;
                 const bool fail = !mbar_wait(&bars[BAR_OFULL + (co & 1)], (co >> 1) & 1, abort_flag, kWaitLimitNs);
@@ -833,7 +908,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
                 tmem_ld_wait();
                 tc_fence_before();
-                const StreamPos po = stream_pos(co, N, nh, lognv);
+                const StreamPos po = stream_pos(co, L, nh, lognv, kSplit ? p.nsu : 1);
                 const int b = po.bh / p.H, h = po.bh % p.H;
                 const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
                 if (t >= 0) {
@@ -950,23 +1025,55 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     return true;
 }
 
-template <typename E, int NH, int NV>
+template <typename E, int NH, int NV, int MODE>
 cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
     cudaError_t e =
-        cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return e;
-    gla_tc_kernel<E, NH, NV><<<grid, kThreads, kSmemBytes, stream>>>(tp);
+    gla_tc_kernel<E, NH, NV, MODE><<<grid, kThreads, kSmemBytes, stream>>>(tp);
     return cudaSuccess;
 }
 
-// One instantiation per (element type, key halves, value slices).
-template <typename E>
+// One instantiation per (element type, key halves, value slices, pass).
+template <typename E, int MODE>
 cudaError_t launch_shape(dim3 grid, const TcParams &tp, cudaStream_t stream) {
-    if (tp.nh == 1) return tp.nv == 1 ? launch_kernel<E, 1, 1>(grid, tp, stream) : launch_kernel<E, 1, 2>(grid, tp, stream);
-    return tp.nv == 1 ? launch_kernel<E, 2, 1>(grid, tp, stream) : launch_kernel<E, 2, 2>(grid, tp, stream);
+    if (tp.nh == 1)
+        return tp.nv == 1 ? launch_kernel<E, 1, 1, MODE>(grid, tp, stream) : launch_kernel<E, 1, 2, MODE>(grid, tp, stream);
+    return tp.nv == 1 ? launch_kernel<E, 2, 1, MODE>(grid, tp, stream) : launch_kernel<E, 2, 2, MODE>(grid, tp, stream);
+}
+
+cudaError_t sm_count(int *n_sm) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    return cudaDeviceGetAttribute(n_sm, cudaDevAttrMultiProcessorCount, dev);
+}
+
+// Segments per sequence.  A launch whose work units fill fewer than half of the
+// SMs splits every sequence into the most equal segments (a divisor of the chunk
+// count, at least kMinSegChunks chunks each) that still fit one wave.
+int choose_nseg(const Problem &p, int n_sm) {
+    const long long N = (p.T + kC - 1) / kC;
+    const long long units = (long long)p.B * p.H * (p.Dv / 64);
+    if (units * 2 > n_sm) return 1;
+    int best = 1;
+    for (long long d = 2; d <= N; ++d)
+        if (N % d == 0 && N / d >= kMinSegChunks && units * d <= n_sm) best = static_cast<int>(d);
+    return best;
+}
+
+size_t summary_bytes(const Problem &p, int nseg) {
+    if (nseg <= 1) return 0;
+    return (size_t)p.B * p.H * (nseg - 1) * ((size_t)p.Dk * p.Dv + p.Dk) * sizeof(float);
 }
 
 }  // namespace
+
+size_t tc_workspace_bytes(const Problem &p) {
+    int n_sm = 0;
+    if (sm_count(&n_sm) != cudaSuccess) return 0;
+    return summary_bytes(p, choose_nseg(p, n_sm));
+}
 
 bool tc_supported(const Problem &p) {
     if (p.dtype != 1 && p.dtype != 2) return false;       // fp16 / bf16 operands only
@@ -977,9 +1084,12 @@ bool tc_supported(const Problem &p) {
     return get_encode() != nullptr;
 }
 
-cudaError_t launch_tc(const Problem &p, cudaStream_t stream) {
+cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes) {
     TcParams tp;
     if (!get_maps(p, tp.maps)) return cudaErrorInvalidValue;
+    int n_sm = 0;
+    cudaError_t e = sm_count(&n_sm);
+    if (e != cudaSuccess) return e;
     tp.out = p.out;
     tp.final_state = p.final_state;
     tp.H = p.H;
@@ -992,16 +1102,30 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream) {
     tp.Dv = p.Dv;
     tp.nh = p.Dk / 64;
     tp.nv = p.Dv / 64;
-    tp.n_units = static_cast<int>(p.B * p.H) * tp.nv;
+    int nseg = choose_nseg(p, n_sm);
+    if (nseg > 1 && (workspace == nullptr || workspace_bytes < summary_bytes(p, nseg))) nseg = 1;
+    tp.nseg = nseg;
+    tp.seg_len = tp.n_chunks / nseg;
+    tp.summary = static_cast<float *>(workspace);
+    const int seqs = static_cast<int>(p.B * p.H) * tp.nv;  // (sequence, value slice) pairs
+    const bool half = p.dtype == 1;
     // persistent: one CTA per SM, each walking its share of the work units
-    int dev = 0, n_sm = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return e;
-    const int n_cta = tp.n_units < n_sm ? tp.n_units : n_sm;
-    const dim3 grid(static_cast<unsigned>(n_cta));
-    e = p.dtype == 1 ? launch_shape<__half>(grid, tp, stream) : launch_shape<__nv_bfloat16>(grid, tp, stream);
+    if (nseg > 1) {  // pass 1: end state from zero and total decay of segments 0 .. nseg-2
+        tp.nsu = nseg - 1;
+        tp.n_units = seqs * tp.nsu;
+        const dim3 grid(static_cast<unsigned>(tp.n_units < n_sm ? tp.n_units : n_sm));
+        e = half ? launch_shape<__half, kSummary>(grid, tp, stream) : launch_shape<__nv_bfloat16, kSummary>(grid, tp, stream);
+        if (e != cudaSuccess) return e;
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    tp.nsu = nseg;
+    tp.n_units = seqs * nseg;
+    const dim3 grid(static_cast<unsigned>(tp.n_units < n_sm ? tp.n_units : n_sm));
+    if (nseg > 1)
+        e = half ? launch_shape<__half, kSplitFull>(grid, tp, stream)
+                 : launch_shape<__nv_bfloat16, kSplitFull>(grid, tp, stream);
+    else
+        e = half ? launch_shape<__half, kFull>(grid, tp, stream) : launch_shape<__nv_bfloat16, kFull>(grid, tp, stream);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

@@ -53,6 +53,10 @@ def load(path: Optional[str] = None):
         lib.gtr_gla_fwd_sched.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, ci, vp]
         lib.gtr_gla_tc_supported.restype = ci
         lib.gtr_gla_tc_supported.argtypes = [ci] * 8
+        lib.gtr_gla_workspace_bytes.restype = st
+        lib.gtr_gla_workspace_bytes.argtypes = [ci] * 7
+        lib.gtr_gla_fwd_ws.restype = ci
+        lib.gtr_gla_fwd_ws.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp, st, vp]
         lib.gtr_gla_host_buffer_bytes.restype = st
         lib.gtr_gla_host_buffer_bytes.argtypes = [ci] * 8
         lib.gtr_gla_fwd_host.restype = ci
@@ -129,6 +133,29 @@ def forward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.T
         SCHEDULES[schedule], _stream_ptr(stream))
     _check(status, "gtr_gla_fwd", lib)
     return out, fs
+
+
+def workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype: torch.dtype) -> int:
+    """Device workspace ``forward_ws`` needs for these arguments (0: none)."""
+    return int(load().gtr_gla_workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, _DTYPES[dtype]))
+
+
+def forward_ws(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,
+               grid_h: int, grid_w: int, order: int, out: torch.Tensor,
+               final_state: Optional[torch.Tensor], workspace: Optional[torch.Tensor],
+               stream: Optional[torch.cuda.Stream] = None) -> None:
+    """Forward through ``gtr_gla_fwd_ws`` with a caller-owned device workspace (a
+    CUDA uint8 tensor of at least workspace_bytes(), or None when that is 0)."""
+    lib = load()
+    B, H, Dk, Dv = _dims(q, v, grid_h, grid_w)
+    status = lib.gtr_gla_fwd_ws(
+        q.data_ptr(), k.data_ptr(), v.data_ptr(), log_gate.data_ptr(), B, H, grid_h, grid_w, Dk,
+        Dv, order, _DTYPES[q.dtype], out.data_ptr(),
+        final_state.data_ptr() if final_state is not None else None,
+        workspace.data_ptr() if workspace is not None else None,
+        workspace.numel() * workspace.element_size() if workspace is not None else 0,
+        _stream_ptr(stream))
+    _check(status, "gtr_gla_fwd_ws", lib)
 
 
 def host_buffer_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype: torch.dtype, with_final_state=True):

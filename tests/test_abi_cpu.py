@@ -36,7 +36,7 @@ def declared_functions():
 def test_header_declares_entry_points():
     names = declared_functions()
     for must in ("gtr_gla_fwd", "gtr_gla_fwd_sched", "gtr_gla_fwd_host", "gtr_gla_sync_status",
-                 "gtr_status_string"):
+                 "gtr_status_string", "gtr_gla_workspace_bytes", "gtr_gla_fwd_ws"):
         assert must in names
 
 
@@ -93,3 +93,13 @@ def test_host_buffer_bytes(lib):
 def test_tc_support_query_is_host_only(lib):
     assert lib.gtr_gla_tc_supported(1, 1, 8, 8, 64, 64, 0, 0) == 0    # fp32 never on tensor cores
     assert lib.gtr_gla_tc_supported(1, 1, 8, 8, 0, 64, 0, 1) == 0     # invalid shape
+
+
+def test_workspace_entry_point_validates_before_any_launch(lib):
+    # invalid shapes ask for no workspace; a misaligned workspace is rejected
+    assert lib.gtr_gla_workspace_bytes(1, 1, 0, 8, 64, 64, 1) == 0
+    assert lib.gtr_gla_workspace_bytes(1, 1, 8, 8, 64, 64, 7) == 0
+    assert lib.gtr_gla_fwd_ws(16, 16, 16, 16, 1, 1, 8, 8, 64, 64, 0, 1, 16, None, 8, 0, None) == 1
+    # an empty batch needs neither inputs nor a workspace
+    assert lib.gtr_gla_fwd_ws(None, None, None, None, 0, 4, 8, 8, 64, 64, 0, 1, None, None, None,
+                              0, None) == 0

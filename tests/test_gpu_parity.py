@@ -144,6 +144,45 @@ def test_many_sequences_per_cta(case):
         assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, dtype, f"state {order}")
 
 
+# Few, long sequences: the tensor-core schedule splits each into equal segments
+# (a summary pass, then every segment from the fold of the earlier summaries).
+SPLIT = [
+    (1, 2, 64, 64, 64, 64, "bf16", 16.0, 0.0, 0.0),     # 8 segments of 8 chunks
+    (1, 1, 48, 40, 64, 64, "f16", 1.0, -1.0, 0.0),      # strong decay: tf32 scores in both passes
+    (1, 1, 32, 32, 128, 128, "bf16", 16.0, 0.0, 0.0),   # two key halves, two value slices
+    (1, 1, 64, 16, 128, 64, "f16", 16.0, 0.0, 0.02),    # Dk != Dv, some gamma = 0 gates (exact path)
+]
+
+
+@pytest.mark.parametrize("case", SPLIT, ids=[f"{c[0]}x{c[1]}-{c[2]}x{c[3]}-d{c[4]}_{c[5]}-{c[6]}"
+                                             for c in SPLIT])
+def test_split_sequences(case):
+    B, H, gh, gw, Dk, Dv, dtype, tau, zm, frac_zero = case
+    ws_bytes = gla.workspace_bytes(B, H, gh, gw, Dk, Dv, TORCH_DT[dtype])
+    assert ws_bytes > 0, "the schedule should split these sequences"
+    inp = wl.make_inputs(B, H, gh, gw, Dk, Dv, dtype, seed=4000 + SPLIT.index(case), tau=tau,
+                         z_mean=zm)
+    if frac_zero > 0:
+        rng = np.random.Generator(np.random.PCG64(77))
+        g = wl.storage_to_f64(inp["g"], dtype)
+        g[rng.random(g.shape) < frac_zero] = -np.inf
+        inp["g"] = wl.round_to_storage(g, dtype)
+    f = inputs_f64(inp, dtype)
+    t = {n: to_torch(inp[n], dtype) for n in ("q", "k", "v", "g")}
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    for order in wl.ALL_ORDERS:
+        ref_o, ref_s = oracle.recurrence(f["q"], f["k"], f["v"], f["g"], gh, gw, order)
+        out, fs = _run(inp, dtype, gh, gw, order, "tc")  # internal workspace
+        assert_within_bar(_np(out), ref_o, dtype, f"out order {order}")
+        assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, dtype, f"state {order}")
+        out2 = torch.empty_like(t["v"])
+        fs2 = torch.empty_like(fs)
+        gla.forward_ws(t["q"], t["k"], t["v"], t["g"], gh, gw, order, out2, fs2, ws)
+        torch.cuda.synchronize()
+        assert gla.sync_status() == 0
+        assert torch.equal(out2, out) and torch.equal(fs2, fs)  # same schedule, same bits
+
+
 @pytest.mark.parametrize("dtype", ["f16", "bf16", "f32"])
 @pytest.mark.parametrize("gate", ["one", "zero"])
 def test_gate_extremes(dtype, gate):
