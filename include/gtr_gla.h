@@ -131,6 +131,43 @@ gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const v
                             float *final_state, void *workspace, size_t workspace_bytes,
                             cudaStream_t stream);
 
+/* Size of the fixed device scratch array behind gtr_gla_fwd_noalloc.  The
+ * library holds one such array on every GPU where it is loaded, from the
+ * module's load until the process exits.  The split schedule needs at most
+ * B*H*(segments-1) summaries of (Dk*Dv + Dk) floats, with segments bounded by
+ * the SM count: about 5 MB on a 152-SM device. */
+#define GTR_GLA_NOALLOC_SCRATCH_BYTES (8u << 20)
+
+/* gtr_gla_fwd for callers that must not allocate device memory on the call
+ * path.  One example is an engine that reserves all of HBM for its own pool at
+ * start-up.  Another is a latency-critical loop: cudaFree synchronises the
+ * whole device, and cudaMalloc can.  gtr_gla_fwd may cudaMalloc its internal
+ * workspace, and gtr_gla_fwd_ws needs a buffer that the caller owns.  This
+ * call uses neither.  The paper has no counterpart; it changes only where the
+ * segment summaries of the split schedule are kept.
+ *
+ * Arguments, results and errors are those of gtr_gla_fwd.  The summaries go to
+ * a fixed array of GTR_GLA_NOALLOC_SCRATCH_BYTES in this library.  A problem
+ * whose gtr_gla_workspace_bytes() exceeds that returns GTR_ERR_WORKSPACE before
+ * anything is launched.  The call allocates no device memory and does not
+ * synchronise.
+ *
+ * Set-up: the first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current).  Make that first call
+ * before capturing any stream on that device; a failed lookup returns
+ * GTR_ERR_CUDA.
+ *
+ * Every call on a device shares the one array, and it keeps what the last call
+ * wrote.  Nothing in it must start at zero: the first kernel of a call writes
+ * every summary that the call's second kernel reads.  Calls whose kernels
+ * overlap on the GPU race on the array and give wrong results, for example
+ * calls on two streams with no ordering between them.  Order them on one
+ * stream or with events. */
+gtr_status_t gtr_gla_fwd_noalloc(const void *q, const void *k, const void *v, const void *log_gate,
+                                 int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                                 gtr_scan_t scan_order, gtr_dtype_t dtype, void *out,
+                                 float *final_state, cudaStream_t stream);
+
 /* 1 when the tensor-core schedule supports these arguments, else 0: fp16 or
  * bf16, Dk and Dv each 64 or 128 (processed in 64-channel key halves and
  * 64-column value slices), T = grid_h * grid_w a multiple of 8, and for the

@@ -1,5 +1,6 @@
 // gla_api.cu -- the C ABI of include/gtr_gla.h: argument validation, schedule
-// dispatch, the host-memory entry point and status reporting.  No kernel code.
+// dispatch, the host-memory entry point and status reporting.  No kernel code;
+// one device array, the scratch of gtr_gla_fwd_noalloc.
 #include <cstdint>
 #include <cstring>
 #include <mutex>
@@ -7,6 +8,12 @@
 
 #include "gla_internal.h"
 #include "gtr_gla.h"
+
+// Segment summaries of gtr_gla_fwd_noalloc, for callers that may not allocate
+// device memory.  Every device that loads this library holds one copy until the
+// process exits.  Host code reaches it only through the address that
+// noalloc_scratch() looks up.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[GTR_GLA_NOALLOC_SCRATCH_BYTES];
 
 namespace {
 
@@ -112,6 +119,28 @@ void *internal_workspace(size_t need, cudaStream_t stream, size_t *got) {
     return w.ptr;
 }
 
+// Device address of g_noalloc_scratch on the current device, looked up on the
+// first call per device and kept (null: not looked up yet).
+std::mutex g_noalloc_mutex;
+std::vector<void *> g_noalloc_ptr;
+
+cudaError_t noalloc_scratch(void **ptr) {
+    *ptr = nullptr;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if ((size_t)dev >= g_noalloc_ptr.size()) g_noalloc_ptr.resize(dev + 1, nullptr);
+    if (g_noalloc_ptr[dev] == nullptr) {
+        void *addr = nullptr;
+        e = cudaGetSymbolAddress(&addr, g_noalloc_scratch);
+        if (e != cudaSuccess) return e;
+        g_noalloc_ptr[dev] = addr;
+    }
+    *ptr = g_noalloc_ptr[dev];
+    return cudaSuccess;
+}
+
 // Dispatch of one validated, non-empty problem; `ws` null means the internal workspace.
 gtr_status_t dispatch(const gtr::Problem &p, gtr_schedule_t schedule, void *ws, size_t ws_bytes, bool own_ws,
                       cudaStream_t stream) {
@@ -165,6 +194,25 @@ gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const v
     const size_t need = gtr_gla_workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype);
     if (need > 0 && (workspace == nullptr || workspace_bytes < need)) return GTR_ERR_WORKSPACE;
     return dispatch(p, GTR_SCHED_AUTO, workspace, workspace_bytes, true, stream);
+}
+
+gtr_status_t gtr_gla_fwd_noalloc(const void *q, const void *k, const void *v, const void *log_gate,
+                                 int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                                 gtr_scan_t scan_order, gtr_dtype_t dtype, void *out,
+                                 float *final_state, cudaStream_t stream) {
+    gtr::Problem p;
+    gtr_status_t st = make_problem(q, k, v, log_gate, B, H, grid_h, grid_w, Dk, Dv, scan_order,
+                                   dtype, out, final_state, &p);
+    if (st != GTR_OK) return st;
+    if (B == 0 || H == 0) return GTR_OK;
+    if (gtr_gla_workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype) > GTR_GLA_NOALLOC_SCRATCH_BYTES)
+        return GTR_ERR_WORKSPACE;
+    void *scratch = nullptr;
+    const cudaError_t e = noalloc_scratch(&scratch);
+    if (e != cudaSuccess) return cuda_fail(e);
+    // The summary pass writes every summary the output pass reads, so what an
+    // earlier call left in the array is never read and nothing is cleared.
+    return dispatch(p, GTR_SCHED_AUTO, scratch, GTR_GLA_NOALLOC_SCRATCH_BYTES, true, stream);
 }
 
 gtr_status_t gtr_gla_fwd(const void *q, const void *k, const void *v, const void *log_gate, int B,

@@ -57,6 +57,8 @@ def load(path: Optional[str] = None):
         lib.gtr_gla_workspace_bytes.argtypes = [ci] * 7
         lib.gtr_gla_fwd_ws.restype = ci
         lib.gtr_gla_fwd_ws.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp, st, vp]
+        lib.gtr_gla_fwd_noalloc.restype = ci
+        lib.gtr_gla_fwd_noalloc.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp]
         lib.gtr_gla_host_buffer_bytes.restype = st
         lib.gtr_gla_host_buffer_bytes.argtypes = [ci] * 8
         lib.gtr_gla_fwd_host.restype = ci
@@ -156,6 +158,22 @@ def forward_ws(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torc
         workspace.numel() * workspace.element_size() if workspace is not None else 0,
         _stream_ptr(stream))
     _check(status, "gtr_gla_fwd_ws", lib)
+
+
+def forward_noalloc(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,
+                    grid_h: int, grid_w: int, order: int, out: torch.Tensor,
+                    final_state: Optional[torch.Tensor],
+                    stream: Optional[torch.cuda.Stream] = None) -> None:
+    """Forward through ``gtr_gla_fwd_noalloc``: no device memory is allocated;
+    split-schedule summaries go to the library's fixed scratch array, which all
+    calls on a device share (calls that overlap on the GPU race)."""
+    lib = load()
+    B, H, Dk, Dv = _dims(q, v, grid_h, grid_w)
+    status = lib.gtr_gla_fwd_noalloc(
+        q.data_ptr(), k.data_ptr(), v.data_ptr(), log_gate.data_ptr(), B, H, grid_h, grid_w, Dk,
+        Dv, order, _DTYPES[q.dtype], out.data_ptr(),
+        final_state.data_ptr() if final_state is not None else None, _stream_ptr(stream))
+    _check(status, "gtr_gla_fwd_noalloc", lib)
 
 
 def host_buffer_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype: torch.dtype, with_final_state=True):

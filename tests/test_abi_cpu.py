@@ -103,3 +103,14 @@ def test_workspace_entry_point_validates_before_any_launch(lib):
     # an empty batch needs neither inputs nor a workspace
     assert lib.gtr_gla_fwd_ws(None, None, None, None, 0, 4, 8, 8, 64, 64, 0, 1, None, None, None,
                               0, None) == 0
+
+
+def test_noalloc_entry_point_validates_before_any_launch(lib):
+    # bad arguments are rejected before the scratch array is looked up
+    assert lib.gtr_gla_fwd_noalloc(None, 16, 16, 16, 1, 1, 8, 8, 64, 64, 0, 1, 16, None,
+                                   None) == 1
+    assert lib.gtr_gla_fwd_noalloc(16, 16, 16, 16, 1, 1, 8, 8, 64, 64, 5, 1, 16, None,
+                                   None) == 1
+    # an empty batch launches nothing and needs no device
+    assert lib.gtr_gla_fwd_noalloc(None, None, None, None, 0, 4, 8, 8, 64, 64, 0, 1, None, None,
+                                   None) == 0
