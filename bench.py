@@ -254,6 +254,11 @@ def main():
     schedule = args.schedule
     tc = gla.tc_supported(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, orders[0], dt)
     kernel_name = "tensor-core chunkwise (tcgen05/TMEM/TMA)" if (tc and schedule != "simt") else "simt recurrence"
+    # a split schedule runs a summary pass before the output pass: two launches a step
+    split = tc and schedule != "simt" and gla.workspace_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt) > 0
+    launches_per_step = 2 if split else 1
+    if split:
+        kernel_name += ", segment-summary pass + output pass"
 
     def step(i):
         gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, orders[i % len(orders)],
@@ -361,7 +366,7 @@ def main():
                 "dtype": w.dtype, "data": "synthetic (seeded, workload recipe in workloads.py)",
                 "config": workload_config(w, world, {"schedule": schedule}),
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-                "gpu_launches": args.steps, "clocks": clk.summary(),
+                "gpu_launches": args.steps * launches_per_step, "clocks": clk.summary(),
                 "token_heads_per_s": value * w.H}
         print(json.dumps(line), flush=True)
     if pg:
