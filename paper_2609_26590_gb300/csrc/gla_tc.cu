@@ -28,23 +28,27 @@
 // Memory: each chunk owns a 32 KB stage slot (q, k, v, g tiles) from its TMA
 // load until its output product completes; the derived fp16 operands are
 // written in place (Q^ or Qtil over q, K^ or Kbar over k, the masked scores P
-// over g, bf16 v converted to fp16 in place), so five chunks can be in flight.
-// Only the tf32 score operands use a separate buffer, freed as soon as P is
-// done.  Row orders load one 64-row TMA box per tensor and chunk; column orders
+// over g, bf16 v converted to fp16 in place), so four chunks can be in flight.
+// Only the tf32 score operands use separate buffers, one per gen warpgroup, so
+// that tf32-mode chunks of the two groups never wait for each other.  Row orders load one 64-row TMA box per tensor and chunk; column orders
 // one box per column segment of the chunk, of the segment's exact height (a
 // tensor map per height).  The scan permutation lives in the box coordinates of
 // the loads and in the addresses of the output stores.
 //
-// Warp roles (448 threads, one CTA per SM).  Few roles with small loops keep
-// the hot code inside the SM's instruction cache:
+// Warp roles (512 threads, one CTA per SM; four warps per SM sub-partition, so a
+// thread keeps 128 registers).  Few roles with small loops keep the hot code
+// inside the SM's instruction cache:
 //   warp 0       TMA producer.
-//   warp 1       TMEM allocator and MMA issuer: issues every product (A, P, U, O)
-//                in a fixed software-pipelined order, one barrier wait per stage.
+//   warp 1       TMEM allocator and issuer of A(c) = L G.
 //   warps 2-5    gen warpgroup 0 (even chunks): reads A, builds the operands of its
 //                chunk, then masks the chunk's scores P into fp16.
 //   warps 6-9    gen warpgroup 1 (odd chunks).
 //   warps 10-13  epi: carries the fp32 state S in registers, writes Diag(c1) S,
 //                and stores each chunk's outputs at the tokens' spatial positions.
+//   warp 14      issuer of P(c) and U(c).
+//   warp 15      issuer of O(c).
+// Each issuer waits only for the inputs of its own product, so the issue overhead
+// of one product does not hold up the others.
 // A warp reads the TMEM lanes of sub-partition (warp % 4); an M = 64 accumulator
 // keeps rows 16q..16q+15 in lanes 32q..32q+15, and each thread takes one row and
 // 32 of its 64 columns.
@@ -71,10 +75,10 @@ using namespace ptx;
 
 constexpr int kC = 64;                    // chunk length
 constexpr int kD = 64;                    // Dk = Dv handled by this kernel
-constexpr int kSlots = 5;                 // stage slots (chunks in flight)
+constexpr int kSlots = 4;                 // stage slots (chunks in flight)
 constexpr int kTile16 = kC * kD * 2;      // 64 x 64 16-bit tile (SW128, 128-byte rows)
 constexpr int kTile32 = kC * kD * 4;      // 64 x 64 fp32 tile (two 32-column K-blocks)
-constexpr int kThreads = 448;
+constexpr int kThreads = 512;
 constexpr int kHeights = 8;               // TMA box heights 8, 16, ..., 64
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
 constexpr float kLog2e = 1.4426950408889634f;
@@ -92,8 +96,8 @@ constexpr int kMinSegChunks = 8;          // a split segment keeps at least this
 constexpr int kSlotBytes = 4 * kTile16;                        // q @0, k @8K, v @16K, g @24K
 constexpr int kQ = 0, kK = kTile16, kV = 2 * kTile16, kG = 3 * kTile16;
 constexpr int kOffSlot = 0;
-constexpr int kOffOp = kOffSlot + kSlots * kSlotBytes;         // tf32 Q^ @0, K^ @16K
-constexpr int kOffS = kOffOp + 2 * kTile32;                    // 2 x S'_[c] (fp16, MN-major)
+constexpr int kOffOp = kOffSlot + kSlots * kSlotBytes;         // per gen group g @32K g: tf32 Q^ @0, K^ @16K
+constexpr int kOffS = kOffOp + 4 * kTile32;                    // 2 x S'_[c] (fp16, MN-major)
 constexpr int kOffL = kOffS + 2 * kTile16;                     // triangle of ones
 constexpr int kRefFloats = 5 * kD;                             // raw mid, raw last, mid*log2e, c1, c2
 constexpr int kOffRef = kOffL + kTile16;                       // per slot
@@ -107,7 +111,7 @@ static_assert(kSmemBytes <= 227 * 1024, "shared memory budget");
 
 enum {
     BAR_FULL = 0,                      // [kSlots] TMA -> issuer (A)
-    BAR_EMPTY = BAR_FULL + kSlots,     // [kSlots] O(c) and everything before it done -> producer
+    BAR_EMPTY = BAR_FULL + kSlots,     // [kSlots] U(c) and O(c) done (two commits) -> producer
     BAR_REFS = BAR_EMPTY + kSlots,     // [kSlots] gen -> epi: chunk constants and mode
     BAR_AFULL = BAR_REFS + kSlots,     // [2] A done -> gen
     BAR_PURDY = BAR_AFULL + 2,         // [2] P/U(c) may go: gen(c) operands in smem and A(c) read
@@ -197,20 +201,6 @@ __device__ __forceinline__ void record_timeout(volatile uint32_t *abort_flag) {
     atomicOr(&g_device_status, kStatusTimeout);
 }
 
-// Bounded wait until *counter >= target (a counter written by one thread of
-// this CTA); false on timeout or when another role gave up.
-__device__ __forceinline__ bool wait_counter(const volatile uint32_t *counter, uint32_t target,
-                                             const volatile uint32_t *abort, uint64_t limit_ns) {
-    if (*counter >= target) return true;
-    const uint64_t t0 = global_timer_ns();
-    while (*counter < target) {
-        if (*abort) return false;
-        if (global_timer_ns() - t0 > limit_ns) return false;
-        __nanosleep(20);
-    }
-    return true;
-}
-
 // Smem row rho of chunk c holds walk position w0 + rho, where the walk is the
 // forward scan (row-major for row orders, down the columns for column orders)
 // and w0 mirrors the range for reverse orders (scan position 64c + 63 - rho).
@@ -267,6 +257,11 @@ __device__ __forceinline__ void chunk_load_boxes(int order, int T, int grid_h, i
         f(len / 8 - 1, w - w0, x, y);
         w += len;
     }
+}
+
+// fp16-pair mask of score columns 2e, 2e + 1 from a bit set of kept columns
+__device__ __forceinline__ uint32_t pmask(uint32_t vbits, int e) {
+    return (((vbits >> (2 * e)) & 1u) ? 0x0000FFFFu : 0u) | (((vbits >> (2 * e + 1)) & 1u) ? 0xFFFF0000u : 0u);
 }
 
 // Spatial token of walk position w (-1 outside the sequence).
@@ -333,7 +328,7 @@ __device__ __noinline__ void exact_chunk(uint8_t *tq, uint8_t *tk, uint8_t *tgat
 }
 
 // Operands of a tf32-mode chunk (split factors beyond the fp16 range): tf32 Q^ and
-// K^ for the score product in the scratch buffer, fp16 Qtil = Q^ c1 over q and
+// K^ for the score product in the group's operand buffer, fp16 Qtil = Q^ c1 over q and
 // Kbar = K^ c2 over k.  Re-reads the thread's 32 log-decays from TMEM (A is kept
 // until the operands are built).
 template <typename E>
@@ -389,9 +384,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBar);
     volatile uint32_t *tmem_base_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc);
     volatile uint32_t *abort_flag = reinterpret_cast<volatile uint32_t *>(smem + kOffMisc + 4);
-    // chunks whose P product is done (a maximum over the two gen groups): the tf32 /
-    // exact-path scratch buffer may be reused by chunk c once op_done >= c
-    uint32_t *op_done = reinterpret_cast<uint32_t *>(smem + kOffMisc + 8);
     float *decay_s = reinterpret_cast<float *>(smem + kOffDecay);
     volatile uint32_t *mode_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMode);
 
@@ -416,10 +408,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 
     if (threadIdx.x == 0) {
         *abort_flag = 0u;
-        *op_done = 0u;
         for (int i = 0; i < kSlots; ++i) {
             mbar_init(&bars[BAR_FULL + i], 1);
-            mbar_init(&bars[BAR_EMPTY + i], 1);
+            mbar_init(&bars[BAR_EMPTY + i], MODE == kSummary ? 1 : 2);  // after U(c) and after O(c)
             mbar_init(&bars[BAR_REFS + i], 1);
         }
         for (int i = 0; i < 2; ++i) {
@@ -430,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             mbar_init(&bars[BAR_ORDY + i], 8);
             mbar_init(&bars[BAR_OFULL + i], 1);
         }
-        mbar_init(&bars[BAR_DONE], 1);
+        mbar_init(&bars[BAR_DONE], 3);  // one commit per issuer warp
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -490,86 +481,89 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     mbar_wait(&bars[BAR_FULL + g % kSlots], (g / kSlots) & 1, nullptr, kWaitLimitNs);
             }
         }
-    } else if (warp == 1) {
-        // ======================================================= MMA issuer
-        // The whole warp runs the issue loop (operands warp-uniform) and one elected
-        // lane issues each MMA.  Fixed software-pipelined order, one wait per stage:
-        //   iteration i:  P(i) = Q^ K^^T, U(i) = Kbar^T V   once PURDY(i)
-        //                 A(i+2) = L G                       once stage i+2 landed
-        //                 O(i-1) = Q S'_[i-1] + P V          once ORDY(i-1)
-        // PURDY(i) also says that gen(i) read A(i) (so A(i+2) may overwrite TMEM A) and
-        // that epi drained U(i-2); ORDY(i-1) says TMEM P and O of the same parity were
-        // read.  P(i) comes after O(i-2), so every two-phase barrier stays at most one
-        // phase ahead of its waiter.
-        const uint32_t idesc_a = instr_desc(Elem<E>::fmt, 64, 64, 0, 1);
-        const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
-        const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
-        const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
-        const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
+    } else if (warp == 1 || warp >= 14) {
+        // ======================================================= MMA issuers
+        // Three warps issue the products, each in program order and waiting only for
+        // its own inputs, so that the issue overhead of one product never delays
+        // another.  A whole warp runs each loop (operands warp-uniform) and one
+        // elected lane issues each MMA.
+        //   warp 1   A(c) = L G          once chunk c landed and gen(c-2) built its
+        //                                operands (so TMEM A of the parity was read)
+        //   warp 14  P(c) = Q^ K^^T,     once PURDY(c): gen(c) operands in smem and epi
+        //            U(c) = Kbar^T V     drained U(c-2)
+        //   warp 15  O(c) = Q S'_[c] + P V   once ORDY(c)
+        // A tcgen05.commit tracks only its own thread's MMAs: the slot of chunk c is
+        // released by two commits, after U(c) (warp 14) and after O(c) (warp 15); P(c)
+        // and A(c) completed before ORDY(c).  No waiter can be overtaken by two phases
+        // of its barrier: PURDY(c + 2) needs A(c + 2) and U(c), FULL of the next chunk
+        // of a slot needs that slot's EMPTY, ORDY(c + 2) needs O(c) read.
         const uint32_t slot0 = smem_u32(smem + kOffSlot);
-        const uint64_t dL = kdesc(smem_u32(smem + kOffL));
-        const uint64_t dqh = kdesc(smem_u32(smem + kOffOp)), dkh = kdesc(smem_u32(smem + kOffOp + kTile32));
-        const uint32_t sbuf = smem_u32(smem + kOffS);
         bool ok = true;
-        for (int c = 0; c < 2 && c < G; ++c) {  // A(0), A(1)
-            ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + c], 0, abort_flag, kWaitLimitNs));
-            if (!ok) break;
-            tc_fence_after();
-            const uint64_t dg = mndesc(slot0 + c * kSlotBytes + kG);
+        if (warp == 1) {
+            const uint32_t idesc_a = instr_desc(Elem<E>::fmt, 64, 64, 0, 1);
+            const uint64_t dL = kdesc(smem_u32(smem + kOffL));
+            int sa = 0;
+            for (int c = 0; c < G; ++c) {
+                if (c >= 2) {
+                    ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_PURDY + (c & 1)], ((c - 2) >> 1) & 1, abort_flag, kWaitLimitNs));
+                    if (!ok) break;
+                }
+                ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + sa], (c / kSlots) & 1, abort_flag, kWaitLimitNs));
+                if (!ok) break;
+                tc_fence_after();
+                const uint64_t dg = mndesc(slot0 + sa * kSlotBytes + kG);
+                const uint32_t d = tmem + kColA + (c & 1) * 64;
 #pragma unroll
-            for (int ks = 0; ks < 4; ++ks)
-                mma_f16_ss_warp(tmem + kColA + c * 64, dL + 2 * ks, dg + 128 * ks, idesc_a, ks > 0);
-            mma_commit_warp(&bars[BAR_AFULL + c]);
-        }
-        int su = 0, sa = 2 % kSlots, so = 0;   // slots of chunks i, i + 2 and of the next O
-        for (int i = 0; ok && i <= G; ++i) {
-            if (i < G) {
-                ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_PURDY + (i & 1)], (i >> 1) & 1, abort_flag, kWaitLimitNs));
+                for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dL + 2 * ks, dg + 128 * ks, idesc_a, ks > 0);
+                mma_commit_warp(&bars[BAR_AFULL + (c & 1)]);
+                sa = (sa == kSlots - 1) ? 0 : sa + 1;
+            }
+        } else if (warp == 14) {
+            const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
+            const uint32_t idesc_p32 = instr_desc(kFmtTF32, 64, 64, 0, 0);
+            const uint32_t idesc_u = instr_desc(kFmtF16, 64, 64, 1, 1);
+            const uint64_t dqh0 = kdesc(smem_u32(smem + kOffOp)), dkh0 = kdesc(smem_u32(smem + kOffOp + kTile32));
+            int su = 0;
+            for (int c = 0; c < G; ++c) {
+                ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_PURDY + (c & 1)], (c >> 1) & 1, abort_flag, kWaitLimitNs));
                 if (!ok) break;
                 tc_fence_after();
                 const uint32_t st = slot0 + su * kSlotBytes;
                 const uint32_t mode = __shfl_sync(0xffffffffu, mode_s[su], 0);
-                const uint32_t dp = tmem + kColP + (i & 1) * 64;
+                const uint32_t dp = tmem + kColP + (c & 1) * 64;
                 if (kSum) {
                     // summaries need no scores
                 } else if (mode == kModeF16) {
                     const uint64_t dq = kdesc(st + kQ), dk = kdesc(st + kK);
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(dp, dq + 2 * ks, dk + 2 * ks, idesc_p16, ks > 0);
-                    mma_commit_warp(&bars[BAR_PFULL + (i & 1)]);
+                    mma_commit_warp(&bars[BAR_PFULL + (c & 1)]);
                 } else if (mode == kModeTF32) {
+                    const uint64_t dqh = dqh0 + (c & 1) * (2 * kTile32 >> 4), dkh = dkh0 + (c & 1) * (2 * kTile32 >> 4);
 #pragma unroll
                     for (int ks = 0; ks < 8; ++ks) {
                         const uint32_t off = (ks >> 2) * 512 + (ks & 3) * 2;  // (8192 B, 32 B) >> 4
                         mma_tf32_ss_warp(dp, dqh + off, dkh + off, idesc_p32, ks > 0);
                     }
-                    mma_commit_warp(&bars[BAR_PFULL + (i & 1)]);
+                    mma_commit_warp(&bars[BAR_PFULL + (c & 1)]);
                 } else if (lane == 0) {
-                    mbar_arrive(&bars[BAR_PFULL + (i & 1)]);  // exact scores are already in smem
+                    mbar_arrive(&bars[BAR_PFULL + (c & 1)]);  // exact scores are already in smem
                 }
                 __syncwarp();
-                // U(i) = Kbar^T V (fp16 mode: K^^T V): the k tile read as the MN-major A
+                // U(c) = Kbar^T V (fp16 mode: K^^T V): the k tile read as the MN-major A
                 const uint64_t dk = mndesc(st + kK), dv = mndesc(st + kV);
-                const uint32_t du = tmem + kColU + (i & 1) * 64;
+                const uint32_t du = tmem + kColU + (c & 1) * 64;
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(du, dk + 128 * ks, dv + 128 * ks, idesc_u, ks > 0);
-                mma_commit_warp(&bars[BAR_UFULL + (i & 1)]);
-                if (kSum) mma_commit_warp(&bars[BAR_EMPTY + su]);  // U is the stage's last reader
+                mma_commit_warp(&bars[BAR_UFULL + (c & 1)]);
+                mma_commit_warp(&bars[BAR_EMPTY + su]);  // U is the slot's last reader among this warp's MMAs
                 su = (su == kSlots - 1) ? 0 : su + 1;
-                if (i + 2 < G) {
-                    ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + sa], ((i + 2) / kSlots) & 1, abort_flag, kWaitLimitNs));
-                    if (!ok) break;
-                    tc_fence_after();
-                    const uint64_t dg = mndesc(slot0 + sa * kSlotBytes + kG);
-                    const uint32_t d = tmem + kColA + (i & 1) * 64;
-#pragma unroll
-                    for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dL + 2 * ks, dg + 128 * ks, idesc_a, ks > 0);
-                    mma_commit_warp(&bars[BAR_AFULL + (i & 1)]);
-                }
-                sa = (sa == kSlots - 1) ? 0 : sa + 1;
             }
-            if (!kSum && i >= 1) {
-                const int c = i - 1;
+        } else if (!kSum) {
+            const uint32_t idesc_o = instr_desc(kFmtF16, 64, 64, 0, 1);
+            const uint32_t sbuf = smem_u32(smem + kOffS);
+            int so = 0;
+            for (int c = 0; c < G; ++c) {
                 ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_ORDY + (c & 1)], (c >> 1) & 1, abort_flag, kWaitLimitNs));
                 if (!ok) break;
                 tc_fence_after();
@@ -603,14 +597,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const int tg = threadIdx.x - 64 - 128 * gw;
         const int rho_mid = rev ? 32 : 31, rho_last = rev ? 0 : 63;
         // causal mask of this thread's 32 score columns as packed fp16-pair masks (scan order)
-        uint32_t pm[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-            const int s0 = ch0 + 2 * e;
-            const bool k0 = rev ? (s0 >= row) : (s0 <= row);
-            const bool k1 = rev ? (s0 + 1 >= row) : (s0 + 1 <= row);
-            pm[e] = (k0 ? 0x0000FFFFu : 0u) | (k1 ? 0xFFFF0000u : 0u);
-        }
+        uint32_t vbits = 0u;  // bit s: score column ch0 + s is kept
+        for (int s = 0; s < 32; ++s)
+            if (rev ? (ch0 + s >= row) : (ch0 + s <= row)) vbits |= 1u << s;
         for (int c = gw; c < G; c += 2) {
             const int sl = c % kSlots, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
@@ -619,11 +608,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             // bf16 values become fp16 MMA operands in place (exact for |v| in the fp16
             // normal range); the loads go first so that their latency hides behind the
             // operand build, the converted words are stored with the operands
-            uint4 vw[4];
-            if constexpr (std::is_same<E, __nv_bfloat16>::value) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) vw[q] = *reinterpret_cast<const uint4 *>(st + kV + sw128(row, (ch0 + 8 * q) * 2));
-            }
             tc_fence_after();
             uint32_t ar[32];
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&ar[0]));
@@ -673,9 +657,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             uint8_t *tq = st + kQ, *tk = st + kK, *tgt = st + kG;
             bool opfail = false;
             if (mode != kModeF16) {
-                // the tf32 / scratch buffer is shared by consecutive chunks: wait for the previous
-                // release; the decision is uniform because the exact path has named barriers
-                opfail = named_barrier_or(bar_id, 128, !wait_counter(op_done, (uint32_t)c, abort_flag, kWaitLimitNs));
+                // the constants written by warp 0 above are read by every warp of the group; the
+                // group's own operand buffer was last read by P(c - 2), complete before mask(c - 2)
+                opfail = named_barrier_or(bar_id, 128, false);
             }
             if (mode == kModeF16) {
 #pragma unroll
@@ -704,12 +688,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
             } else if (!opfail) {
                 if (mode == kModeTF32)
-                    tf32_operands<E>(tq, tk, smem + kOffOp, ref, tmem + lane_base + kColA + bb * 64, row, ch0);
+                    tf32_operands<E>(tq, tk, smem + kOffOp + gw * 2 * kTile32, ref, tmem + lane_base + kColA + bb * 64, row, ch0);
                 else
-                    exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp), decay_s + sl * kD, rev, tg,
+                    exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp + gw * 2 * kTile32), decay_s + sl * kD, rev, tg,
                                    bar_id);
             }
             if constexpr (std::is_same<E, __nv_bfloat16>::value) {
+                uint4 vw[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) vw[q] = *reinterpret_cast<const uint4 *>(st + kV + sw128(row, (ch0 + 8 * q) * 2));
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     uint32_t *wp = reinterpret_cast<uint32_t *>(&vw[q]);
@@ -730,17 +717,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (tg == 0) mbar_arrive(&bars[BAR_REFS + sl]);  // constants and mode of chunk c -> epi
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // operands in smem, A(c) read
-            if (kSum) {  // no scores: the scratch buffer is free once the operands are built
-                if (tg == 0) atomicMax(op_done, (uint32_t)c + 1u);
-                continue;
-            }
+            if (kSum) continue;  // no scores
             // ---- masked scores of chunk c over its gate tile (consumed by A(c) long ago)
             const bool pfail = !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
             if (named_barrier_or(bar_id, 128, pfail)) {
                 record_timeout(abort_flag);
                 break;
             }
-            if (tg == 0) atomicMax(op_done, (uint32_t)c + 1u);  // P(c) is done
             if (mode != kModeExact) {
                 tc_fence_after();
                 uint32_t r[32];
@@ -750,10 +733,10 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 #pragma unroll
                 for (int q = 0; q < 4; ++q)
                     *reinterpret_cast<uint4 *>(tgt + sw128(row, (ch0 + 8 * q) * 2)) = make_uint4(
-                        h2bits(__uint_as_float(r[8 * q + 0]), __uint_as_float(r[8 * q + 1])) & pm[4 * q + 0],
-                        h2bits(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])) & pm[4 * q + 1],
-                        h2bits(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])) & pm[4 * q + 2],
-                        h2bits(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])) & pm[4 * q + 3]);
+                        h2bits(__uint_as_float(r[8 * q + 0]), __uint_as_float(r[8 * q + 1])) & pmask(vbits, 4 * q + 0),
+                        h2bits(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])) & pmask(vbits, 4 * q + 1),
+                        h2bits(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])) & pmask(vbits, 4 * q + 2),
+                        h2bits(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])) & pmask(vbits, 4 * q + 3));
             }
             tc_fence_before();
             fence_proxy_async_smem();
@@ -761,7 +744,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // this warp's rows of P are in smem
         }
     } else {
-        // ======================================================= epi warpgroup
+        // ======================================================= epi warpgroup (warps 10-13)
         // Carries the fp32 state of the current key half in registers (thread: channel
         // row, 32 value columns; with two key halves the other half's state waits in So
         // and the two swap after every virtual chunk), writes Diag(c1) S for the readout
@@ -858,12 +841,23 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     break;
                 }
                 tc_fence_after();
-                uint32_t r[32];
-                tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-                tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
-                tmem_ld_wait();
+                if constexpr (NH == 2) {  // two states live: read U in halves to save registers
 #pragma unroll
-                for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
+                    for (int hf = 0; hf < 2; ++hf) {
+                        uint32_t r[16];
+                        tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16 * hf, r);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) S[16 * hf + j] = fmaf(dc, S[16 * hf + j], c2 * __uint_as_float(r[j]));
+                    }
+                } else {
+                    uint32_t r[32];
+                    tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+                    tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
+                }
                 tc_fence_before();
                 if (kSum) {
                     dp *= dc;
@@ -903,10 +897,15 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     break;
                 }
                 tc_fence_after();
-                uint32_t r[32];
-                tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-                tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
-                tmem_ld_wait();
+                uint32_t ow[16];  // the row's 32 outputs packed in pairs
+#pragma unroll
+                for (int hf = 0; hf < 2; ++hf) {
+                    uint32_t r[16];
+                    tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 16 * hf, r);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) ow[8 * hf + j] = Elem<E>::pack(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+                }
                 tc_fence_before();
                 const StreamPos po = stream_pos(co, L, nh, lognv, kSplit ? p.nsu : 1);
                 const int b = po.bh / p.H, h = po.bh % p.H;
@@ -914,11 +913,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 if (t >= 0) {
                     uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * kDv + 64 * po.vb + ch0);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        dst[q] = make_uint4(Elem<E>::pack(__uint_as_float(r[8 * q + 0]), __uint_as_float(r[8 * q + 1])),
-                                            Elem<E>::pack(__uint_as_float(r[8 * q + 2]), __uint_as_float(r[8 * q + 3])),
-                                            Elem<E>::pack(__uint_as_float(r[8 * q + 4]), __uint_as_float(r[8 * q + 5])),
-                                            Elem<E>::pack(__uint_as_float(r[8 * q + 6]), __uint_as_float(r[8 * q + 7])));
+                    for (int q = 0; q < 4; ++q) dst[q] = make_uint4(ow[4 * q], ow[4 * q + 1], ow[4 * q + 2], ow[4 * q + 3]);
                 }
             }
         }
