@@ -90,7 +90,7 @@ enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
 // Kernel passes: kFull (sequences whole), kSplitFull (outputs of segments that
 // start from the fold of the earlier segments' summaries), kSummary (the summaries).
 enum : int { kFull = 0, kSplitFull = 1, kSummary = 2 };
-constexpr int kMinSegChunks = 8;          // a split segment keeps at least this many chunks
+constexpr int kMinSegChunks = 4;          // a split segment keeps at least this many chunks
 
 // Shared-memory map (byte offsets from a 1024-aligned base).
 constexpr int kSlotBytes = 4 * kTile16;                        // q @0, k @8K, v @16K, g @24K

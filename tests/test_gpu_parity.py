@@ -245,25 +245,39 @@ def test_guard_bands_and_full_coverage():
 
 
 def test_cuda_graph_capture():
+    """Replaying a captured graph equals eager execution.  With a caller-owned
+    workspace both run the same schedule (here the split one: two kernels), bit for
+    bit.  gtr_gla_fwd does not use its internal workspace under capture and runs
+    the sequences unsplit there: that result is held to the oracle's bar."""
     w = wl.WORKLOADS[1]
     inp, _ = _Cache.get(1)
+    ref_o, ref_s = _Cache.oracle(1, wl.ROW_REV)
     t = {n: to_torch(inp[n], w.dtype) for n in ("q", "k", "v", "g")}
+    ws_bytes = gla.workspace_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, TORCH_DT[w.dtype])
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda") if ws_bytes else None
     out = torch.empty_like(t["v"])
     fs = torch.empty((w.B, w.H, w.Dk, w.Dv), device="cuda")
-    gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, wl.ROW_REV, out=out,
-                final_state=fs)   # warm-up outside capture
+    gla.forward_ws(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, wl.ROW_REV, out, fs, ws)
     torch.cuda.synchronize()
-    ref = out.clone()
+    ref, ref_fs = out.clone(), fs.clone()
     out.zero_()
+    fs.zero_()
+    out2 = torch.empty_like(t["v"])
+    fs2 = torch.empty_like(fs)
     g = torch.cuda.CUDAGraph()
     s = torch.cuda.Stream()
     with torch.cuda.stream(s):
         with torch.cuda.graph(g, stream=s):
-            gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, wl.ROW_REV, out=out,
-                        final_state=fs, stream=s)
+            gla.forward_ws(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, wl.ROW_REV, out, fs, ws,
+                           stream=s)
+            gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, wl.ROW_REV, out=out2,
+                        final_state=fs2, stream=s)
     g.replay()
     torch.cuda.synchronize()
-    assert torch.equal(out, ref)
+    assert gla.sync_status() == 0
+    assert torch.equal(out, ref) and torch.equal(fs, ref_fs)
+    assert_within_bar(_np(out2), ref_o, w.dtype, "captured gtr_gla_fwd")
+    assert_within_bar(fs2.cpu().numpy().astype(np.float64), ref_s, w.dtype, "captured state")
 
 
 def test_host_memory_entry_point():
