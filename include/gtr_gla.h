@@ -197,7 +197,12 @@ gtr_status_t gtr_gla_fwd_host(const void *q_host, const void *k_host, const void
 /* Synchronises `stream`, then returns and clears the device status word of the
  * current device (GTR_OK when no device-side condition was recorded,
  * GTR_ERR_TIMEOUT when a bounded wait gave up), or GTR_ERR_CUDA when the
- * synchronisation itself failed. */
+ * synchronisation itself failed.  Every device-side wait gives up after 1 s;
+ * the kernel then drains its copies, frees its tensor memory and returns, so
+ * the context stays usable (the outputs of that call are undefined).  Test
+ * hook for this path: with the environment variable GTR_GLA_TEST_DROP_LOAD=1
+ * the tensor-core schedule withholds one chunk's load in its first CTA, so the
+ * call reports GTR_ERR_TIMEOUT (no fault is involved). */
 gtr_status_t gtr_gla_sync_status(cudaStream_t stream);
 
 /* Static, NUL-terminated description of a status code. */

@@ -57,6 +57,7 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
+#include <cstdlib>
 #include <cstring>
 #include <list>
 #include <mutex>
@@ -145,6 +146,8 @@ struct TcParams {
     int nsu;                               // segments per (sequence, value slice) among this launch's units
     float *summary;                        // nseg > 1: per (sequence, segment < nseg - 1) end state from zero
                                            // [Dk][Dv] and total decay [Dk], fp32
+    int drop_load;                         // test hook: CTA 0 withholds its first chunk's load, so the
+                                           // bounded waits run out and the call reports a timeout
 };
 
 // ---------------------------------------------------------------- helpers
@@ -467,18 +470,21 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
                 uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
                 uint64_t *fb = &bars[BAR_FULL + sl];
-                mbar_arrive_expect_tx(fb, kSum ? kSlotBytes - kTile16 : kSlotBytes);  // summaries need no q
-                chunk_load_boxes(p.order, p.T, p.grid_h, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
-                    if (!kSum) tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, xk, h, c2, c3, b);
-                    tma_load_5d(st + kK + row * 128, &p.maps[T_K][hi], fb, xk, h, c2, c3, b);
-                    tma_load_5d(st + kV + row * 128, &p.maps[T_V][hi], fb, xv, h, c2, c3, b);
-                    tma_load_5d(st + kG + row * 128, &p.maps[T_G][hi], fb, xk, h, c2, c3, b);
-                });
+                if (!(p.drop_load && blockIdx.x == 0 && g == 0)) {
+                    mbar_arrive_expect_tx(fb, kSum ? kSlotBytes - kTile16 : kSlotBytes);  // summaries need no q
+                    chunk_load_boxes(p.order, p.T, p.grid_h, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
+                        if (!kSum) tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, xk, h, c2, c3, b);
+                        tma_load_5d(st + kK + row * 128, &p.maps[T_K][hi], fb, xk, h, c2, c3, b);
+                        tma_load_5d(st + kV + row * 128, &p.maps[T_V][hi], fb, xv, h, c2, c3, b);
+                        tma_load_5d(st + kG + row * 128, &p.maps[T_G][hi], fb, xk, h, c2, c3, b);
+                    });
+                }
                 ++issued;
             }
             if (*abort_flag) {  // never leave while copies are still landing in shared memory
                 for (int g = (issued > kSlots ? issued - kSlots : 0); g < issued; ++g)
-                    mbar_wait(&bars[BAR_FULL + g % kSlots], (g / kSlots) & 1, nullptr, kWaitLimitNs);
+                    if (!(p.drop_load && blockIdx.x == 0 && g == 0))
+                        mbar_wait(&bars[BAR_FULL + g % kSlots], (g / kSlots) & 1, nullptr, kWaitLimitNs);
             }
         }
     } else if (warp == 1 || warp >= 14) {
@@ -1102,6 +1108,9 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     tp.nseg = nseg;
     tp.seg_len = tp.n_chunks / nseg;
     tp.summary = static_cast<float *>(workspace);
+    // test hook for the timeout path (no fault: the data of one chunk simply never arrives)
+    const char *drop = std::getenv("GTR_GLA_TEST_DROP_LOAD");
+    tp.drop_load = (drop != nullptr && drop[0] == '1') ? 1 : 0;
     const int seqs = static_cast<int>(p.B * p.H) * tp.nv;  // (sequence, value slice) pairs
     const bool half = p.dtype == 1;
     // persistent: one CTA per SM, each walking its share of the work units
