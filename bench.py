@@ -60,6 +60,27 @@ def dist_env():
     return rank, world, local
 
 
+def rank_seed(w: wl.Workload, rank: int) -> int:
+    """Seed of rank r's batch: every rank draws its own batch of the same workload
+    (same distributions), so N ranks process N independent batches."""
+    return 1234 + w.wid + 1000 * rank
+
+
+def max_over_ranks(ms: float, pg, device) -> float:
+    """The slowest rank's time (all-reduce MAX); `ms` itself without a process group."""
+    if pg is None:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_tokens_per_s(tokens_per_rank_step: int, world: int, ms_per_step: float) -> float:
+    """Whole-job throughput: the tokens of all ranks over the max-over-ranks step time."""
+    return tokens_per_rank_step * world / (ms_per_step * 1e-3)
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -239,7 +260,7 @@ def main():
     dt = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}[w.dtype]
 
     # inputs: rank r draws batch r of the workload (same distributions, own seed)
-    inp = wl.workload_inputs(w, B=w.B, seed=1234 + w.wid + 1000 * rank)
+    inp = wl.workload_inputs(w, B=w.B, seed=rank_seed(w, rank))
 
     def to_dev(a):
         if w.dtype == "bf16":
@@ -291,13 +312,9 @@ def main():
     per_launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     if gla.sync_status() != 0:
         raise RuntimeError("device status word set during the timed region")
-    if pg:
-        tt = torch.tensor([total_ms], device=dev)
-        pg.all_reduce(tt, op=pg.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = max_over_ranks(total_ms, pg, dev)
     ms_per_step = total_ms / args.steps
-    tokens_per_step = w.B * w.T * world
-    value = tokens_per_step / (ms_per_step * 1e-3)
+    value = job_tokens_per_s(w.B * w.T, world, ms_per_step)
 
     # roofline of the (single) kernel of a step
     hbm_peak, peak_src = load_peaks()
@@ -340,11 +357,8 @@ def main():
         e1.record(stream)
         torch.cuda.synchronize()
         e_ms = e0.elapsed_time(e1)
-        if pg:
-            tt = torch.tensor([e_ms], device=dev)
-            pg.all_reduce(tt, op=pg.ReduceOp.MAX)
-            e_ms = float(tt.item())
-        es = w.B * w.T * world / (e_ms / args.e2e_steps * 1e-3)
+        e_ms = max_over_ranks(e_ms, pg, dev)
+        es = job_tokens_per_s(w.B * w.T, world, e_ms / args.e2e_steps)
         h2d = sum(host[n].numel() * host[n].element_size() for n in ("q", "k", "v", "g"))
         d2h = hout.numel() * hout.element_size() + (hfs.numel() * 4 if hfs is not None else 0)
         e2e = {"value": es, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
