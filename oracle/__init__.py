@@ -17,8 +17,11 @@ Prediction"):
   formula after it, with a free chunk size; a second restatement used to pin
   the chunk equations against the recurrence.
 * :func:`scan_tokens` -- the scan permutation alone (position -> spatial token).
+* :func:`gated_output` -- Sec. 3.1, the output gate applied to the mixer's
+  output: ``u_t = SiLU(r_t) * RMSNorm(o_t)`` (the epilogue the paper's deployed
+  kernel fuses, App. C.3).
 
-Pins: tests/test_oracle_pins.py checks both functions against a hand-worked
+Pins: tests/test_oracle_pins.py checks the functions against hand-worked
 example (tests/golden/), brute-force quadratic forms, closed forms (gate 1 =
 causal linear attention, gate 0 = (q.k) v, T = 1) and invariants (reversal,
 grid transpose, linearity, chunk-size invariance).
@@ -190,3 +193,24 @@ def chunkwise(q, k, v, g, grid_h: int, grid_w: int, order: int = ROW_FWD, chunk:
     if rc != 0:
         raise RuntimeError(f"gla_oracle_chunkwise failed ({rc})")
     return out, fs
+
+
+def gated_output(o, r_pre, weight, eps: float) -> np.ndarray:
+    """Output gate of Sec. 3.1: ``u_t = SiLU(r_t) * RMSNorm(o_t)``.
+
+    ``r_pre`` is the gate's pre-activation ``x_t W_r`` (the paper writes
+    ``r_t = SiLU(x_t W_r)``; the fused epilogue of App. C.3 applies the SiLU).
+    RMSNorm (Zhang and Sennrich, 2019) runs over each head's Dv outputs,
+    ``o_j / sqrt(mean_j o_j^2 + eps) * weight_j``, with one weight vector of
+    length Dv shared by the heads.  o, r_pre: [B, T, H, Dv]; weight: [Dv].
+    Plain fp64 numpy, written out from the definitions.
+    """
+    o = np.asarray(o, dtype=np.float64)
+    r = np.asarray(r_pre, dtype=np.float64)
+    w = np.asarray(weight, dtype=np.float64)
+    if o.shape != r.shape or w.shape != (o.shape[-1],):
+        raise ValueError("o, r_pre must share a shape and weight must have Dv entries")
+    rms = np.sqrt(np.mean(o * o, axis=-1, keepdims=True) + float(eps))
+    with np.errstate(over="ignore"):
+        silu = r / (1.0 + np.exp(-r))   # r * sigmoid(r); exp overflow gives -0 for r << 0
+    return silu * (o / rms) * w

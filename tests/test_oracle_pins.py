@@ -254,3 +254,49 @@ def test_rejects_bad_arguments():
         oracle.recurrence(q, q, q, q, 3, 2)
     with pytest.raises(RuntimeError):
         oracle.recurrence(q, q, q, q, 2, 2, order=7)
+
+
+# ----------------------------------------------------------------- output gate
+def test_gated_output_hand_worked():
+    """Sec. 3.1 output gate on a hand-worked head (tests/golden/gated_epilogue_1x4.json)."""
+    d = json.load(open(os.path.join(GOLDEN, "gated_epilogue_1x4.json")))
+    o = np.array(d["o"]).reshape(1, 1, 1, 4)
+    r = np.array(d["r_pre"]).reshape(1, 1, 1, 4)
+    u = oracle.gated_output(o, r, np.array(d["weight"]), d["eps"])
+    np.testing.assert_allclose(u.reshape(-1), d["u"], rtol=0, atol=1e-15)
+
+
+def test_gated_output_matches_library_rmsnorm_and_silu():
+    """The same gate through torch's own RMSNorm and SiLU routines, in float64."""
+    import torch
+    rng = np.random.Generator(np.random.PCG64(31))
+    o = rng.standard_normal((2, 5, 3, 16)) * 4.0
+    r = rng.standard_normal((2, 5, 3, 16)) * 3.0
+    w = rng.standard_normal(16)
+    eps = 1e-5
+    ref = (torch.nn.functional.silu(torch.from_numpy(r)) *
+           torch.nn.functional.rms_norm(torch.from_numpy(o), (16,), torch.from_numpy(w), eps)).numpy()
+    np.testing.assert_allclose(oracle.gated_output(o, r, w, eps), ref, rtol=1e-12, atol=1e-14)
+
+
+def test_gated_output_invariants():
+    rng = np.random.Generator(np.random.PCG64(32))
+    o = rng.standard_normal((1, 7, 4, 8))
+    r = rng.standard_normal((1, 7, 4, 8)) * 2.0
+    w = rng.standard_normal(8)
+    eps = 1e-3
+    u = oracle.gated_output(o, r, w, eps)
+    # SiLU(z) - SiLU(-z) = z  =>  u(r) - u(-r) = r * RMSNorm(o) * w  (pins the sigmoid's sign)
+    rms = np.sqrt(np.mean(o * o, axis=-1, keepdims=True) + eps)
+    np.testing.assert_allclose(u - oracle.gated_output(o, -r, w, eps), r * o / rms * w, rtol=1e-12,
+                               atol=1e-14)
+    # scale invariance: o -> c o with eps -> c^2 eps leaves u unchanged
+    np.testing.assert_allclose(oracle.gated_output(3.0 * o, r, w, 9.0 * eps), u, rtol=1e-12, atol=1e-14)
+    # each head is normalised on its own: changing head 0 leaves the other heads' u unchanged
+    o2 = o.copy()
+    o2[:, :, 0, :] *= 10.0
+    np.testing.assert_array_equal(oracle.gated_output(o2, r, w, eps)[:, :, 1:, :], u[:, :, 1:, :])
+    # a zero gate pre-activation closes the output (SiLU(0) = 0); a large one passes r * RMSNorm(o)
+    np.testing.assert_array_equal(oracle.gated_output(o, np.zeros_like(r), w, eps), 0.0 * u)
+    big = np.full_like(r, 40.0)
+    np.testing.assert_allclose(oracle.gated_output(o, big, w, eps), 40.0 * o / rms * w, rtol=1e-15)
