@@ -45,6 +45,8 @@ def parse():
     ap.add_argument("--workload", type=int, default=DEFAULT_WORKLOAD)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--schedule", default="auto", choices=["auto", "simt", "tc"])
+    ap.add_argument("--gated", action="store_true",
+                    help="time the mixer with its output gate u = SiLU(r) * RMSNorm(o) (Sec. 3.1) instead of o")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -280,10 +282,22 @@ def main():
     launches_per_step = 2 if split else 1
     if split:
         kernel_name += ", segment-summary pass + output pass"
+    if args.gated:  # the output gate runs as one more kernel right after the mixer
+        launches_per_step += 1
+        kernel_name += " + output-gate kernel"
+
+    if args.gated:
+        rng = np.random.Generator(np.random.PCG64(rank_seed(w, rank) + 17))
+        gate_r = to_dev(wl.round_to_storage(rng.standard_normal((w.B, w.T, w.H, w.Dv)) * 1.5, w.dtype))
+        gate_w = torch.from_numpy((1.0 + 0.2 * rng.standard_normal(w.Dv)).astype(np.float32)).to(dev)
 
     def step(i):
-        gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, orders[i % len(orders)],
-                    out=out, final_state=fs if fs is not None else None, schedule=schedule)
+        if args.gated:
+            gla.forward_gated(t["q"], t["k"], t["v"], t["g"], gate_r, gate_w, 1e-5, w.grid_h, w.grid_w,
+                              orders[i % len(orders)], out=out, final_state=fs if fs is not None else None)
+        else:
+            gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, orders[i % len(orders)],
+                        out=out, final_state=fs if fs is not None else None, schedule=schedule)
 
     for i in range(max(3, args.warmup)):
         step(i)
@@ -319,6 +333,8 @@ def main():
     # roofline of the (single) kernel of a step
     hbm_peak, peak_src = load_peaks()
     alg_bytes = w.algorithmic_bytes()
+    if args.gated:  # the gate's pre-activation is read once more per token-head (u replaces o)
+        alg_bytes += w.B * w.T * w.H * w.Dv * wl.ELEM_SIZE[w.dtype]
     kernel_ms = sum(per_launch_ms) / len(per_launch_ms)
     achieved = alg_bytes / (kernel_ms * 1e-3) / 1e9
     traffic = None
@@ -336,7 +352,7 @@ def main():
 
     # end to end through the host-memory entry point (pinned host buffers)
     e2e = None
-    if args.e2e_steps > 0:
+    if args.e2e_steps > 0 and not args.gated:
         host = {n: (torch.from_numpy(inp[n].view(np.int16)).view(torch.bfloat16) if w.dtype == "bf16"
                     else torch.from_numpy(inp[n])).pin_memory() for n in ("q", "k", "v", "g")}
         hout = torch.empty(host["v"].shape, dtype=host["v"].dtype).pin_memory()
@@ -378,7 +394,10 @@ def main():
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": w.dtype, "data": "synthetic (seeded, workload recipe in workloads.py)",
-                "config": workload_config(w, world, {"schedule": schedule}),
+                "config": workload_config(w, world, dict({"schedule": schedule},
+                                                         **({"epilogue": "output gate u = SiLU(r) * RMSNorm(o), "
+                                                             "second kernel right after the mixer"}
+                                                            if args.gated else {}))),
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
                 "gpu_launches": args.steps * launches_per_step, "clocks": clk.summary(),
                 "token_heads_per_s": value * w.H}

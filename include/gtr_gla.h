@@ -131,6 +131,24 @@ gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const v
                             float *final_state, void *workspace, size_t workspace_bytes,
                             cudaStream_t stream);
 
+/* The mixer followed by its output gate (Sec. 3.1): instead of o, `out`
+ * receives u = SiLU(r) * RMSNorm(o) per head, where `gate` holds the gate's
+ * pre-activation r = x W_r ([B, T, H, Dv], same dtype and layout as v) and
+ * RMSNorm(o)_j = o_j / sqrt(mean over the head's Dv outputs of o^2 + eps) *
+ * norm_weight[j] (`norm_weight`: Dv fp32 values on the device, shared by the
+ * heads; eps >= 0).  App. C.3 fuses this epilogue into the mixer kernel's
+ * output stores; here a second kernel applies it to `out` in place right after
+ * the mixer (o is rounded to the dtype in between), reading o back while it is
+ * still in L2 for outputs that fit there: on GB300 that was measured 1.45-1.7x
+ * faster than the fused stores, whose extra work lands on the mixer's critical
+ * path.  final_state is the mixer's state as in gtr_gla_fwd.  `gate` and `norm_weight` must be 16-byte
+ * aligned and `gate` must not overlap `out`.  Allocation, workspace and errors
+ * as gtr_gla_fwd. */
+gtr_status_t gtr_gla_fwd_gated(const void *q, const void *k, const void *v, const void *log_gate,
+                               const void *gate, const float *norm_weight, float eps, int B, int H,
+                               int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
+                               gtr_dtype_t dtype, void *out, float *final_state, cudaStream_t stream);
+
 /* Size of the fixed device scratch array behind gtr_gla_fwd_noalloc.  The
  * library holds one such array on every GPU where it is loaded, from the
  * module's load until the process exits.  The split schedule needs at most

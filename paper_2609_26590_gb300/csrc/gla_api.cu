@@ -196,6 +196,28 @@ gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const v
     return dispatch(p, GTR_SCHED_AUTO, workspace, workspace_bytes, true, stream);
 }
 
+gtr_status_t gtr_gla_fwd_gated(const void *q, const void *k, const void *v, const void *log_gate,
+                               const void *gate, const float *norm_weight, float eps, int B, int H,
+                               int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
+                               gtr_dtype_t dtype, void *out, float *final_state, cudaStream_t stream) {
+    gtr::Problem p;
+    gtr_status_t st = make_problem(q, k, v, log_gate, B, H, grid_h, grid_w, Dk, Dv, scan_order,
+                                   dtype, out, final_state, &p);
+    if (st != GTR_OK) return st;
+    if (!(eps >= 0.f) || !(eps < 3.0e38f)) return GTR_ERR_INVALID_ARG;  // also rejects NaN
+    if (B == 0 || H == 0) return GTR_OK;
+    if (!gate || !norm_weight || !aligned(gate) || !aligned(norm_weight)) return GTR_ERR_INVALID_ARG;
+    const size_t nv = (size_t)B * p.T * H * Dv * elem_size(dtype);
+    if (overlaps(out, nv, gate, nv)) return GTR_ERR_INVALID_ARG;
+    // the mixer, then the gate over its output in place (the output is still in L2
+    // for workloads that fit there)
+    st = dispatch(p, GTR_SCHED_AUTO, nullptr, 0, false, stream);
+    if (st != GTR_OK) return st;
+    const cudaError_t e = gtr::launch_gate_epilogue(p, gtr::Gate{gate, norm_weight, eps}, stream);
+    if (e != cudaSuccess) return cuda_fail(e);
+    return GTR_OK;
+}
+
 gtr_status_t gtr_gla_fwd_noalloc(const void *q, const void *k, const void *v, const void *log_gate,
                                  int B, int H, int grid_h, int grid_w, int Dk, int Dv,
                                  gtr_scan_t scan_order, gtr_dtype_t dtype, void *out,

@@ -18,8 +18,19 @@ struct Problem {
     long long T;                // grid_h * grid_w
 };
 
+// Output gate of Sec. 3.1, u = SiLU(r) * RMSNorm(o) per head (RMSNorm over Dv
+// with a weight vector of Dv entries shared by the heads).
+struct Gate {
+    const void *r;    // [B,T,H,Dv] gate pre-activation x W_r, input dtype
+    const float *w;   // [Dv] RMSNorm weight
+    float eps;
+};
+
 // Plain fp32 CUDA-core recurrence (gla_simt.cu).  Any dtype, Dk, Dv <= 128.
 cudaError_t launch_simt(const Problem &p, cudaStream_t stream);
+// The gate applied in place to a finished output (gla_simt.cu, CUDA cores; any
+// dtype, Dv <= 128): 16-byte vectors per lane, a row's lanes reduce its RMS.
+cudaError_t launch_gate_epilogue(const Problem &p, const Gate &gate, cudaStream_t stream);
 
 // Tensor-core chunkwise schedule (gla_tc.cu).
 bool tc_supported(const Problem &p);

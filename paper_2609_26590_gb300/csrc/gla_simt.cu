@@ -132,7 +132,111 @@ cudaError_t launch_typed(const Problem &p, cudaStream_t stream) {
     return cudaGetLastError();
 }
 
+// Output gate of Sec. 3.1 applied in place: one warp per (token, head) row of
+// Dv <= 128 outputs; lane j takes columns j, j + 32, j + 64, j + 96.
+template <typename E>
+__global__ void __launch_bounds__(256) gate_epilogue_kernel(E *out, const E *r, const float *w, float eps,
+                                                            long long rows, int Dv) {
+    const long long row = static_cast<long long>(blockIdx.x) * 8 + (threadIdx.x >> 5);
+    if (row >= rows) return;
+    const int lane = threadIdx.x & 31;
+    E *o_row = out + row * Dv;
+    const E *r_row = r + row * Dv;
+    float o[4];
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int col = lane + 32 * i;
+        o[i] = col < Dv ? to_f32(o_row[col]) : 0.f;
+        ss += o[i] * o[i];
+    }
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, m);
+    const float inv = rsqrtf(ss / static_cast<float>(Dv) + eps);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int col = lane + 32 * i;
+        if (col < Dv) {
+            const float z = to_f32(r_row[col]);
+            const float silu = __fdividef(z, 1.f + __expf(-z));
+            o_row[col] = from_f32<E>(silu * o[i] * inv * w[col]);
+        }
+    }
+}
+
+// The same gate for 16-byte vectors: LPR = Dv / VEC lanes per row, each moving
+// VEC = 16 / sizeof(E) contiguous values (coalesced 16-byte loads and stores).
+template <typename E, int LPR>
+__global__ void __launch_bounds__(256) gate_epilogue_vec_kernel(E *out, const E *r, const float *w, float eps,
+                                                                long long rows) {
+    constexpr int VEC = 16 / static_cast<int>(sizeof(E));
+    constexpr int Dv = LPR * VEC;
+    const long long gid = static_cast<long long>(blockIdx.x) * 256 + threadIdx.x;
+    const long long row = gid / LPR;
+    const int part = static_cast<int>(gid % LPR);
+    const bool live = row < rows;
+    const size_t off = static_cast<size_t>(live ? row : 0) * Dv + static_cast<size_t>(part) * VEC;
+    uint4 ov = live ? *reinterpret_cast<const uint4 *>(out + off) : make_uint4(0u, 0u, 0u, 0u);
+    const uint4 rv = live ? *reinterpret_cast<const uint4 *>(r + off) : make_uint4(0u, 0u, 0u, 0u);
+    const E *oe = reinterpret_cast<const E *>(&ov);
+    const E *re = reinterpret_cast<const E *>(&rv);
+    float o[VEC];
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) {
+        o[i] = to_f32(oe[i]);
+        ss += o[i] * o[i];
+    }
+#pragma unroll
+    for (int m = LPR / 2; m >= 1; m >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, m);
+    const float inv = rsqrtf(ss / static_cast<float>(Dv) + eps);
+    uint4 uv;
+    E *ue = reinterpret_cast<E *>(&uv);
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) {
+        const float z = to_f32(re[i]);
+        ue[i] = from_f32<E>(__fdividef(z, 1.f + __expf(-z)) * o[i] * inv * w[part * VEC + i]);
+    }
+    if (live) *reinterpret_cast<uint4 *>(out + off) = uv;
+}
+
+template <typename E, int LPR>
+cudaError_t launch_gate_vec(E *out, const E *r, const float *w, float eps, long long rows, cudaStream_t stream) {
+    const long long blocks = (rows * LPR + 255) / 256;
+    if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+    gate_epilogue_vec_kernel<E, LPR><<<static_cast<unsigned>(blocks), 256, 0, stream>>>(out, r, w, eps, rows);
+    return cudaGetLastError();
+}
+
+template <typename E>
+cudaError_t launch_gate_typed(const Problem &p, const Gate &gate, cudaStream_t stream) {
+    const long long rows = static_cast<long long>(p.B) * p.T * p.H;
+    E *out = static_cast<E *>(p.out);
+    const E *r = static_cast<const E *>(gate.r);
+    constexpr int VEC = 16 / static_cast<int>(sizeof(E));
+    // rows of a 16-byte-multiple width take the vector kernel (row starts stay 16-byte aligned)
+    switch (p.Dv % VEC == 0 ? p.Dv / VEC : 0) {
+    case 1: return launch_gate_vec<E, 1>(out, r, gate.w, gate.eps, rows, stream);
+    case 2: return launch_gate_vec<E, 2>(out, r, gate.w, gate.eps, rows, stream);
+    case 4: return launch_gate_vec<E, 4>(out, r, gate.w, gate.eps, rows, stream);
+    case 8: return launch_gate_vec<E, 8>(out, r, gate.w, gate.eps, rows, stream);
+    case 16: return launch_gate_vec<E, 16>(out, r, gate.w, gate.eps, rows, stream);
+    case 32: return launch_gate_vec<E, 32>(out, r, gate.w, gate.eps, rows, stream);
+    default: break;
+    }
+    const long long blocks = (rows + 7) / 8;
+    if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+    gate_epilogue_kernel<E><<<static_cast<unsigned>(blocks), 256, 0, stream>>>(out, r, gate.w, gate.eps, rows, p.Dv);
+    return cudaGetLastError();
+}
+
 }  // namespace
+
+cudaError_t launch_gate_epilogue(const Problem &p, const Gate &gate, cudaStream_t stream) {
+    if (p.dtype == 0) return launch_gate_typed<float>(p, gate, stream);
+    if (p.dtype == 1) return launch_gate_typed<__half>(p, gate, stream);
+    return launch_gate_typed<__nv_bfloat16>(p, gate, stream);
+}
 
 cudaError_t launch_simt(const Problem &p, cudaStream_t stream) {
     switch (p.dtype) {

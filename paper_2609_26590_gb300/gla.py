@@ -57,6 +57,8 @@ def load(path: Optional[str] = None):
         lib.gtr_gla_workspace_bytes.argtypes = [ci] * 7
         lib.gtr_gla_fwd_ws.restype = ci
         lib.gtr_gla_fwd_ws.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp, st, vp]
+        lib.gtr_gla_fwd_gated.restype = ci
+        lib.gtr_gla_fwd_gated.argtypes = [vp] * 6 + [ctypes.c_float] + [ci] * 8 + [vp, vp, vp]
         lib.gtr_gla_fwd_noalloc.restype = ci
         lib.gtr_gla_fwd_noalloc.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp]
         lib.gtr_gla_host_buffer_bytes.restype = st
@@ -158,6 +160,30 @@ def forward_ws(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torc
         workspace.numel() * workspace.element_size() if workspace is not None else 0,
         _stream_ptr(stream))
     _check(status, "gtr_gla_fwd_ws", lib)
+
+
+def forward_gated(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,
+                  gate: torch.Tensor, norm_weight: torch.Tensor, eps: float, grid_h: int, grid_w: int,
+                  order: int = ROW_FWD, out: Optional[torch.Tensor] = None, final_state=True,
+                  stream: Optional[torch.cuda.Stream] = None) -> Tuple[torch.Tensor, Optional[torch.Tensor]]:
+    """Mixer plus output gate through ``gtr_gla_fwd_gated``: returns
+    (u = SiLU(gate) * RMSNorm(o) per head, final_state).  gate: like v;
+    norm_weight: Dv float32 values on the device."""
+    lib = load()
+    B, H, Dk, Dv = _dims(q, v, grid_h, grid_w)
+    if out is None:
+        out = torch.empty(v.shape, dtype=v.dtype, device=v.device)
+    fs = None
+    if final_state is True:
+        fs = torch.empty((B, H, Dk, Dv), dtype=torch.float32, device=q.device)
+    elif isinstance(final_state, torch.Tensor):
+        fs = final_state
+    status = lib.gtr_gla_fwd_gated(
+        q.data_ptr(), k.data_ptr(), v.data_ptr(), log_gate.data_ptr(), gate.data_ptr(),
+        norm_weight.data_ptr(), float(eps), B, H, grid_h, grid_w, Dk, Dv, order, _DTYPES[q.dtype],
+        out.data_ptr(), fs.data_ptr() if fs is not None else None, _stream_ptr(stream))
+    _check(status, "gtr_gla_fwd_gated", lib)
+    return out, fs
 
 
 def forward_noalloc(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,
