@@ -80,7 +80,9 @@ constexpr int kSlots = 4;                 // stage slots (chunks in flight)
 constexpr int kTile16 = kC * kD * 2;      // 64 x 64 16-bit tile (SW128, 128-byte rows)
 constexpr int kTile32 = kC * kD * 4;      // 64 x 64 fp32 tile (two 32-column K-blocks)
 constexpr int kThreads = 512;
-constexpr int kHeights = 8;               // TMA box heights 8, 16, ..., 64
+constexpr int kHeights = 15;              // TMA box heights 1 .. 7, then 8, 16, ..., 64
+// Rows of the TMA box of height index hi (one tensor map per height).
+__host__ __device__ constexpr int box_height(int hi) { return hi < 7 ? hi + 1 : 8 * (hi - 6); }
 constexpr uint64_t kWaitLimitNs = 1000000000ull;  // bounded waits give up after 1 s
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kGateMinLog2 = -1.0e4f * 1.4426950408889634f;  // g < -1e4 acts as -1e4
@@ -133,7 +135,7 @@ constexpr uint32_t kColA = 0, kColP = 128, kColU = 256, kColO = 384;
 enum { T_Q = 0, T_K = 1, T_V = 2, T_G = 3, kTensors = 4 };
 
 struct TcParams {
-    CUtensorMap maps[kTensors][kHeights];  // box height 8 (i + 1)
+    CUtensorMap maps[kTensors][kHeights];  // box height box_height(i)
     void *out;
     float *final_state;
     int H, grid_h, grid_w, order, n_chunks, T;
@@ -240,9 +242,13 @@ __device__ __forceinline__ StreamPos stream_pos(int v, int L, int nh, int lognv,
 
 // Visit the TMA load boxes of one chunk: calls f(map height index, smem row, c2, c3).
 // Row orders: one 64-row box at token w0 (rows outside the sequence are
-// zero-filled).  Column orders: one box per column segment, of the segment's
-// exact height, plus zero-fill boxes placed past the last column for rows
-// outside the sequence.  Heights and offsets are multiples of 8 (T and grid_h are).
+// zero-filled).  Column orders: boxes for each column segment, of the segment's
+// exact height (at most two: its multiple of 8 and the remainder), plus zero-fill
+// boxes placed past the last column for rows outside the sequence.
+//
+// Runs of rows down one column (at most two zero-fill runs, then the column
+// segments), each loaded as at most two boxes: its multiple of 8 and the remainder.
+// One call site for f keeps the producer's issue code small.
 template <typename F>
 __device__ __forceinline__ void chunk_load_boxes(int order, int T, int grid_h, int grid_w, int c, F &&f) {
     const int w0 = chunk_w0(order, T, c);
@@ -251,14 +257,33 @@ __device__ __forceinline__ void chunk_load_boxes(int order, int T, int grid_h, i
         return;
     }
     const int lo = w0 < 0 ? 0 : w0, hi = (w0 + kC > T) ? T : w0 + kC;
-    if (lo > w0) f((lo - w0) / 8 - 1, 0, grid_w, 0);
-    if (hi < w0 + kC) f((w0 + kC - hi) / 8 - 1, hi - w0, grid_w, 0);
-    for (int w = lo; w < hi;) {
-        const int x = w / grid_h, y = w - x * grid_h;
-        int len = grid_h - y;
-        if (len > hi - w) len = hi - w;
-        f(len / 8 - 1, w - w0, x, y);
-        w += len;
+    int phase = 0, w = lo;
+#pragma unroll 1
+    for (;;) {
+        int len, row, c2, c3;
+        if (phase == 0) {  // rows before the sequence: zero-fill past the last column
+            phase = 1;
+            if (lo <= w0) continue;
+            len = lo - w0, row = 0, c2 = grid_w, c3 = 0;
+        } else if (phase == 1) {  // rows after the sequence
+            phase = 2;
+            if (hi >= w0 + kC) continue;
+            len = w0 + kC - hi, row = hi - w0, c2 = grid_w, c3 = 0;
+        } else {  // the next column segment
+            if (w >= hi) break;
+            const int x = w / grid_h, y = w - x * grid_h;
+            len = grid_h - y;
+            if (len > hi - w) len = hi - w;
+            row = w - w0, c2 = x, c3 = y;
+            w += len;
+        }
+        const int len8 = len & ~7;
+#pragma unroll 1
+        for (int part = 0; part < 2; ++part) {
+            const int n = part == 0 ? len8 : len - len8;
+            if (n == 0) continue;
+            f(part == 0 ? 6 + n / 8 : n - 1, row + (part == 0 ? 0 : len8), c2, c3 + (part == 0 ? 0 : len8));
+        }
     }
 }
 
@@ -1019,7 +1044,7 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     e.key = key;
     for (int t = 0; t < kTensors; ++t)
         for (int hi = 0; hi < kHeights; ++hi)
-            if (!encode_map(&e.maps[t][hi], key.ptr[t], p, t == T_V ? p.Dv : p.Dk, 8 * (hi + 1))) return false;
+            if (!encode_map(&e.maps[t][hi], key.ptr[t], p, t == T_V ? p.Dv : p.Dk, box_height(hi))) return false;
     std::memcpy(out, e.maps, sizeof(out));
     g_map_cache.push_front(e);
     if (g_map_cache.size() > kMapCacheSize) g_map_cache.pop_back();
@@ -1079,8 +1104,6 @@ size_t tc_workspace_bytes(const Problem &p) {
 bool tc_supported(const Problem &p) {
     if (p.dtype != 1 && p.dtype != 2) return false;       // fp16 / bf16 operands only
     if ((p.Dk != 64 && p.Dk != 128) || (p.Dv != 64 && p.Dv != 128)) return false;  // 64-wide halves
-    if (p.T % 8 != 0) return false;                        // box heights are multiples of 8
-    if ((p.order >> 1) != 0 && p.grid_h % 8 != 0) return false;  // column segments are too
     if (p.T > (1 << 30)) return false;
     return get_encode() != nullptr;
 }

@@ -98,6 +98,8 @@ SMALL = [
     (2, 2, 8, 24, 64, 128, "f16", 16.0, 0.0),
     (1, 3, 16, 12, 128, 64, "bf16", 1.0, -1.0),
     (1, 2, 24, 8, 128, 128, "f16", 1.0, -3.0),
+    (1, 6, 44, 44, 64, 64, "f16", 16.0, 0.0),     # 704^2 input at stride 16 (1936 tokens): ragged columns
+    (2, 2, 7, 11, 64, 64, "bf16", 1.0, -1.0),      # odd grid: every column segment has a remainder box
 ]
 
 
