@@ -187,8 +187,9 @@ gtr_status_t gtr_gla_fwd_noalloc(const void *q, const void *k, const void *v, co
                                  float *final_state, cudaStream_t stream);
 
 /* 1 when the tensor-core schedule supports these arguments, else 0: fp16 or
- * bf16, Dk and Dv each 64 or 128 (processed in 64-channel key halves and
- * 64-column value slices); any grid. */
+ * bf16, Dk and Dv each a multiple of 8 up to 128 (processed in 64-channel key
+ * halves and 64-column value slices, a narrower last one zero-padded on
+ * load); any grid. */
 int gtr_gla_tc_supported(int B, int H, int grid_h, int grid_w, int Dk, int Dv,
                          gtr_scan_t scan_order, gtr_dtype_t dtype);
 

@@ -139,9 +139,9 @@ struct TcParams {
     void *out;
     float *final_state;
     int H, grid_h, grid_w, order, n_chunks, T;
-    int Dk, Dv;                            // 64 or 128 each
-    int nh;                                // Dk / 64: 64-channel key halves per chunk
-    int nv;                                // Dv / 64: 64-column value slices, one per CTA work unit
+    int Dk, Dv;                            // multiples of 8 up to 128 (the tensors' row widths)
+    int nh;                                // ceil(Dk / 64): 64-channel key halves per chunk
+    int nv;                                // ceil(Dv / 64): 64-column value slices, one per CTA work unit
     int n_units;                           // work units of this launch, dealt out round-robin to the CTAs
     int seg_len;                           // chunks per segment (a sequence split into nseg equal segments)
     int nseg;                              // segments per sequence (1: no split)
@@ -899,11 +899,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
                         if (ps.vb == 0 && hc == 0) base[(size_t)kDk * kDv + 64 * ps.a + row] = dp;
                     }
-                } else if (ps.c == N - 1 && p.final_state != nullptr) {  // the sequence's final state
-                    float4 *dst = reinterpret_cast<float4 *>(
-                        p.final_state + ((size_t)ps.bh * kDk + 64 * ps.a + row) * kDv + 64 * ps.vb + ch0);
+                } else if (ps.c == N - 1 && p.final_state != nullptr && 64 * ps.a + row < p.Dk) {
+                    // the sequence's final state [Dk][Dv] (padded channels and columns stay behind)
+                    const int col0 = 64 * ps.vb + ch0;
+                    float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)ps.bh * p.Dk + 64 * ps.a + row) * p.Dv + col0);
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
+                    for (int j = 0; j < 8; ++j)
+                        if (col0 + 4 * j < p.Dv) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // U(c) drained: counts for chunk c + 2
@@ -941,10 +943,12 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 const StreamPos po = stream_pos(co, L, nh, lognv, kSplit ? p.nsu : 1);
                 const int b = po.bh / p.H, h = po.bh % p.H;
                 const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
-                if (t >= 0) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * kDv + 64 * po.vb + ch0);
+                if (t >= 0) {  // the row's columns inside Dv (padded columns stay behind)
+                    const int col0 = 64 * po.vb + ch0;
+                    uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * p.Dv + col0);
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) dst[q] = make_uint4(ow[4 * q], ow[4 * q + 1], ow[4 * q + 2], ow[4 * q + 3]);
+                    for (int q = 0; q < 4; ++q)
+                        if (col0 + 8 * q < p.Dv) dst[q] = make_uint4(ow[4 * q], ow[4 * q + 1], ow[4 * q + 2], ow[4 * q + 3]);
                 }
             }
         }
@@ -1078,9 +1082,13 @@ cudaError_t sm_count(int *n_sm) {
 // Segments per sequence.  A launch whose work units fill fewer than half of the
 // SMs splits every sequence into the most equal segments (a divisor of the chunk
 // count, at least kMinSegChunks chunks each) that still fit one wave.
+// Key channels and value columns are processed in 64-wide halves and slices; a
+// narrower last one is zero-padded by the TMA loads (boxes past the tensor's row).
+int pad64(int d) { return (d + 63) / 64 * 64; }
+
 int choose_nseg(const Problem &p, int n_sm) {
     const long long N = (p.T + kC - 1) / kC;
-    const long long units = (long long)p.B * p.H * (p.Dv / 64);
+    const long long units = (long long)p.B * p.H * (pad64(p.Dv) / 64);
     if (units * 2 > n_sm) return 1;
     int best = 1;
     for (long long d = 2; d <= N; ++d)
@@ -1090,7 +1098,7 @@ int choose_nseg(const Problem &p, int n_sm) {
 
 size_t summary_bytes(const Problem &p, int nseg) {
     if (nseg <= 1) return 0;
-    return (size_t)p.B * p.H * (nseg - 1) * ((size_t)p.Dk * p.Dv + p.Dk) * sizeof(float);
+    return (size_t)p.B * p.H * (nseg - 1) * ((size_t)pad64(p.Dk) * pad64(p.Dv) + pad64(p.Dk)) * sizeof(float);
 }
 
 }  // namespace
@@ -1103,7 +1111,8 @@ size_t tc_workspace_bytes(const Problem &p) {
 
 bool tc_supported(const Problem &p) {
     if (p.dtype != 1 && p.dtype != 2) return false;       // fp16 / bf16 operands only
-    if ((p.Dk != 64 && p.Dk != 128) || (p.Dv != 64 && p.Dv != 128)) return false;  // 64-wide halves
+    // rows of 16-byte multiples (TMA strides); up to two 64-wide halves / slices
+    if (p.Dk % 8 != 0 || p.Dv % 8 != 0 || p.Dk > 128 || p.Dv > 128) return false;
     if (p.T > (1 << 30)) return false;
     return get_encode() != nullptr;
 }
@@ -1124,8 +1133,8 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     tp.n_chunks = static_cast<int>((p.T + kC - 1) / kC);
     tp.Dk = p.Dk;
     tp.Dv = p.Dv;
-    tp.nh = p.Dk / 64;
-    tp.nv = p.Dv / 64;
+    tp.nh = pad64(p.Dk) / 64;
+    tp.nv = pad64(p.Dv) / 64;
     int nseg = choose_nseg(p, n_sm);
     if (nseg > 1 && (workspace == nullptr || workspace_bytes < summary_bytes(p, nseg))) nseg = 1;
     tp.nseg = nseg;

@@ -100,6 +100,8 @@ SMALL = [
     (1, 2, 24, 8, 128, 128, "f16", 1.0, -3.0),
     (1, 6, 44, 44, 64, 64, "f16", 16.0, 0.0),     # 704^2 input at stride 16 (1936 tokens): ragged columns
     (2, 2, 7, 11, 64, 64, "bf16", 1.0, -1.0),      # odd grid: every column segment has a remainder box
+    (2, 2, 16, 16, 32, 64, "bf16", 1.0, -1.0),     # the paper's dk = 32, dv = 64: zero-padded key half
+    (1, 3, 12, 10, 96, 40, "bf16", 16.0, 0.0),     # padded second key half and value slice
 ]
 
 
@@ -153,6 +155,7 @@ SPLIT = [
     (1, 1, 48, 40, 64, 64, "f16", 1.0, -1.0, 0.0),      # strong decay: tf32 scores in both passes
     (1, 1, 32, 32, 128, 128, "bf16", 16.0, 0.0, 0.0),   # two key halves, two value slices
     (1, 1, 64, 16, 128, 64, "f16", 16.0, 0.0, 0.02),    # Dk != Dv, some gamma = 0 gates (exact path)
+    (1, 2, 64, 40, 32, 64, "bf16", 16.0, 0.0, 0.0),     # padded key half: summaries keep the padded layout
 ]
 
 
