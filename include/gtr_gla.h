@@ -203,9 +203,14 @@ size_t gtr_gla_host_buffer_bytes(int B, int H, int grid_h, int grid_w, int Dk, i
  * asynchronous) into `dev_buffer` (caller-owned device memory of at least
  * gtr_gla_host_buffer_bytes() bytes), runs gtr_gla_fwd on `stream`, and
  * copies `out` (and `final_state` when non-NULL) back to the host pointers.
- * Everything is enqueued on `stream`; synchronise it before reading the
- * results.  Errors as gtr_gla_fwd, plus GTR_ERR_WORKSPACE when dev_buffer is
- * NULL or too small. */
+ * The batch is processed in up to four pieces so that uploads, compute and
+ * downloads overlap: the uploads and downloads run on two internal streams of
+ * the current device (created with a set of events on its first call and kept
+ * until exit), forked from and joined back into `stream` with events, so the
+ * call is ordered on `stream` like any other work: synchronise it before
+ * reading the results.  Calls from several host threads are serialised.
+ * Errors as gtr_gla_fwd, plus GTR_ERR_WORKSPACE when dev_buffer is NULL or
+ * too small. */
 gtr_status_t gtr_gla_fwd_host(const void *q_host, const void *k_host, const void *v_host,
                               const void *log_gate_host, int B, int H, int grid_h, int grid_w,
                               int Dk, int Dv, gtr_scan_t scan_order, gtr_dtype_t dtype,

@@ -141,6 +141,41 @@ cudaError_t noalloc_scratch(void **ptr) {
     return cudaSuccess;
 }
 
+// Per-device streams and events of gtr_gla_fwd_host's pipeline (created on first
+// use and kept; calls are serialised by g_pipe_mutex, so the events are reused).
+constexpr int kPipePieces = 4;
+struct HostPipe {
+    bool ready = false;
+    cudaStream_t up = nullptr, down = nullptr;
+    cudaEvent_t fork = nullptr, join = nullptr;
+    cudaEvent_t in[kPipePieces] = {}, done[kPipePieces] = {};
+};
+std::mutex g_pipe_mutex;
+std::vector<HostPipe> g_pipe;
+
+cudaError_t host_pipe(HostPipe **out) {  // caller holds g_pipe_mutex
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if ((size_t)dev >= g_pipe.size()) g_pipe.resize(dev + 1);
+    HostPipe &hp = g_pipe[dev];
+    if (!hp.ready) {
+        const unsigned ef = cudaEventDisableTiming;
+        if ((e = cudaStreamCreateWithFlags(&hp.up, cudaStreamNonBlocking)) != cudaSuccess ||
+            (e = cudaStreamCreateWithFlags(&hp.down, cudaStreamNonBlocking)) != cudaSuccess ||
+            (e = cudaEventCreateWithFlags(&hp.fork, ef)) != cudaSuccess ||
+            (e = cudaEventCreateWithFlags(&hp.join, ef)) != cudaSuccess)
+            return e;
+        for (int j = 0; j < kPipePieces; ++j)
+            if ((e = cudaEventCreateWithFlags(&hp.in[j], ef)) != cudaSuccess ||
+                (e = cudaEventCreateWithFlags(&hp.done[j], ef)) != cudaSuccess)
+                return e;
+        hp.ready = true;
+    }
+    *out = &hp;
+    return cudaSuccess;
+}
+
 // Dispatch of one validated, non-empty problem; `ws` null means the internal workspace.
 gtr_status_t dispatch(const gtr::Problem &p, gtr_schedule_t schedule, void *ws, size_t ws_bytes, bool own_ws,
                       cudaStream_t stream) {
@@ -277,24 +312,47 @@ gtr_status_t gtr_gla_fwd_host(const void *q_host, const void *k_host, const void
     if (B == 0 || H == 0) return GTR_OK;
     const size_t T = (size_t)grid_h * grid_w, es = elem_size(dtype);
     const size_t bk = (size_t)B * T * H * Dk * es, bv = (size_t)B * T * H * Dv * es;
-    const size_t bfs = (size_t)B * H * Dk * Dv * 4;
     char *base = static_cast<char *>(dev_buffer);
     char *dq = base, *dk = dq + round_up(bk, 256), *dg = dk + round_up(bk, 256);
     char *dv = dg + round_up(bk, 256), *dout = dv + round_up(bv, 256);
     float *dfs = with_fs ? reinterpret_cast<float *>(dout + round_up(bv, 256)) : nullptr;
-    cudaError_t e;
-    if ((e = cudaMemcpyAsync(dq, q_host, bk, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(dk, k_host, bk, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(dg, log_gate_host, bk, cudaMemcpyHostToDevice, stream)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(dv, v_host, bv, cudaMemcpyHostToDevice, stream)) != cudaSuccess)
+    // Batch pieces in a pipeline: piece j's uploads (stream `up`) overlap piece j-1's
+    // forward (the caller's stream) and piece j-2's downloads (stream `down`); events
+    // fork the two internal streams off the caller's stream and join them back.
+    HostPipe *hp = nullptr;
+    std::lock_guard<std::mutex> lock(g_pipe_mutex);
+    cudaError_t e = host_pipe(&hp);
+    if (e != cudaSuccess) return cuda_fail(e);
+    const int P = B < kPipePieces ? B : kPipePieces;
+    const size_t row_k = T * H * Dk * es, row_v = T * H * Dv * es, row_fs = (size_t)H * Dk * Dv * 4;
+    if ((e = cudaEventRecord(hp->fork, stream)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(hp->up, hp->fork, 0)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(hp->down, hp->fork, 0)) != cudaSuccess)
         return cuda_fail(e);
-    st = gtr_gla_fwd(dq, dk, dv, dg, B, H, grid_h, grid_w, Dk, Dv, scan_order, dtype, dout, dfs,
-                     stream);
-    if (st != GTR_OK) return st;
-    if ((e = cudaMemcpyAsync(out_host, dout, bv, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
-        return cuda_fail(e);
-    if (with_fs &&
-        (e = cudaMemcpyAsync(final_state_host, dfs, bfs, cudaMemcpyDeviceToHost, stream)) != cudaSuccess)
+    for (int j = 0; j < P; ++j) {
+        const size_t b0 = (size_t)B * j / P, nb = (size_t)B * (j + 1) / P - b0;
+        const size_t ok0 = b0 * row_k, ov0 = b0 * row_v, nk = nb * row_k, nvb = nb * row_v;
+        if ((e = cudaMemcpyAsync(dq + ok0, static_cast<const char *>(q_host) + ok0, nk, cudaMemcpyHostToDevice, hp->up)) != cudaSuccess ||
+            (e = cudaMemcpyAsync(dk + ok0, static_cast<const char *>(k_host) + ok0, nk, cudaMemcpyHostToDevice, hp->up)) != cudaSuccess ||
+            (e = cudaMemcpyAsync(dg + ok0, static_cast<const char *>(log_gate_host) + ok0, nk, cudaMemcpyHostToDevice, hp->up)) != cudaSuccess ||
+            (e = cudaMemcpyAsync(dv + ov0, static_cast<const char *>(v_host) + ov0, nvb, cudaMemcpyHostToDevice, hp->up)) != cudaSuccess ||
+            (e = cudaEventRecord(hp->in[j], hp->up)) != cudaSuccess ||
+            (e = cudaStreamWaitEvent(stream, hp->in[j], 0)) != cudaSuccess)
+            return cuda_fail(e);
+        st = gtr_gla_fwd(dq + ok0, dk + ok0, dv + ov0, dg + ok0, static_cast<int>(nb), H, grid_h, grid_w, Dk, Dv,
+                         scan_order, dtype, dout + ov0, with_fs ? dfs + b0 * row_fs / 4 : nullptr, stream);
+        if (st != GTR_OK) return st;
+        if ((e = cudaEventRecord(hp->done[j], stream)) != cudaSuccess ||
+            (e = cudaStreamWaitEvent(hp->down, hp->done[j], 0)) != cudaSuccess ||
+            (e = cudaMemcpyAsync(static_cast<char *>(out_host) + ov0, dout + ov0, nvb, cudaMemcpyDeviceToHost, hp->down)) != cudaSuccess)
+            return cuda_fail(e);
+        if (with_fs && (e = cudaMemcpyAsync(reinterpret_cast<char *>(final_state_host) + b0 * row_fs,
+                                            reinterpret_cast<char *>(dfs) + b0 * row_fs, nb * row_fs,
+                                            cudaMemcpyDeviceToHost, hp->down)) != cudaSuccess)
+            return cuda_fail(e);
+    }
+    if ((e = cudaEventRecord(hp->join, hp->down)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(stream, hp->join, 0)) != cudaSuccess)
         return cuda_fail(e);
     return GTR_OK;
 }
