@@ -50,6 +50,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--graph", action="store_true",
+                    help="replay each step from a CUDA graph (one per scan order) instead of eager calls")
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch size (smaller cases for profiling)")
     return ap.parse_args()
@@ -305,6 +307,38 @@ def main():
     if gla.sync_status() != 0:
         raise RuntimeError("device status word set during warm-up")
 
+    run = step
+    if args.graph:
+        # one graph per scan order; the mixer is captured through the caller-workspace entry
+        # point (no allocation, no synchronisation), the gated call after the warm-up above
+        # has grown the internal workspace it uses
+        if schedule != "auto":
+            raise SystemExit("--graph times the automatic schedule only")
+        ws_n = gla.workspace_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt)
+        ws = torch.empty(ws_n, dtype=torch.uint8, device=dev) if ws_n else None
+        cap = torch.cuda.Stream(dev)
+        cap.wait_stream(stream)
+        graphs = []
+        with torch.cuda.stream(cap):
+            for j in range(len(orders)):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=cap):
+                    if args.gated:
+                        step(j)
+                    else:
+                        gla.forward_ws(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, orders[j], out, fs, ws,
+                                       stream=cap)
+                graphs.append(g)
+        stream.wait_stream(cap)
+        for j in range(max(3, args.warmup)):
+            graphs[j % len(graphs)].replay()
+        torch.cuda.synchronize()
+        if gla.sync_status() != 0:
+            raise RuntimeError("device status word set during graph warm-up")
+
+        def run(i):
+            graphs[i % len(graphs)].replay()
+
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     if pg:
@@ -316,7 +350,7 @@ def main():
         t_begin.record(stream)
         for i in range(args.steps):
             starts[i].record(stream)
-            step(i)
+            run(i)
             ends[i].record(stream)
         t_end.record(stream)
         torch.cuda.synchronize()
@@ -394,7 +428,8 @@ def main():
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": w.dtype, "data": "synthetic (seeded, workload recipe in workloads.py)",
-                "config": workload_config(w, world, dict({"schedule": schedule},
+                "config": workload_config(w, world, dict({"schedule": schedule,
+                                                          "launch": "cuda-graph replay" if args.graph else "eager"},
                                                          **({"epilogue": "output gate u = SiLU(r) * RMSNorm(o), "
                                                              "second kernel right after the mixer"}
                                                             if args.gated else {}))),

@@ -90,7 +90,8 @@ typedef enum { GTR_SCHED_AUTO = 0, GTR_SCHED_SIMT = 1, GTR_SCHED_TC = 2 } gtr_sc
 /* Forward of the token mixer with the AUTO schedule (argument rules above).
  * Returns GTR_OK once the work is enqueued on `stream`.  When few, long
  * sequences would leave most SMs idle, the tensor-core schedule splits each
- * sequence into equal segments (a first pass stores every segment's end state
+ * sequence into segments of equal length but the last, which may run past the
+ * sequence over all-zero chunks (a first pass stores every segment's end state
  * from zero and its total decay, the second pass starts each segment from the
  * fold of the earlier ones: the state carry of Eq. chunk_boundary_main applied
  * across segments).  Those summaries live in an internal per-device workspace

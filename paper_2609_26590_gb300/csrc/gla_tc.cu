@@ -57,6 +57,7 @@
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
+#include <atomic>
 #include <cstdlib>
 #include <cstring>
 #include <list>
@@ -93,7 +94,7 @@ enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
 // Kernel passes: kFull (sequences whole), kSplitFull (outputs of segments that
 // start from the fold of the earlier segments' summaries), kSummary (the summaries).
 enum : int { kFull = 0, kSplitFull = 1, kSummary = 2 };
-constexpr int kMinSegChunks = 4;          // a split segment keeps at least this many chunks
+constexpr int kMinSegChunks = 2;          // a split segment keeps at least this many chunks
 
 // Shared-memory map (byte offsets from a 1024-aligned base).
 constexpr int kSlotBytes = 4 * kTile16;                        // q @0, k @8K, v @16K, g @24K
@@ -143,7 +144,7 @@ struct TcParams {
     int nh;                                // ceil(Dk / 64): 64-channel key halves per chunk
     int nv;                                // ceil(Dv / 64): 64-column value slices, one per CTA work unit
     int n_units;                           // work units of this launch, dealt out round-robin to the CTAs
-    int seg_len;                           // chunks per segment (a sequence split into nseg equal segments)
+    int seg_len;                           // chunks per segment (the last one may run past the sequence)
     int nseg;                              // segments per sequence (1: no split)
     int nsu;                               // segments per (sequence, value slice) among this launch's units
     float *summary;                        // nseg > 1: per (sequence, segment < nseg - 1) end state from zero
@@ -254,6 +255,10 @@ __device__ __forceinline__ void chunk_load_boxes(int order, int T, int grid_h, i
     const int w0 = chunk_w0(order, T, c);
     if ((order >> 1) == 0) {
         f(kHeights - 1, 0, w0, 0);
+        return;
+    }
+    if (w0 >= T || w0 + kC <= 0) {  // a padding chunk wholly past the sequence: all zeros
+        f(kHeights - 1, 0, grid_w, 0);
         return;
     }
     const int lo = w0 < 0 ? 0 : w0, hi = (w0 + kC > T) ? T : w0 + kC;
@@ -1057,9 +1062,17 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
 
 template <typename E, int NH, int NV, int MODE>
 cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
-    cudaError_t e =
-        cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+    // the shared-memory opt-in, once per process and device (setting it again is harmless)
+    static std::atomic<unsigned long long> set_on_devices(0);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (!(set_on_devices.load(std::memory_order_relaxed) & bit)) {
+        e = cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e != cudaSuccess) return e;
+        set_on_devices.fetch_or(bit);
+    }
     gla_tc_kernel<E, NH, NV, MODE><<<grid, kThreads, kSmemBytes, stream>>>(tp);
     return cudaSuccess;
 }
@@ -1072,27 +1085,60 @@ cudaError_t launch_shape(dim3 grid, const TcParams &tp, cudaStream_t stream) {
     return tp.nv == 1 ? launch_kernel<E, 2, 1, MODE>(grid, tp, stream) : launch_kernel<E, 2, 2, MODE>(grid, tp, stream);
 }
 
-cudaError_t sm_count(int *n_sm) {
+cudaError_t sm_count(int *n_sm) {  // cached per device
+    static std::atomic<int> cache[64] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    return cudaDeviceGetAttribute(n_sm, cudaDevAttrMultiProcessorCount, dev);
+    if (dev >= 0 && dev < 64) {
+        const int v = cache[dev].load(std::memory_order_relaxed);
+        if (v > 0) {
+            *n_sm = v;
+            return cudaSuccess;
+        }
+    }
+    e = cudaDeviceGetAttribute(n_sm, cudaDevAttrMultiProcessorCount, dev);
+    if (e == cudaSuccess && dev >= 0 && dev < 64) cache[dev].store(*n_sm, std::memory_order_relaxed);
+    return e;
 }
 
-// Segments per sequence.  A launch whose work units fill fewer than half of the
-// SMs splits every sequence into the most equal segments (a divisor of the chunk
-// count, at least kMinSegChunks chunks each) that still fit one wave.
 // Key channels and value columns are processed in 64-wide halves and slices; a
 // narrower last one is zero-padded by the TMA loads (boxes past the tensor's row).
 int pad64(int d) { return (d + 63) / 64 * 64; }
 
-int choose_nseg(const Problem &p, int n_sm) {
+// Segments per sequence.  A launch whose work units fill fewer than half of the
+// SMs splits every sequence into segments of `len` chunks, so that the split
+// launch still fits one wave (units x ceil(N / len) <= SMs).  The split's critical
+// path is the last segment: `len` chunks in each of the two passes, plus the fold
+// of the nseg - 1 earlier summaries into its start state.  On a GB300 a chunk of
+// segment length costs about 2.5 us over both passes and a folded summary about
+// 0.55 us, so the length minimises 9 len + 2 ceil(N / len) + 10 (the second
+// launch), at least kMinSegChunks; the unsplit launch (about 6 per chunk) is
+// kept when it is cheaper.
+// The last segment may be shorter than the others: its chunks past the sequence
+// load as zeros (no key, decay 1), so they leave the state unchanged, and their
+// outputs are not stored.
+struct Split {
+    int nseg;  // segments per sequence (1: no split)
+    int len;   // chunks per segment
+};
+
+Split choose_split(const Problem &p, int n_sm) {
     const long long N = (p.T + kC - 1) / kC;
     const long long units = (long long)p.B * p.H * (pad64(p.Dv) / 64);
-    if (units * 2 > n_sm) return 1;
-    int best = 1;
-    for (long long d = 2; d <= N; ++d)
-        if (N % d == 0 && N / d >= kMinSegChunks && units * d <= n_sm) best = static_cast<int>(d);
+    const Split none{1, static_cast<int>(N)};
+    if (units * 2 > n_sm) return none;
+    Split best = none;
+    long long best_cost = 6 * N;
+    for (long long L = kMinSegChunks; L < N; ++L) {
+        const long long d = (N + L - 1) / L;
+        if (units * d > n_sm) continue;
+        const long long cost = 9 * L + 2 * d + 10;
+        if (cost < best_cost) {
+            best = Split{static_cast<int>(d), static_cast<int>(L)};
+            best_cost = cost;
+        }
+    }
     return best;
 }
 
@@ -1106,7 +1152,7 @@ size_t summary_bytes(const Problem &p, int nseg) {
 size_t tc_workspace_bytes(const Problem &p) {
     int n_sm = 0;
     if (sm_count(&n_sm) != cudaSuccess) return 0;
-    return summary_bytes(p, choose_nseg(p, n_sm));
+    return summary_bytes(p, choose_split(p, n_sm).nseg);
 }
 
 bool tc_supported(const Problem &p) {
@@ -1135,10 +1181,12 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     tp.Dv = p.Dv;
     tp.nh = pad64(p.Dk) / 64;
     tp.nv = pad64(p.Dv) / 64;
-    int nseg = choose_nseg(p, n_sm);
-    if (nseg > 1 && (workspace == nullptr || workspace_bytes < summary_bytes(p, nseg))) nseg = 1;
+    Split sp = choose_split(p, n_sm);
+    if (sp.nseg > 1 && (workspace == nullptr || workspace_bytes < summary_bytes(p, sp.nseg)))
+        sp = Split{1, tp.n_chunks};
+    const int nseg = sp.nseg;
     tp.nseg = nseg;
-    tp.seg_len = tp.n_chunks / nseg;
+    tp.seg_len = sp.len;
     tp.summary = static_cast<float *>(workspace);
     // test hook for the timeout path (no fault: the data of one chunk simply never arrives)
     const char *drop = std::getenv("GTR_GLA_TEST_DROP_LOAD");

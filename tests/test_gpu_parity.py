@@ -148,14 +148,20 @@ def test_many_sequences_per_cta(case):
         assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, dtype, f"state {order}")
 
 
-# Few, long sequences: the tensor-core schedule splits each into equal segments
-# (a summary pass, then every segment from the fold of the earlier summaries).
+# Few, long sequences: the tensor-core schedule splits each into segments of equal
+# length but the last (a summary pass, then every segment from the fold of the earlier
+# summaries).  When the chunk count is not a multiple of the length, the last segment
+# runs past the sequence over all-zero padding chunks, in every scan order.
 SPLIT = [
-    (1, 2, 64, 64, 64, 64, "bf16", 16.0, 0.0, 0.0),     # 8 segments of 8 chunks
-    (1, 1, 48, 40, 64, 64, "f16", 1.0, -1.0, 0.0),      # strong decay: tf32 scores in both passes
+    (1, 2, 64, 64, 64, 64, "bf16", 16.0, 0.0, 0.0),     # 64 chunks, segments of 4
+    (1, 1, 48, 40, 64, 64, "f16", 1.0, -1.0, 0.0),      # strong decay: tf32 scores; 30 chunks, 2 padding
     (1, 1, 32, 32, 128, 128, "bf16", 16.0, 0.0, 0.0),   # two key halves, two value slices
     (1, 1, 64, 16, 128, 64, "f16", 16.0, 0.0, 0.02),    # Dk != Dv, some gamma = 0 gates (exact path)
     (1, 2, 64, 40, 32, 64, "bf16", 16.0, 0.0, 0.0),     # padded key half: summaries keep the padded layout
+    (1, 6, 40, 40, 64, 64, "f16", 16.0, 0.0, 0.0),      # 25 chunks: 3 padding chunks in the last segment
+    (1, 6, 44, 44, 64, 64, "bf16", 16.0, 0.0, 0.0),     # 31 chunks, the last one ragged (16 tokens)
+    (1, 3, 40, 36, 32, 64, "bf16", 16.0, 0.0, 0.0),     # Dk = 32, Dv = 64; 23 chunks
+    (1, 1, 36, 36, 128, 128, "f16", 16.0, 0.0, 0.0),    # two key halves over padding chunks; 21 chunks
 ]
 
 
