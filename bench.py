@@ -309,9 +309,8 @@ def main():
 
     run = step
     if args.graph:
-        # one graph per scan order; the mixer is captured through the caller-workspace entry
-        # point (no allocation, no synchronisation), the gated call after the warm-up above
-        # has grown the internal workspace it uses
+        # one graph per scan order, captured through the caller-workspace entry points
+        # (no allocation, no synchronisation; the split schedule stays on)
         if schedule != "auto":
             raise SystemExit("--graph times the automatic schedule only")
         ws_n = gla.workspace_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt)
@@ -324,7 +323,8 @@ def main():
                 g = torch.cuda.CUDAGraph()
                 with torch.cuda.graph(g, stream=cap):
                     if args.gated:
-                        step(j)
+                        gla.forward_gated(t["q"], t["k"], t["v"], t["g"], gate_r, gate_w, 1e-5, w.grid_h,
+                                          w.grid_w, orders[j], out=out, final_state=fs, stream=cap, workspace=ws)
                     else:
                         gla.forward_ws(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, orders[j], out, fs, ws,
                                        stream=cap)

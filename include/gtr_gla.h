@@ -121,6 +121,18 @@ gtr_status_t gtr_gla_fwd_sched(const void *q, const void *k, const void *v,
 size_t gtr_gla_workspace_bytes(int B, int H, int grid_h, int grid_w, int Dk, int Dv,
                                gtr_dtype_t dtype);
 
+/* The sequence split the tensor-core schedule would use for these shapes on a
+ * device with n_sm SMs: *nseg segments per sequence of *seg_len 64-token chunks
+ * each (the last segment may run past the sequence over all-zero padding
+ * chunks; *nseg == 1: unsplit, *seg_len = the chunk count).  Host arithmetic
+ * only: no device is queried, so it answers for any SM count.  The split is the
+ * chunkwise state carry (Eq. chunk_boundary_main) applied across segments; the
+ * segment length minimises a cost model of the split's critical path measured
+ * on a GB300.  Returns GTR_ERR_INVALID_ARG for invalid shapes, n_sm < 1 or
+ * NULL outputs (the outputs are then not written). */
+gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm,
+                                int *nseg, int *seg_len);
+
 /* gtr_gla_fwd with a caller-owned device workspace of workspace_bytes >=
  * gtr_gla_workspace_bytes() bytes, 256-byte aligned (may be NULL when that is
  * 0).  The call allocates nothing and does not synchronise.  Returns
@@ -149,6 +161,19 @@ gtr_status_t gtr_gla_fwd_gated(const void *q, const void *k, const void *v, cons
                                const void *gate, const float *norm_weight, float eps, int B, int H,
                                int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
                                gtr_dtype_t dtype, void *out, float *final_state, cudaStream_t stream);
+
+/* gtr_gla_fwd_gated with a caller-owned device workspace, as gtr_gla_fwd_ws:
+ * workspace_bytes >= gtr_gla_workspace_bytes() (the gate needs none of its
+ * own), 256-byte aligned, NULL allowed when that is 0.  Allocates nothing and
+ * does not synchronise, so it may be captured into a CUDA graph with the split
+ * schedule (gtr_gla_fwd_gated under capture runs unsplit).  Returns
+ * GTR_ERR_WORKSPACE when the workspace is missing or too small; other
+ * arguments and errors as gtr_gla_fwd_gated. */
+gtr_status_t gtr_gla_fwd_gated_ws(const void *q, const void *k, const void *v, const void *log_gate,
+                                  const void *gate, const float *norm_weight, float eps, int B, int H,
+                                  int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
+                                  gtr_dtype_t dtype, void *out, float *final_state, void *workspace,
+                                  size_t workspace_bytes, cudaStream_t stream);
 
 /* Size of the fixed device scratch array behind gtr_gla_fwd_noalloc.  The
  * library holds one such array on every GPU where it is loaded, from the

@@ -216,6 +216,22 @@ size_t gtr_gla_workspace_bytes(int B, int H, int grid_h, int grid_w, int Dk, int
     return gtr::tc_supported(p) ? gtr::tc_workspace_bytes(p) : 0;
 }
 
+gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm, int *nseg,
+                                int *seg_len) {
+    if (!nseg || !seg_len || n_sm < 1) return GTR_ERR_INVALID_ARG;
+    const gtr_status_t st = check_shape(B, H, grid_h, grid_w, Dk, Dv, 0, GTR_F16);
+    if (st != GTR_OK) return st;
+    gtr::Problem p{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, B, H, grid_h, grid_w,
+                   Dk, Dv, 0, GTR_F16, (long long)grid_h * grid_w};
+    if (B == 0 || H == 0) {
+        *nseg = 1;
+        *seg_len = static_cast<int>((p.T + 63) / 64);
+        return GTR_OK;
+    }
+    gtr::tc_split_plan(p, n_sm, nseg, seg_len);
+    return GTR_OK;
+}
+
 gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const void *log_gate, int B,
                             int H, int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
                             gtr_dtype_t dtype, void *out, float *final_state, void *workspace,
@@ -231,10 +247,16 @@ gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const v
     return dispatch(p, GTR_SCHED_AUTO, workspace, workspace_bytes, true, stream);
 }
 
-gtr_status_t gtr_gla_fwd_gated(const void *q, const void *k, const void *v, const void *log_gate,
-                               const void *gate, const float *norm_weight, float eps, int B, int H,
-                               int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
-                               gtr_dtype_t dtype, void *out, float *final_state, cudaStream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// The mixer, then the gate over its output in place (the output is still in L2 for
+// workloads that fit there); `own_ws`: the caller's workspace, else the internal one.
+gtr_status_t gated(const void *q, const void *k, const void *v, const void *log_gate, const void *gate,
+                   const float *norm_weight, float eps, int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                   gtr_scan_t scan_order, gtr_dtype_t dtype, void *out, float *final_state, void *ws,
+                   size_t ws_bytes, bool own_ws, cudaStream_t stream) {
     gtr::Problem p;
     gtr_status_t st = make_problem(q, k, v, log_gate, B, H, grid_h, grid_w, Dk, Dv, scan_order,
                                    dtype, out, final_state, &p);
@@ -244,13 +266,36 @@ gtr_status_t gtr_gla_fwd_gated(const void *q, const void *k, const void *v, cons
     if (!gate || !norm_weight || !aligned(gate) || !aligned(norm_weight)) return GTR_ERR_INVALID_ARG;
     const size_t nv = (size_t)B * p.T * H * Dv * elem_size(dtype);
     if (overlaps(out, nv, gate, nv)) return GTR_ERR_INVALID_ARG;
-    // the mixer, then the gate over its output in place (the output is still in L2
-    // for workloads that fit there)
-    st = dispatch(p, GTR_SCHED_AUTO, nullptr, 0, false, stream);
+    if (own_ws) {
+        const size_t need = gtr_gla_workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype);
+        if (need > 0 && (ws == nullptr || ws_bytes < need)) return GTR_ERR_WORKSPACE;
+    }
+    st = dispatch(p, GTR_SCHED_AUTO, ws, ws_bytes, own_ws, stream);
     if (st != GTR_OK) return st;
     const cudaError_t e = gtr::launch_gate_epilogue(p, gtr::Gate{gate, norm_weight, eps}, stream);
     if (e != cudaSuccess) return cuda_fail(e);
     return GTR_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+gtr_status_t gtr_gla_fwd_gated(const void *q, const void *k, const void *v, const void *log_gate,
+                               const void *gate, const float *norm_weight, float eps, int B, int H,
+                               int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
+                               gtr_dtype_t dtype, void *out, float *final_state, cudaStream_t stream) {
+    return gated(q, k, v, log_gate, gate, norm_weight, eps, B, H, grid_h, grid_w, Dk, Dv, scan_order, dtype,
+                 out, final_state, nullptr, 0, false, stream);
+}
+
+gtr_status_t gtr_gla_fwd_gated_ws(const void *q, const void *k, const void *v, const void *log_gate,
+                                  const void *gate, const float *norm_weight, float eps, int B, int H,
+                                  int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
+                                  gtr_dtype_t dtype, void *out, float *final_state, void *workspace,
+                                  size_t workspace_bytes, cudaStream_t stream) {
+    return gated(q, k, v, log_gate, gate, norm_weight, eps, B, H, grid_h, grid_w, Dk, Dv, scan_order, dtype,
+                 out, final_state, workspace, workspace_bytes, true, stream);
 }
 
 gtr_status_t gtr_gla_fwd_noalloc(const void *q, const void *k, const void *v, const void *log_gate,

@@ -34,6 +34,9 @@ cudaError_t launch_gate_epilogue(const Problem &p, const Gate &gate, cudaStream_
 
 // Tensor-core chunkwise schedule (gla_tc.cu).
 bool tc_supported(const Problem &p);
+// Segments per sequence and chunks per segment the tensor-core schedule uses for
+// this problem on a device with n_sm SMs (host arithmetic only; nseg 1: unsplit).
+void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len);
 // Scratch the tensor-core schedule uses for this problem on the current device:
 // per-segment summaries when it splits sequences (few, long ones), else 0.
 size_t tc_workspace_bytes(const Problem &p);

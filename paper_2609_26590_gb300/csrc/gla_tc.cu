@@ -363,7 +363,8 @@ __device__ __noinline__ void exact_chunk(uint8_t *tq, uint8_t *tk, uint8_t *tgat
 // Operands of a tf32-mode chunk (split factors beyond the fp16 range): tf32 Q^ and
 // K^ for the score product in the group's operand buffer, fp16 Qtil = Q^ c1 over q and
 // Kbar = K^ c2 over k.  Re-reads the thread's 32 log-decays from TMEM (A is kept
-// until the operands are built).
+// until the operands are built): out of line, this rarer path leaves the fp16 path's
+// code and registers as they are (inlined it cost workload 2 6 %).
 template <typename E>
 __device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *opbuf, const float *ref,
                                            uint32_t taddr, int row, int ch0) {
@@ -379,12 +380,20 @@ __device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *op
         const uint4 qw = *reinterpret_cast<const uint4 *>(tq + o16);
         const uint4 kw = *reinterpret_cast<const uint4 *>(tk + o16);
         const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w}, ka[4] = {kw.x, kw.y, kw.z, kw.w};
+        // A_mid log2, c1 and c2 of the 8 channels (16-byte aligned rows of the references)
+        float am[8], c1v[8], c2v[8];
+        *reinterpret_cast<float4 *>(&am[0]) = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl);
+        *reinterpret_cast<float4 *>(&am[4]) = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl + 4);
+        *reinterpret_cast<float4 *>(&c1v[0]) = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl);
+        *reinterpret_cast<float4 *>(&c1v[4]) = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl + 4);
+        *reinterpret_cast<float4 *>(&c2v[0]) = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl);
+        *reinterpret_cast<float4 *>(&c2v[4]) = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl + 4);
         float qs[8], ks[8];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const float2 q2 = Elem<E>::unpack(qa[e]), k2 = Elem<E>::unpack(ka[e]);
-            const float e0 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e]), kLog2e, -ref[2 * kD + cl + 2 * e]);
-            const float e1 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e + 1]), kLog2e, -ref[2 * kD + cl + 2 * e + 1]);
+            const float e0 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e]), kLog2e, -am[2 * e]);
+            const float e1 = fmaf(__uint_as_float(ar[8 * g8 + 2 * e + 1]), kLog2e, -am[2 * e + 1]);
             qs[2 * e] = q2.x * ex2(e0);
             qs[2 * e + 1] = q2.y * ex2(e1);
             ks[2 * e] = k2.x * ex2(-e0);
@@ -401,8 +410,8 @@ __device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *op
         uint32_t qo[4], ko[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-            qo[e] = h2bits(qs[2 * e] * ref[3 * kD + cl + 2 * e], qs[2 * e + 1] * ref[3 * kD + cl + 2 * e + 1]);
-            ko[e] = h2bits(ks[2 * e] * ref[4 * kD + cl + 2 * e], ks[2 * e + 1] * ref[4 * kD + cl + 2 * e + 1]);
+            qo[e] = h2bits(qs[2 * e] * c1v[2 * e], qs[2 * e + 1] * c1v[2 * e + 1]);
+            ko[e] = h2bits(ks[2 * e] * c2v[2 * e], ks[2 * e + 1] * c2v[2 * e + 1]);
         }
         *reinterpret_cast<uint4 *>(tq + o16) = make_uint4(qo[0], qo[1], qo[2], qo[3]);
         *reinterpret_cast<uint4 *>(tk + o16) = make_uint4(ko[0], ko[1], ko[2], ko[3]);
@@ -1148,6 +1157,12 @@ size_t summary_bytes(const Problem &p, int nseg) {
 }
 
 }  // namespace
+
+void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len) {
+    const Split sp = choose_split(p, n_sm);
+    *nseg = sp.nseg;
+    *seg_len = sp.len;
+}
 
 size_t tc_workspace_bytes(const Problem &p) {
     int n_sm = 0;

@@ -55,10 +55,14 @@ def load(path: Optional[str] = None):
         lib.gtr_gla_tc_supported.argtypes = [ci] * 8
         lib.gtr_gla_workspace_bytes.restype = st
         lib.gtr_gla_workspace_bytes.argtypes = [ci] * 7
+        lib.gtr_gla_split_plan.restype = ci
+        lib.gtr_gla_split_plan.argtypes = [ci] * 7 + [ctypes.POINTER(ci)] * 2
         lib.gtr_gla_fwd_ws.restype = ci
         lib.gtr_gla_fwd_ws.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp, st, vp]
         lib.gtr_gla_fwd_gated.restype = ci
         lib.gtr_gla_fwd_gated.argtypes = [vp] * 6 + [ctypes.c_float] + [ci] * 8 + [vp, vp, vp]
+        lib.gtr_gla_fwd_gated_ws.restype = ci
+        lib.gtr_gla_fwd_gated_ws.argtypes = [vp] * 6 + [ctypes.c_float] + [ci] * 8 + [vp, vp, vp, st, vp]
         lib.gtr_gla_fwd_noalloc.restype = ci
         lib.gtr_gla_fwd_noalloc.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp]
         lib.gtr_gla_host_buffer_bytes.restype = st
@@ -144,6 +148,17 @@ def workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype: torch.dtype) -> int:
     return int(load().gtr_gla_workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, _DTYPES[dtype]))
 
 
+def split_plan(B: int, H: int, grid_h: int, grid_w: int, Dk: int, Dv: int, n_sm: int) -> Tuple[int, int]:
+    """(segments per sequence, chunks per segment) of the tensor-core schedule on a
+    device with ``n_sm`` SMs, through ``gtr_gla_split_plan`` (host arithmetic only)."""
+    lib = load()
+    nseg, seg_len = ctypes.c_int(0), ctypes.c_int(0)
+    status = lib.gtr_gla_split_plan(B, H, grid_h, grid_w, Dk, Dv, n_sm, ctypes.byref(nseg),
+                                    ctypes.byref(seg_len))
+    _check(status, "gtr_gla_split_plan", lib)
+    return nseg.value, seg_len.value
+
+
 def forward_ws(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,
                grid_h: int, grid_w: int, order: int, out: torch.Tensor,
                final_state: Optional[torch.Tensor], workspace: Optional[torch.Tensor],
@@ -165,10 +180,13 @@ def forward_ws(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torc
 def forward_gated(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,
                   gate: torch.Tensor, norm_weight: torch.Tensor, eps: float, grid_h: int, grid_w: int,
                   order: int = ROW_FWD, out: Optional[torch.Tensor] = None, final_state=True,
-                  stream: Optional[torch.cuda.Stream] = None) -> Tuple[torch.Tensor, Optional[torch.Tensor]]:
+                  stream: Optional[torch.cuda.Stream] = None,
+                  workspace: Optional[torch.Tensor] = None) -> Tuple[torch.Tensor, Optional[torch.Tensor]]:
     """Mixer plus output gate through ``gtr_gla_fwd_gated``: returns
     (u = SiLU(gate) * RMSNorm(o) per head, final_state).  gate: like v;
-    norm_weight: Dv float32 values on the device."""
+    norm_weight: Dv float32 values on the device.  With ``workspace`` (a CUDA
+    uint8 tensor of at least workspace_bytes()) the call goes through
+    ``gtr_gla_fwd_gated_ws``: no allocation, safe to capture into a CUDA graph."""
     lib = load()
     B, H, Dk, Dv = _dims(q, v, grid_h, grid_w)
     if out is None:
@@ -178,11 +196,16 @@ def forward_gated(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: t
         fs = torch.empty((B, H, Dk, Dv), dtype=torch.float32, device=q.device)
     elif isinstance(final_state, torch.Tensor):
         fs = final_state
-    status = lib.gtr_gla_fwd_gated(
-        q.data_ptr(), k.data_ptr(), v.data_ptr(), log_gate.data_ptr(), gate.data_ptr(),
-        norm_weight.data_ptr(), float(eps), B, H, grid_h, grid_w, Dk, Dv, order, _DTYPES[q.dtype],
-        out.data_ptr(), fs.data_ptr() if fs is not None else None, _stream_ptr(stream))
-    _check(status, "gtr_gla_fwd_gated", lib)
+    args = (q.data_ptr(), k.data_ptr(), v.data_ptr(), log_gate.data_ptr(), gate.data_ptr(),
+            norm_weight.data_ptr(), float(eps), B, H, grid_h, grid_w, Dk, Dv, order, _DTYPES[q.dtype],
+            out.data_ptr(), fs.data_ptr() if fs is not None else None)
+    if workspace is None:
+        status = lib.gtr_gla_fwd_gated(*args, _stream_ptr(stream))
+        _check(status, "gtr_gla_fwd_gated", lib)
+    else:
+        status = lib.gtr_gla_fwd_gated_ws(*args, workspace.data_ptr(),
+                                          workspace.numel() * workspace.element_size(), _stream_ptr(stream))
+        _check(status, "gtr_gla_fwd_gated_ws", lib)
     return out, fs
 
 

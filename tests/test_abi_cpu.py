@@ -132,3 +132,20 @@ def test_gated_entry_point_validates_before_any_launch(lib):
     assert call(gate=(1 << 26) + 64) == 1         # overlaps the output
     # an empty batch launches nothing
     assert fwd(None, None, None, None, None, None, 1e-6, 0, 2, 8, 8, 64, 64, 0, 1, None, None, None) == 0
+
+
+def test_gated_ws_entry_point_validates_before_any_launch(lib):
+    fwd = lib.gtr_gla_fwd_gated_ws
+    ok = dict(q=16, k=16, v=16, g=16, gate=1 << 24, w=1 << 25, eps=1e-6)
+
+    def call(**kw):
+        a = dict(ok, **kw)
+        return fwd(a["q"], a["k"], a["v"], a["g"], a["gate"], a["w"], a["eps"], 1, 1, 8, 8, 64, 64,
+                   0, 1, 1 << 26, None, None, 0, None)
+    assert call(gate=None) == 1
+    assert call(w=None) == 1
+    assert call(gate=(1 << 24) + 8) == 1          # not 16-byte aligned
+    assert call(eps=-1.0) == 1
+    assert call(gate=(1 << 26) + 64) == 1         # overlaps the output
+    assert fwd(None, None, None, None, None, None, 1e-6, 0, 2, 8, 8, 64, 64, 0, 1, None, None, None, 0,
+               None) == 0

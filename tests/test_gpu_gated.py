@@ -91,3 +91,42 @@ def test_gated_matches_forward_then_gate():
     ref = oracle.gated_output(o.float().cpu().numpy(), wl.storage_to_f64(r, dtype), w, 1e-6)
     e = errors(u.float().cpu().numpy().astype(np.float64), ref)
     assert e["finite"] and e["rel_l2"] <= 4e-3 and e["max_abs"] <= 4e-2 * e["max_ref"], e
+
+
+def test_gated_ws_matches_and_captures_split():
+    """gtr_gla_fwd_gated_ws: the caller's workspace gives the same split schedule as the
+    internal one (identical bits), a short workspace is refused before any launch, and
+    the call captured into a CUDA graph keeps the split and reproduces the bits."""
+    B, H, gh, gw, D, dtype = 1, 6, 40, 40, 64, "f16"      # 25 chunks per sequence: split
+    T = gh * gw
+    need = gla.workspace_bytes(B, H, gh, gw, D, D, TORCH_DT[dtype])
+    assert need > 0, "this shape should split its sequences"
+    inp = wl.make_inputs(B, H, gh, gw, D, D, dtype, seed=9701)
+    r, w = _gate_inputs(B, H, T, D, dtype, seed=9702)
+    t = {n: to_torch(inp[n], dtype) for n in ("q", "k", "v", "g")}
+    tr, tw = to_torch(r, dtype), torch.from_numpy(w).cuda()
+    ref, ref_fs = gla.forward_gated(t["q"], t["k"], t["v"], t["g"], tr, tw, 1e-5, gh, gw, wl.COL_REV)
+    ws = torch.empty(need, dtype=torch.uint8, device="cuda")
+    out, fs = gla.forward_gated(t["q"], t["k"], t["v"], t["g"], tr, tw, 1e-5, gh, gw, wl.COL_REV,
+                                workspace=ws)
+    torch.cuda.synchronize()
+    assert gla.sync_status() == 0
+    assert torch.equal(out, ref) and torch.equal(fs, ref_fs)
+    with pytest.raises(gla.GLAError) as ei:
+        gla.forward_gated(t["q"], t["k"], t["v"], t["g"], tr, tw, 1e-5, gh, gw, wl.COL_REV,
+                          workspace=ws[: need - 256])
+    assert ei.value.status == 3                             # GTR_ERR_WORKSPACE
+    out2 = torch.full_like(out, float("nan"))
+    fs2 = torch.full_like(fs, float("nan"))
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            gla.forward_gated(t["q"], t["k"], t["v"], t["g"], tr, tw, 1e-5, gh, gw, wl.COL_REV, out=out2,
+                              final_state=fs2, stream=s, workspace=ws)
+    torch.cuda.current_stream().wait_stream(s)
+    g.replay()
+    torch.cuda.synchronize()
+    assert gla.sync_status() == 0
+    assert torch.equal(out2, ref) and torch.equal(fs2, ref_fs)

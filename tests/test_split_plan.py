@@ -1,0 +1,93 @@
+"""The sequence split of the tensor-core schedule (Eq. chunk_boundary_main applied
+across segments), through gtr_gla_split_plan: host arithmetic, so it runs
+without a GPU.  The plans below are the segment lengths a GB300 sweep measured
+fastest (graph-replayed calls, interleaved rounds); the invariants hold for any
+shape: the last segment is not empty, a split fits one wave of the SMs, and
+sequences that already fill half the SMs are never split."""
+import math
+
+import numpy as np
+import pytest
+
+from paper_2609_26590_gb300 import build as gbuild
+
+GB300_SMS = 152
+
+
+@pytest.fixture(scope="module")
+def gla():
+    gbuild.build()
+    from paper_2609_26590_gb300 import gla as g
+    g.load()
+    return g
+
+
+# (B, H, grid_h, grid_w, Dk, Dv) -> (segments, chunks per segment) on 152 SMs
+MEASURED = [
+    ((1, 6, 40, 40, 64, 64), (13, 2)),      # 25 chunks: length 2 measured fastest (19.9 us vs 21.2 at 4)
+    ((1, 2, 128, 128, 64, 64), (32, 8)),    # 256 chunks over 2 sequences: length 8 (43.7 us vs 51.5 at 4)
+    ((1, 1, 128, 128, 128, 128), (32, 8)),  # two key halves, two value slices: 2 units, length 8
+    ((1, 4, 80, 80, 32, 64), (20, 5)),      # 100 chunks: between the measured best lengths 4 and 6
+    ((1, 6, 44, 44, 64, 64), (11, 3)),      # 31 chunks (prime): 2 padding chunks in the last segment
+    ((2, 8, 128, 128, 128, 128), (4, 64)),  # 32 units: at most 4 segments fit one wave
+    ((1, 1, 16, 20, 64, 64), (1, 5)),       # 5 chunks: unsplit (13.7 us against 21.2 split)
+    ((32, 12, 40, 40, 64, 64), (1, 25)),    # 384 units fill the device: unsplit
+    ((8, 16, 80, 80, 64, 64), (1, 100)),    # 128 units > half the SMs: unsplit
+]
+
+
+@pytest.mark.parametrize("shape,plan", MEASURED, ids=[f"{s[0]}x{s[1]}-{s[2]}x{s[3]}-d{s[4]}_{s[5]}"
+                                                      for s, _ in MEASURED])
+def test_plan_matches_measured_choice(gla, shape, plan):
+    assert gla.split_plan(*shape, GB300_SMS) == plan
+
+
+def test_plan_invariants_random_shapes(gla):
+    rng = np.random.Generator(np.random.PCG64(2609))
+    for _ in range(400):
+        B, H = int(rng.integers(1, 5)), int(rng.integers(1, 13))
+        gh, gw = int(rng.integers(1, 140)), int(rng.integers(1, 140))
+        Dk, Dv = 8 * int(rng.integers(1, 17)), 8 * int(rng.integers(1, 17))
+        n_sm = int(rng.choice([8, 32, 132, 148, 152]))
+        nseg, L = gla.split_plan(B, H, gh, gw, Dk, Dv, n_sm)
+        N = math.ceil(gh * gw / 64)
+        units = B * H * math.ceil(Dv / 64)
+        if nseg == 1:
+            assert L == N
+            continue
+        assert 2 <= L < N
+        assert nseg == math.ceil(N / L)
+        assert (nseg - 1) * L < N <= nseg * L          # the last segment holds a real chunk
+        assert units * nseg <= n_sm                     # one wave
+        assert 2 * units <= n_sm                        # only launches that leave SMs idle split
+        # cheaper than unsplit under the plan's own cost model
+        assert 9 * L + 2 * nseg + 10 < 6 * N
+
+
+def test_plan_is_optimal_under_its_cost_model(gla):
+    # brute force over every admissible length on small problems
+    for N in range(1, 80):
+        for units in (1, 2, 3, 6, 19, 40, 76, 77):
+            H, gh, gw = units, N, 64          # grid_w = 64: exactly N chunks per sequence
+            nseg, L = gla.split_plan(1, H, gh, gw, 64, 64, GB300_SMS)
+            cost = {1: 6 * N}
+            if 2 * units <= GB300_SMS:
+                for l in range(2, N):
+                    d = math.ceil(N / l)
+                    if units * d <= GB300_SMS:
+                        cost[l] = 9 * l + 2 * d + 10
+            best = min(cost.values())
+            got = 6 * N if nseg == 1 else 9 * L + 2 * nseg + 10
+            assert got == best, (N, units, nseg, L)
+
+
+def test_plan_rejects_invalid_arguments(gla):
+    import ctypes
+    lib = gla.load()
+    a, b = ctypes.c_int(-7), ctypes.c_int(-7)
+    assert lib.gtr_gla_split_plan(1, 1, 8, 8, 64, 64, 0, ctypes.byref(a), ctypes.byref(b)) == 1
+    assert lib.gtr_gla_split_plan(1, 1, 0, 8, 64, 64, 152, ctypes.byref(a), ctypes.byref(b)) == 1
+    assert lib.gtr_gla_split_plan(1, 1, 8, 8, 64, 300, 152, ctypes.byref(a), ctypes.byref(b)) == 1
+    assert lib.gtr_gla_split_plan(1, 1, 8, 8, 64, 64, 152, None, ctypes.byref(b)) == 1
+    assert a.value == -7 and b.value == -7
+    assert gla.split_plan(0, 3, 8, 8, 64, 64, 152) == (1, 1)
