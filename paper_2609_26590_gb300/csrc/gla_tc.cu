@@ -418,7 +418,7 @@ __device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *op
     }
 }
 
-template <typename E, int NH, int NV, int MODE>
+template <typename E, int NH, int NV, int MODE, bool GENOUT>
 __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_constant__ TcParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -435,6 +435,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     // the end state from zero and the total decay (k, v and gates; no scores or outputs).
     constexpr bool kSum = MODE == kSummary;
     constexpr bool kSplit = MODE != kFull;
+    // GENOUT (one key half, outputs): the gen warpgroup that built a chunk also reads its
+    // outputs back from TMEM and stores them, while it waits for the P of its next chunk,
+    // which takes that work off the epi's serial per-chunk chain.  The host selects it where
+    // that was measured faster (fp16 launches of at most one wave); elsewhere the epi stores.
+    constexpr bool kGenOut = GENOUT && NH == 1 && !kSum;
     const int N = p.n_chunks;   // chunks per sequence
     const int L = p.seg_len;    // chunks per unit
     constexpr int nh = NH;   // 64-channel key halves per chunk (Dk / 64)
@@ -645,6 +650,31 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         uint32_t vbits = 0u;  // bit s: score column ch0 + s is kept
         for (int s = 0; s < 32; ++s)
             if (rev ? (ch0 + s >= row) : (ch0 + s <= row)) vbits |= 1u << s;
+        // outputs of chunk co (this group's) once O(co) completed: TMEM -> this thread's row at its
+        // token's spatial position; false when the wait gave up
+        auto gen_out = [&](int co) -> bool {
+            if (!mbar_wait(&bars[BAR_OFULL + (co & 1)], (co >> 1) & 1, abort_flag, kWaitLimitNs)) return false;
+            tc_fence_after();
+            uint32_t r[32];
+            tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + (co & 1) * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+            tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + (co & 1) * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+            tmem_ld_wait();
+            uint32_t ow[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) ow[j] = Elem<E>::pack(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+            const StreamPos po = stream_pos(co, L, nh, lognv, kSplit ? p.nsu : 1);
+            const int b = po.bh / p.H, h = po.bh % p.H;
+            const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
+            if (t >= 0) {  // the row's columns inside Dv (padded columns stay behind)
+                const int col0 = 64 * po.vb + ch0;
+                uint4 *dst = reinterpret_cast<uint4 *>(static_cast<E *>(p.out) + (((size_t)b * p.T + t) * p.H + h) * p.Dv + col0);
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    if (col0 + 8 * q < p.Dv) dst[q] = make_uint4(ow[4 * q], ow[4 * q + 1], ow[4 * q + 2], ow[4 * q + 3]);
+            }
+            return true;
+        };
+        int last_c = -1;  // the group's last chunk completed (its outputs are stored after the loop)
         for (int c = gw; c < G; c += 2) {
             const int sl = c % kSlots, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
@@ -763,8 +793,14 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // operands in smem, A(c) read
             if (kSum) continue;  // no scores
+            // ---- outputs of the group's previous chunk c-2 (O(c) reuses its TMEM buffer only
+            // after ORDY(c), which this group signals below)
+            bool ofail = false;
+            if constexpr (kGenOut) {
+                if (c >= 2) ofail = !gen_out(c - 2);
+            }
             // ---- masked scores of chunk c over its gate tile (consumed by A(c) long ago)
-            const bool pfail = !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
+            const bool pfail = ofail || !mbar_wait(&bars[BAR_PFULL + bb], ph, abort_flag, kWaitLimitNs);
             if (named_barrier_or(bar_id, 128, pfail)) {
                 record_timeout(abort_flag);
                 break;
@@ -787,6 +823,10 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // this warp's rows of P are in smem
+            last_c = c;
+        }
+        if constexpr (kGenOut) {
+            if (last_c >= 0 && last_c + 2 >= G && !gen_out(last_c)) record_timeout(abort_flag);
         }
     } else {
         // ======================================================= epi warpgroup (warps 10-13)
@@ -854,9 +894,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     dp = dpo = 1.f;
                 }
                 bool fail = !mbar_wait(&bars[BAR_REFS + sl], (c / kSlots) & 1, abort_flag, kWaitLimitNs);
-                // buffer bb was last read by O(c-2) (one key half: observed by the readout of
-                // the previous iteration already)
-                if (!kSum && NH == 2 && c >= 2)
+                // buffer bb was last read by O(c-2) (epi outputs with one key half: observed by
+                // the readout of the previous iteration already)
+                if (!kSum && (NH == 2 || kGenOut) && c >= 2)
                     fail = fail || !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs);
                 if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
                     ok = false;
@@ -935,7 +975,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     dpo = t;
                 }
             }
-            if (!kSum && c >= nh && c % nh == 0) {
+            if (!kSum && !kGenOut && c >= nh && c % nh == 0) {
                 // outputs of the real chunk whose last key half is c-1
                 const int co = c - 1, ob = (co / nh) & 1;
                 const bool fail = !mbar_wait(&bars[BAR_OFULL + (co & 1)], (co >> 1) & 1, abort_flag, kWaitLimitNs);
@@ -1069,7 +1109,7 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     return true;
 }
 
-template <typename E, int NH, int NV, int MODE>
+template <typename E, int NH, int NV, int MODE, bool GENOUT = false>
 cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
     // the shared-memory opt-in, once per process and device (setting it again is harmless)
     static std::atomic<unsigned long long> set_on_devices(0);
@@ -1078,17 +1118,23 @@ cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     const unsigned long long bit = 1ull << (dev & 63);
     if (!(set_on_devices.load(std::memory_order_relaxed) & bit)) {
-        e = cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        e = cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV, MODE, GENOUT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
         if (e != cudaSuccess) return e;
         set_on_devices.fetch_or(bit);
     }
-    gla_tc_kernel<E, NH, NV, MODE><<<grid, kThreads, kSmemBytes, stream>>>(tp);
+    gla_tc_kernel<E, NH, NV, MODE, GENOUT><<<grid, kThreads, kSmemBytes, stream>>>(tp);
     return cudaSuccess;
 }
 
 // One instantiation per (element type, key halves, value slices, pass).
+// gen_out: outputs stored by the gen warpgroups (fp16, one key half, outputs only)
 template <typename E, int MODE>
-cudaError_t launch_shape(dim3 grid, const TcParams &tp, cudaStream_t stream) {
+cudaError_t launch_shape(dim3 grid, const TcParams &tp, cudaStream_t stream, bool gen_out = false) {
+    if constexpr (std::is_same<E, __half>::value && MODE != kSummary) {
+        if (gen_out && tp.nh == 1)
+            return tp.nv == 1 ? launch_kernel<E, 1, 1, MODE, true>(grid, tp, stream)
+                              : launch_kernel<E, 1, 2, MODE, true>(grid, tp, stream);
+    }
     if (tp.nh == 1)
         return tp.nv == 1 ? launch_kernel<E, 1, 1, MODE>(grid, tp, stream) : launch_kernel<E, 1, 2, MODE>(grid, tp, stream);
     return tp.nv == 1 ? launch_kernel<E, 2, 1, MODE>(grid, tp, stream) : launch_kernel<E, 2, 2, MODE>(grid, tp, stream);
@@ -1220,11 +1266,15 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     tp.nsu = nseg;
     tp.n_units = seqs * nseg;
     const dim3 grid(static_cast<unsigned>(tp.n_units < n_sm ? tp.n_units : n_sm));
+    // outputs from the gen warpgroups: fp16 launches of at most one wave (measured on a GB300:
+    // +3 to +6 % there; with several units per CTA, or bf16, the epi storing them was faster)
+    const bool gen_out = half && tp.n_units <= n_sm;
     if (nseg > 1)
-        e = half ? launch_shape<__half, kSplitFull>(grid, tp, stream)
+        e = half ? launch_shape<__half, kSplitFull>(grid, tp, stream, gen_out)
                  : launch_shape<__nv_bfloat16, kSplitFull>(grid, tp, stream);
     else
-        e = half ? launch_shape<__half, kFull>(grid, tp, stream) : launch_shape<__nv_bfloat16, kFull>(grid, tp, stream);
+        e = half ? launch_shape<__half, kFull>(grid, tp, stream, gen_out)
+                 : launch_shape<__nv_bfloat16, kFull>(grid, tp, stream);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
