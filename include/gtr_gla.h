@@ -133,6 +133,18 @@ size_t gtr_gla_workspace_bytes(int B, int H, int grid_h, int grid_w, int Dk, int
 gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm,
                                 int *nseg, int *seg_len);
 
+/* Introspection of the scan-order gather (Sec. 3.1, directional scanning): the
+ * TMA boxes the tensor-core schedule loads for 64-token chunk c of a sequence
+ * on a grid_h x grid_w patch grid, computed on the host by the same code the
+ * kernel's producer runs.  Writes min(count, cap) boxes of 4 ints to `boxes`:
+ * rows (1-64), first row of the chunk's 64-row shared-memory tile, and the two
+ * token coordinates of the box's first row (row orders: token index, 0; column
+ * orders: column x, row y; x == grid_w marks a box that lies wholly outside the
+ * tensor and loads zeros).  Chunks at or past the sequence's end are the
+ * all-zero padding chunks of a split's last segment.  Returns the chunk's box
+ * count, or -1 for invalid arguments.  No device is used. */
+int gtr_gla_chunk_boxes(int grid_h, int grid_w, gtr_scan_t scan_order, int c, int *boxes, int cap);
+
 /* gtr_gla_fwd with a caller-owned device workspace of workspace_bytes >=
  * gtr_gla_workspace_bytes() bytes, 256-byte aligned (may be NULL when that is
  * 0).  The call allocates nothing and does not synchronise.  Returns

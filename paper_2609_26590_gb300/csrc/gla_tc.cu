@@ -210,7 +210,7 @@ __device__ __forceinline__ void record_timeout(volatile uint32_t *abort_flag) {
 // Smem row rho of chunk c holds walk position w0 + rho, where the walk is the
 // forward scan (row-major for row orders, down the columns for column orders)
 // and w0 mirrors the range for reverse orders (scan position 64c + 63 - rho).
-__device__ __forceinline__ int chunk_w0(int order, int T, int c) {
+__host__ __device__ __forceinline__ int chunk_w0(int order, int T, int c) {
     return (order & 1) ? (T - kC * (c + 1)) : kC * c;
 }
 
@@ -251,7 +251,7 @@ __device__ __forceinline__ StreamPos stream_pos(int v, int L, int nh, int lognv,
 // segments), each loaded as at most two boxes: its multiple of 8 and the remainder.
 // One call site for f keeps the producer's issue code small.
 template <typename F>
-__device__ __forceinline__ void chunk_load_boxes(int order, int T, int grid_h, int grid_w, int c, F &&f) {
+__host__ __device__ __forceinline__ void chunk_load_boxes(int order, int T, int grid_h, int grid_w, int c, F &&f) {
     const int w0 = chunk_w0(order, T, c);
     if ((order >> 1) == 0) {
         f(kHeights - 1, 0, w0, 0);
@@ -1203,6 +1203,20 @@ size_t summary_bytes(const Problem &p, int nseg) {
 }
 
 }  // namespace
+
+int tc_chunk_boxes(int order, int T, int grid_h, int grid_w, int c, int *boxes, int cap) {
+    int n = 0;
+    chunk_load_boxes(order, T, grid_h, grid_w, c, [&](int hi, int row, int c2, int c3) {
+        if (n < cap) {
+            boxes[4 * n + 0] = box_height(hi);
+            boxes[4 * n + 1] = row;
+            boxes[4 * n + 2] = c2;
+            boxes[4 * n + 3] = c3;
+        }
+        ++n;
+    });
+    return n;
+}
 
 void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len) {
     const Split sp = choose_split(p, n_sm);

@@ -55,6 +55,8 @@ def load(path: Optional[str] = None):
         lib.gtr_gla_tc_supported.argtypes = [ci] * 8
         lib.gtr_gla_workspace_bytes.restype = st
         lib.gtr_gla_workspace_bytes.argtypes = [ci] * 7
+        lib.gtr_gla_chunk_boxes.restype = ci
+        lib.gtr_gla_chunk_boxes.argtypes = [ci] * 4 + [ctypes.POINTER(ci), ci]
         lib.gtr_gla_split_plan.restype = ci
         lib.gtr_gla_split_plan.argtypes = [ci] * 7 + [ctypes.POINTER(ci)] * 2
         lib.gtr_gla_fwd_ws.restype = ci
@@ -157,6 +159,18 @@ def split_plan(B: int, H: int, grid_h: int, grid_w: int, Dk: int, Dv: int, n_sm:
                                     ctypes.byref(seg_len))
     _check(status, "gtr_gla_split_plan", lib)
     return nseg.value, seg_len.value
+
+
+def chunk_boxes(grid_h: int, grid_w: int, order: int, c: int):
+    """The TMA boxes (rows, tile row, coordinate 2, coordinate 3) the tensor-core
+    producer loads for chunk c, through ``gtr_gla_chunk_boxes`` (host only)."""
+    lib = load()
+    cap = 80  # a chunk has at most 64 column segments plus 4 zero-fill boxes
+    buf = (ctypes.c_int * (4 * cap))()
+    n = lib.gtr_gla_chunk_boxes(grid_h, grid_w, order, c, buf, cap)
+    if n < 0 or n > cap:
+        raise ValueError(f"gtr_gla_chunk_boxes returned {n}")
+    return [tuple(buf[4 * i:4 * i + 4]) for i in range(n)]
 
 
 def forward_ws(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,

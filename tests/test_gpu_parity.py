@@ -313,3 +313,17 @@ def test_explicit_schedule_rejects_unsupported():
     with pytest.raises(gla.GLAError) as ei:
         gla.forward(t["q"], t["k"], t["v"], t["g"], 4, 4, 0, schedule="tc")
     assert ei.value.status == 2
+
+
+def test_workspace_matches_split_plan():
+    """The summaries the schedule allocates are those of the split gtr_gla_split_plan
+    reports for this device's SM count: (segments - 1) per sequence of padded
+    (Dk x Dv + Dk) floats."""
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    pad = lambda d: (d + 63) // 64 * 64
+    for B, H, gh, gw, Dk, Dv in [(1, 6, 40, 40, 64, 64), (1, 6, 44, 44, 64, 64), (2, 8, 128, 128, 128, 128),
+                                 (32, 12, 40, 40, 64, 64), (1, 3, 40, 36, 32, 64), (1, 1, 16, 20, 64, 64)]:
+        nseg, seg_len = gla.split_plan(B, H, gh, gw, Dk, Dv, n_sm)
+        expect = 0 if nseg == 1 else B * H * (nseg - 1) * (pad(Dk) * pad(Dv) + pad(Dk)) * 4
+        for dt in (torch.float16, torch.bfloat16):
+            assert gla.workspace_bytes(B, H, gh, gw, Dk, Dv, dt) == expect, (B, H, gh, gw, Dk, Dv, nseg, seg_len)
