@@ -20,6 +20,9 @@ Prediction"):
 * :func:`gated_output` -- Sec. 3.1, the output gate applied to the mixer's
   output: ``u_t = SiLU(r_t) * RMSNorm(o_t)`` (the epilogue the paper's deployed
   kernel fuses, App. C.3).
+* :func:`sswiglu_dwconv` -- Sec. 3.1, "Spatial SwiGLU", Eq. (spatial_swiglu):
+  the part between its two projections, ``SiLU(X W_g) * DWConv3x3(X W_v)``
+  on the patch grid (the part the deployed S-SwiGLU kernel fuses, Sec. 4).
 
 Pins: tests/test_oracle_pins.py checks the functions against hand-worked
 example (tests/golden/), brute-force quadratic forms, closed forms (gate 1 =
@@ -214,3 +217,38 @@ def gated_output(o, r_pre, weight, eps: float) -> np.ndarray:
     with np.errstate(over="ignore"):
         silu = r / (1.0 + np.exp(-r))   # r * sigmoid(r); exp overflow gives -0 for r << 0
     return silu * (o / rms) * w
+
+
+def sswiglu_dwconv(gate_pre, value_pre, weight, bias, grid_h: int, grid_w: int) -> np.ndarray:
+    """Sec. 3.1, Eq. (spatial_swiglu), between the projections:
+    ``Z = SiLU(X W_g) * DWConv3x3(X W_v)``.
+
+    gate_pre = X W_g and value_pre = X W_v: [B, T, F] with T = grid_h * grid_w
+    tokens in spatial row-major order.  The value branch is read as the
+    grid_h x grid_w image of F channels and convolved per channel with its own
+    3 x 3 kernel: ``weight[f, i, j]`` multiplies the value at row offset i - 1
+    and column offset j - 1 (a cross-correlation, as a depthwise 2-D
+    convolution layer computes it), with zeros outside the grid, plus
+    ``bias[f]`` (None: no bias).  Plain fp64 numpy: nine shifted, weighted
+    copies of the zero-padded image summed, then the SiLU gate.
+    """
+    g = np.asarray(gate_pre, dtype=np.float64)
+    v = np.asarray(value_pre, dtype=np.float64)
+    w = np.asarray(weight, dtype=np.float64)
+    if g.shape != v.shape or g.ndim != 3 or g.shape[1] != grid_h * grid_w:
+        raise ValueError("gate_pre and value_pre must be [B, grid_h*grid_w, F]")
+    B, T, F = v.shape
+    if w.shape != (F, 3, 3):
+        raise ValueError("weight must be [F, 3, 3]")
+    img = v.reshape(B, grid_h, grid_w, F)
+    pad = np.zeros((B, grid_h + 2, grid_w + 2, F))
+    pad[:, 1:grid_h + 1, 1:grid_w + 1, :] = img
+    conv = np.zeros((B, grid_h, grid_w, F))
+    for i in range(3):
+        for j in range(3):
+            conv += w[:, i, j] * pad[:, i:i + grid_h, j:j + grid_w, :]
+    if bias is not None:
+        conv += np.asarray(bias, dtype=np.float64)
+    with np.errstate(over="ignore"):
+        silu = g / (1.0 + np.exp(-g))
+    return silu * conv.reshape(B, T, F)

@@ -300,3 +300,76 @@ def test_gated_output_invariants():
     np.testing.assert_array_equal(oracle.gated_output(o, np.zeros_like(r), w, eps), 0.0 * u)
     big = np.full_like(r, 40.0)
     np.testing.assert_allclose(oracle.gated_output(o, big, w, eps), 40.0 * o / rms * w, rtol=1e-15)
+
+
+# ---------------------------------------------------------------- Spatial SwiGLU (Eq. spatial_swiglu)
+
+def _golden_sswiglu():
+    with open(os.path.join(GOLDEN, "sswiglu_dwconv_2x3.json")) as f:
+        return json.load(f)
+
+
+def test_sswiglu_hand_worked_2x3():
+    d = _golden_sswiglu()
+    gh, gw = d["grid_h"], d["grid_w"]
+    v = np.array(d["value_image"], dtype=np.float64).reshape(1, gh * gw, 1)
+    gate = []
+    for e in d["gate"]:
+        gate.append(0.0 if e[0] == "zero" else e[2] * np.log(e[1]))
+    g = np.array(gate).reshape(1, gh * gw, 1)
+    w = np.array(d["weight"], dtype=np.float64).reshape(1, 3, 3)
+    z = oracle.sswiglu_dwconv(g, v, w, np.array([d["bias"]]), gh, gw).ravel()
+    expect = np.array([c * np.log(base) for c, base in d["z_as_coefficient_of_log"]])
+    np.testing.assert_allclose(z, expect, rtol=1e-14, atol=1e-14)
+    # the convolution alone: gate so large that SiLU(g) = g to double precision, then divide
+    big = np.full_like(g, 1e3)
+    conv = oracle.sswiglu_dwconv(big, v, w, np.array([d["bias"]]), gh, gw).ravel() / 1e3
+    np.testing.assert_allclose(conv, d["conv"], rtol=1e-14)
+
+
+def test_sswiglu_matches_scipy_correlate2d():
+    scipy_signal = pytest.importorskip("scipy.signal")
+    rng = np.random.Generator(np.random.PCG64(42))
+    B, gh, gw, F = 2, 7, 4, 5
+    g = rng.standard_normal((B, gh * gw, F))
+    v = rng.standard_normal((B, gh * gw, F))
+    w = rng.standard_normal((F, 3, 3))
+    bias = rng.standard_normal(F)
+    z = oracle.sswiglu_dwconv(g, v, w, bias, gh, gw)
+    for b in range(B):
+        for f in range(F):
+            img = v[b, :, f].reshape(gh, gw)
+            conv = scipy_signal.correlate2d(img, w[f], mode="same", boundary="fill", fillvalue=0.0)
+            silu = g[b, :, f] * scipy_expit(g[b, :, f])
+            np.testing.assert_allclose(z[b, :, f], silu * (conv.ravel() + bias[f]), rtol=1e-12, atol=1e-12)
+
+
+def scipy_expit(x):
+    special = pytest.importorskip("scipy.special")
+    return special.expit(x)
+
+
+def test_sswiglu_special_cases():
+    rng = np.random.Generator(np.random.PCG64(7))
+    B, gh, gw, F = 1, 5, 6, 3
+    g = rng.standard_normal((B, gh * gw, F))
+    v = rng.standard_normal((B, gh * gw, F))
+    ident = np.zeros((F, 3, 3))
+    ident[:, 1, 1] = 1.0
+    silu = g * scipy_expit(g)
+    # identity kernel, no bias: the tokenwise SwiGLU product
+    np.testing.assert_allclose(oracle.sswiglu_dwconv(g, v, ident, None, gh, gw), silu * v, rtol=1e-14)
+    # zero kernel: only the bias survives, gated
+    bias = np.array([0.5, -2.0, 3.0])
+    np.testing.assert_allclose(oracle.sswiglu_dwconv(g, v, np.zeros((F, 3, 3)), bias, gh, gw), silu * bias,
+                               rtol=1e-14)
+    # all-ones kernel on a constant image: 9c inside, 6c on edges, 4c at corners
+    ones = np.ones((F, 3, 3))
+    big = np.full((B, gh * gw, F), 1e3)
+    conv = oracle.sswiglu_dwconv(big, np.full((B, gh * gw, F), 2.0), ones, None, gh, gw)[0, :, 0] / 1e3
+    img = conv.reshape(gh, gw)
+    assert img[2, 2] == 18.0 and img[0, 3] == 12.0 and img[0, 0] == 8.0 and img[gh - 1, gw - 1] == 8.0
+    # a 1 x 1 grid sees only the centre tap
+    w = rng.standard_normal((F, 3, 3))
+    np.testing.assert_allclose(oracle.sswiglu_dwconv(g[:, :1], v[:, :1], w, None, 1, 1),
+                               silu[:, :1] * v[:, :1] * w[:, 1, 1], rtol=1e-14)
