@@ -52,6 +52,10 @@ def parse():
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--graph", action="store_true",
                     help="replay each step from a CUDA graph (one per scan order) instead of eager calls")
+    ap.add_argument("--op", default="mixer", choices=["mixer", "sswiglu"],
+                    help="mixer: the chunkwise GLA token mixer (default); sswiglu: the Spatial SwiGLU "
+                         "gate-and-depthwise-conv step (Eq. spatial_swiglu) on --sw-workload")
+    ap.add_argument("--sw-workload", type=int, default=2)
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch size (smaller cases for profiling)")
     return ap.parse_args()
@@ -238,9 +242,130 @@ def run_reference(args, w: wl.Workload, rank: int, world: int):
 # GPU arm
 # --------------------------------------------------------------------------------------
 
+def run_sswiglu(args, rank: int, world: int, local: int):
+    """The Spatial SwiGLU step between its projections (Sec. 3.1, Eq. spatial_swiglu) on
+    one S-SwiGLU workload: device-resident timing, roofline, CPU oracle and end to end."""
+    if world > 1:
+        raise SystemExit("--op sswiglu runs on one GPU")
+    sw = wl.SWIGLU_WORKLOADS[args.sw_workload]
+    inp = wl.sswiglu_inputs(sw.B, sw.grid_h, sw.grid_w, sw.F, sw.dtype, seed=2609 + sw.wid)
+    metric = "tokens/s (Spatial SwiGLU gate-and-conv step)"
+    cfg = {"workload": sw.name, "B": sw.B, "grid": [sw.grid_h, sw.grid_w], "T": sw.T, "F": sw.F,
+           "layout": "one [B, T, 2F] projection output (gate | value)",
+           "l2": "inputs larger than L2 (%.0f MB per step > 129 MB)" % (sw.algorithmic_bytes() / 1e6),
+           "parallelism": "single GPU"}
+
+    def time_cpu(budget_s=10.0):
+        import oracle
+        h64 = wl.storage_to_f64(inp["h"], sw.dtype)
+        F, n, t0 = sw.F, 0, time.perf_counter()
+        while True:  # one image at a time, all channels, until the budget is spent
+            b = n % sw.B
+            oracle.sswiglu_dwconv(h64[b:b + 1, :, :F], h64[b:b + 1, :, F:], inp["weight"], inp["bias"],
+                                  sw.grid_h, sw.grid_w)
+            n += 1
+            el = time.perf_counter() - t0
+            if el >= budget_s or n >= 4 * sw.B:
+                return n * sw.T / el, el, n
+
+    if args.impl == "reference":
+        val, el, n = time_cpu(budget_s=max(5.0, 2.0 * args.steps))
+        print(json.dumps({"impl": "reference", "metric": metric, "value": val, "unit": "tokens/s", "n_gpus": world,
+                          "steps": args.steps, "warmup": args.warmup, "ms_per_step": sw.B * sw.T / val * 1e3,
+                          "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                          "data": "synthetic", "config": cfg,
+                          "cpu_baseline": {"value": val, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                                           "sample": f"{n} images x {sw.T} tokens x {sw.F} channels ({el:.1f} s)"},
+                          "e2e": {"value": val, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                                  "d2h_bytes_per_step": 0}}), flush=True)
+        return
+
+    import torch
+    from paper_2609_26590_gb300 import gla
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    gla.load()
+    dt = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}[sw.dtype]
+    hh = torch.from_numpy(inp["h"].view(np.int16)).view(torch.bfloat16) if sw.dtype == "bf16" \
+        else torch.from_numpy(inp["h"])
+    h = hh.to(dev)
+    wt = torch.from_numpy(inp["weight"]).to(dev)
+    bs = torch.from_numpy(inp["bias"]).to(dev)
+    out = torch.empty((sw.B, sw.T, sw.F), dtype=dt, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        gla.sswiglu_dwconv(h[:, :, :sw.F], h[:, :, sw.F:], wt, bs, sw.grid_h, sw.grid_w, out=out)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    with ClockSampler(local, enabled=not args.no_clocks) as clk:
+        t_begin, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t_begin.record(stream)
+        for i in range(args.steps):
+            starts[i].record(stream)
+            step()
+            ends[i].record(stream)
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    if gla.sync_status() != 0:
+        raise RuntimeError("device status word set during the timed region")
+    ms_per_step = t_begin.elapsed_time(t_end) / args.steps
+    value = sw.B * sw.T / (ms_per_step * 1e-3)
+    kernel_ms = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / args.steps
+    peak, src = load_peaks()
+    achieved = sw.algorithmic_bytes() / (kernel_ms * 1e-3) / 1e9
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        with open(tpath) as f:
+            traffic = json.load(f).get(f"{sw.name}:sswiglu")
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": traffic, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs)" if src == "measured"
+                else "fallback", "kernel": "sswiglu_kernel (TMA value box with zero-padding halo, TMA gate box)",
+                "kernel_ms": kernel_ms, "algorithmic_bytes_per_launch": sw.algorithmic_bytes()}
+    # end to end: pinned host input -> device, the call, output -> pinned host, every step
+    e2e = None
+    if args.e2e_steps > 0:
+        hin = hh.pin_memory()
+        hout = torch.empty(out.shape, dtype=dt).pin_memory()
+        for _ in range(2):
+            h.copy_(hin, non_blocking=True); step(); hout.copy_(out, non_blocking=True)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.e2e_steps):
+            h.copy_(hin, non_blocking=True)
+            step()
+            hout.copy_(out, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = e0.elapsed_time(e1) / args.e2e_steps
+        e2e = {"value": sw.B * sw.T / (e_ms * 1e-3), "unit": "tokens/s",
+               "h2d_bytes_per_step": hin.numel() * hin.element_size(),
+               "d2h_bytes_per_step": hout.numel() * hout.element_size()}
+    cpu = None
+    if not args.no_cpu_baseline:
+        val, el, n = time_cpu()
+        cpu = {"value": val, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+               "sample": f"{n} images x {sw.T} tokens x {sw.F} channels ({el:.1f} s wall, numpy fp64)"}
+    print(json.dumps({"metric": metric, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+                      "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+                      "scaling": "weak", "vs_baseline": None, "dtype": sw.dtype,
+                      "data": "synthetic (seeded, recipe in workloads.py)", "config": cfg, "roofline": roofline,
+                      "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": args.steps, "clocks": clk.summary()}),
+          flush=True)
+
+
 def main():
     args = parse()
     rank, world, local = dist_env()
+    if args.op == "sswiglu":
+        run_sswiglu(args, rank, world, local)
+        return
     w = wl.WORKLOADS[args.workload]
     if args.batch is not None:
         import dataclasses

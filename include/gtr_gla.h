@@ -187,6 +187,27 @@ gtr_status_t gtr_gla_fwd_gated_ws(const void *q, const void *k, const void *v, c
                                   gtr_dtype_t dtype, void *out, float *final_state, void *workspace,
                                   size_t workspace_bytes, cudaStream_t stream);
 
+/* Spatial SwiGLU between its two projections (Sec. 3.1, Eq. spatial_swiglu):
+ *   out = SiLU(X W_g) * DWConv3x3(X W_v),
+ * the step the deployed S-SwiGLU kernel fuses (Sec. 4).  `gate` = X W_g and
+ * `value` = X W_v are [B, T, F] with T = grid_h * grid_w tokens in spatial
+ * row-major order and in_stride elements from one token to the next (F for
+ * separate tensors, 2F when both halves of one [B, T, 2F] projection output
+ * are passed, value = gate + F).  The value branch is convolved per channel on
+ * the grid_h x grid_w grid with zero padding: weight[f][i][j] (fp32, [F][3][3])
+ * multiplies the value at row offset i - 1 and column offset j - 1 (the
+ * cross-correlation of a depthwise 2-D convolution layer), plus bias[f] (fp32
+ * [F], or NULL for none); the product with SiLU(gate) is accumulated in fp32
+ * and rounded once to the dtype.  out: [B, T, F] contiguous, same dtype; it
+ * must not overlap gate or value.  gate, value and out 16-byte aligned, F and
+ * in_stride multiples of 8 elements (4 for fp32); grid_w <= 254.  Device
+ * pointers; allocates nothing and does not synchronise (capturable).
+ * Returns GTR_ERR_INVALID_ARG / GTR_ERR_UNSUPPORTED before any launch; a
+ * device-side wait that gives up is reported by gtr_gla_sync_status. */
+gtr_status_t gtr_sswiglu_dwconv(const void *gate, const void *value, long long in_stride,
+                                const float *weight, const float *bias, int B, int grid_h,
+                                int grid_w, int F, gtr_dtype_t dtype, void *out, cudaStream_t stream);
+
 /* Size of the fixed device scratch array behind gtr_gla_fwd_noalloc.  The
  * library holds one such array on every GPU where it is loaded, from the
  * module's load until the process exits.  The split schedule needs at most

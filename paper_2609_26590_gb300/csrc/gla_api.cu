@@ -414,10 +414,37 @@ gtr_status_t gtr_gla_fwd_host(const void *q_host, const void *k_host, const void
 gtr_status_t gtr_gla_sync_status(cudaStream_t stream) {
     cudaError_t e = cudaStreamSynchronize(stream);
     if (e != cudaSuccess) return cuda_fail(e);
-    unsigned int word = 0;
+    unsigned int word = 0, sw = 0;
     e = gtr::read_and_clear_device_status(&word);
     if (e != cudaSuccess) return cuda_fail(e);
-    if (word & gtr::kStatusTimeout) return GTR_ERR_TIMEOUT;
+    e = gtr::read_and_clear_sswiglu_status(&sw);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if ((word | sw) & gtr::kStatusTimeout) return GTR_ERR_TIMEOUT;
+    return GTR_OK;
+}
+
+gtr_status_t gtr_sswiglu_dwconv(const void *gate, const void *value, long long in_stride, const float *weight,
+                                const float *bias, int B, int grid_h, int grid_w, int F, gtr_dtype_t dtype,
+                                void *out, cudaStream_t stream) {
+    if (dtype < GTR_F32 || dtype > GTR_BF16) return GTR_ERR_INVALID_ARG;
+    if (B < 0 || grid_h < 1 || grid_w < 1 || F < 1) return GTR_ERR_INVALID_ARG;
+    const long long es = elem_size(dtype), vec = 16 / es;
+    const long long T = (long long)grid_h * grid_w;
+    if (F % vec != 0 || in_stride < F || (in_stride * es) % 16 != 0) return GTR_ERR_INVALID_ARG;
+    if (T > 0x7fffffffLL || (long long)B * T > (1LL << 40) / (in_stride + 1)) return GTR_ERR_INVALID_ARG;
+    if (B == 0) return GTR_OK;
+    if (!gate || !value || !weight || !out || !aligned(gate) || !aligned(value) || !aligned(out))
+        return GTR_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(weight) & 3u) || (bias && (reinterpret_cast<uintptr_t>(bias) & 3u)))
+        return GTR_ERR_INVALID_ARG;
+    // the output must not overlap the inputs (the convolution reads neighbouring tokens)
+    const size_t in_bytes = (size_t)((B * T - 1) * in_stride + F) * es, out_bytes = (size_t)(B * T * F) * es;
+    if (overlaps(out, out_bytes, gate, in_bytes) || overlaps(out, out_bytes, value, in_bytes))
+        return GTR_ERR_INVALID_ARG;
+    gtr::SwProblem p{gate, value, in_stride, weight, bias, out, B, grid_h, grid_w, F, (int)dtype};
+    if (!gtr::sswiglu_supported(p)) return GTR_ERR_UNSUPPORTED;
+    const cudaError_t e = gtr::launch_sswiglu(p, stream);
+    if (e != cudaSuccess) return cuda_fail(e);
     return GTR_OK;
 }
 

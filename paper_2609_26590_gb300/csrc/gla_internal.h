@@ -51,6 +51,25 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
 // Device status word of the current device (set by bounded device waits).
 cudaError_t read_and_clear_device_status(unsigned int *status);
 
+// The driver's cuTensorMapEncodeTiled (as void *; null when the driver lacks it).
+void *tensor_map_encoder();
+
+// Spatial SwiGLU between its projections (sswiglu.cu): out = SiLU(gate) * DWConv3x3(value).
+struct SwProblem {
+    const void *gate, *value;   // [B, T, F] at in_stride elements per token
+    long long in_stride;
+    const float *weight;        // [F][3][3]
+    const float *bias;          // [F] or null
+    void *out;                  // [B, T, F], F elements per token
+    int B, grid_h, grid_w, F;
+    int dtype;                  // 0 f32, 1 f16, 2 bf16
+};
+// Grids the kernel takes (a tile's box spans the grid width plus the halo).
+bool sswiglu_supported(const SwProblem &p);
+cudaError_t launch_sswiglu(const SwProblem &p, cudaStream_t stream);
+// Status word of the S-SwiGLU kernel's bounded wait (kStatusTimeout).
+cudaError_t read_and_clear_sswiglu_status(unsigned int *status);
+
 enum : unsigned int { kStatusTimeout = 1u };
 
 }  // namespace gtr

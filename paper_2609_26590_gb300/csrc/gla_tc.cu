@@ -1293,6 +1293,8 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     return cudaGetLastError();
 }
 
+void *tensor_map_encoder() { return reinterpret_cast<void *>(get_encode()); }
+
 cudaError_t read_and_clear_device_status(unsigned int *status) {
     cudaError_t e = cudaMemcpyFromSymbol(status, g_device_status, sizeof(unsigned int));
     if (e != cudaSuccess) return e;

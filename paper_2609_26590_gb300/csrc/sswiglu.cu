@@ -1,0 +1,324 @@
+// sswiglu.cu -- Spatial SwiGLU between its two projections (Sec. 3.1, Eq.
+// spatial_swiglu): Z = SiLU(X W_g) * DWConv3x3(X W_v) on the patch grid, the
+// step the deployed S-SwiGLU kernel fuses (Sec. 4).
+//
+// Memory-bound: per token it reads F gate and F value elements and writes F
+// outputs.  Work is cut into tiles of R grid rows x one 128-byte channel slice
+// (64 channels at 16 bits, 32 at fp32) of one image, one CTA of 256 threads per
+// tile, two CTAs per SM (up to 108 KB of shared memory each), so that one CTA's
+// TMA loads overlap the other's arithmetic.  (A persistent CTA per SM with two
+// stages, or two persistent CTAs per SM, measured 4-25 % slower on a GB300: a
+// CTA-wide barrier per tile idles its warps.)  A tile's value box covers rows y0-1 ..
+// y0+R and columns -1 .. W of the slice: it starts at -1 on both grid axes and
+// runs one past the last row and column, where the tensor map returns zeros,
+// which is exactly the convolution's zero padding; the gate box covers the
+// tile's own tokens.  Each thread owns one 16-byte channel group (its 9 taps and
+// bias in registers, reloaded per tile) and walks the tile's tokens: 9 + 1
+// shared-memory reads, fp32 accumulation, one 16-byte store.  Neighbouring row
+// tiles re-read their halo rows, which L2 serves.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include <atomic>
+#include <cstdint>
+#include <cstring>
+
+#include "gla_internal.h"
+#include "tc_ptx.cuh"
+
+namespace gtr {
+
+__device__ unsigned int g_sswiglu_status;
+
+namespace {
+
+using namespace ptx;
+
+constexpr int kSwThreads = 256;
+constexpr int kSwStageBudget = 108 * 1024;        // a tile's boxes (two CTAs per SM)
+constexpr int kSwSmemBudget = 2 * kSwStageBudget;  // wide grids: one CTA per SM
+constexpr int kSwMaxRows = 32;
+constexpr uint64_t kSwWaitNs = 1000000000ull;     // 1 s: a tile's copies never take that long
+
+struct SwParams {
+    CUtensorMap vmap;       // value tensor: dims (F, W, Hg, B), box (slice, W + 2, rows + 2, 1)
+    CUtensorMap gmap;       // gate tensor: same dims, box (slice, W, rows, 1)
+    void *out;
+    const float *weight;
+    const float *bias;
+    int grid_h, grid_w, F, rows, ntile_y, ntile_f, ntiles, nstage;
+    uint32_t vbytes, gbytes, stage_bytes;  // box bytes, and the stride of the stages
+};
+
+template <typename E> struct Vec16;
+template <> struct Vec16<float> {
+    static constexpr int n = 4;
+    static __device__ __forceinline__ void unpack(uint4 q, float (&v)[4]) {
+        v[0] = __uint_as_float(q.x);
+        v[1] = __uint_as_float(q.y);
+        v[2] = __uint_as_float(q.z);
+        v[3] = __uint_as_float(q.w);
+    }
+    static __device__ __forceinline__ uint4 pack(const float (&v)[4]) {
+        return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
+                          __float_as_uint(v[3]));
+    }
+};
+template <> struct Vec16<__half> {
+    static constexpr int n = 8;
+    static __device__ __forceinline__ void unpack(uint4 q, float (&v)[8]) {
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
+            v[2 * i] = f.x;
+            v[2 * i + 1] = f.y;
+        }
+    }
+    static __device__ __forceinline__ uint4 pack(const float (&v)[8]) {
+        uint32_t w[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const __half2 h = __floats2half2_rn(v[2 * i], v[2 * i + 1]);
+            w[i] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        return make_uint4(w[0], w[1], w[2], w[3]);
+    }
+};
+template <> struct Vec16<__nv_bfloat16> {
+    static constexpr int n = 8;
+    static __device__ __forceinline__ void unpack(uint4 q, float (&v)[8]) {
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            v[2 * i] = __uint_as_float(w[i] << 16);
+            v[2 * i + 1] = __uint_as_float(w[i] & 0xFFFF0000u);
+        }
+    }
+    static __device__ __forceinline__ uint4 pack(const float (&v)[8]) {
+        uint32_t w[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+            w[i] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        return make_uint4(w[0], w[1], w[2], w[3]);
+    }
+};
+
+struct TilePos {
+    int f0, y0, b;
+};
+template <int SLICE>
+__device__ __forceinline__ TilePos tile_pos(const SwParams &p, int t) {
+    const int tf = t % p.ntile_f, rest = t / p.ntile_f;
+    return {tf * SLICE, (rest % p.ntile_y) * p.rows, rest / p.ntile_y};
+}
+
+// TMA loads of the CTA's k-th tile into stage k % nstage (one thread).  Always
+// inlined: the tensor maps are addressed in the kernel's parameter space.
+template <int SLICE>
+__device__ __forceinline__ void issue_tile(const SwParams &p, uint8_t *smem, uint64_t *full, int first, int step,
+                                           int k) {
+    const TilePos tp = tile_pos<SLICE>(p, first + k * step);
+    uint8_t *st = smem + (size_t)(k % p.nstage) * p.stage_bytes;
+    uint64_t *bar = &full[k % p.nstage];
+    mbar_arrive_expect_tx(bar, p.vbytes + p.gbytes);
+    tma_load_4d(st, &p.vmap, bar, tp.f0, -1, tp.y0 - 1, tp.b);
+    tma_load_4d(st + p.vbytes, &p.gmap, bar, tp.f0, 0, tp.y0, tp.b);
+}
+
+template <typename E>
+__global__ void __launch_bounds__(kSwThreads, 2) sswiglu_kernel(const __grid_constant__ SwParams p) {
+    constexpr int VEC = Vec16<E>::n;        // elements per 16 bytes
+    constexpr int SLICE = 8 * VEC;          // channels per tile: 128 bytes, eight groups
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
+    __shared__ uint64_t full[2];
+
+    const int W = p.grid_w;
+    // the CTA's tiles: blockIdx.x, blockIdx.x + gridDim.x, ...
+    const int first = static_cast<int>(blockIdx.x), step = static_cast<int>(gridDim.x);
+    const int count = first < p.ntiles ? (p.ntiles - 1 - first) / step + 1 : 0;
+    if (threadIdx.x == 0) {
+        mbar_init(&full[0], 1);
+        mbar_init(&full[1], 1);
+        fence_mbar_init();
+        for (int k = 0; k < p.nstage && k < count; ++k) issue_tile<SLICE>(p, smem, full, first, step, k);
+    }
+    __syncthreads();
+
+    const int cg = static_cast<int>(threadIdx.x & 7u);
+    E *out = static_cast<E *>(p.out);
+    const long long T = (long long)p.grid_h * W;
+    for (int k = 0; k < count; ++k) {
+        const TilePos tp = tile_pos<SLICE>(p, first + k * step);
+        const int fc = tp.f0 + cg * VEC;
+        const bool live = fc < p.F;   // F is a multiple of VEC
+        const int R = p.grid_h - tp.y0 < p.rows ? p.grid_h - tp.y0 : p.rows;
+        // this tile's taps and bias for the thread's channel group, read while its copies land
+        float w[9][VEC], bs[VEC];
+#pragma unroll
+        for (int e = 0; e < VEC; ++e) {
+#pragma unroll
+            for (int q = 0; q < 9; ++q) w[q][e] = live ? p.weight[(size_t)(fc + e) * 9 + q] : 0.f;
+            bs[e] = (live && p.bias != nullptr) ? p.bias[fc + e] : 0.f;
+        }
+        const bool ok = mbar_wait(&full[k % p.nstage], (k / p.nstage) & 1, nullptr, kSwWaitNs);
+        if (__syncthreads_or(!ok)) {  // the CTA gives up together
+            if (threadIdx.x == 0) {
+                atomicOr(&g_sswiglu_status, kStatusTimeout);
+                // never leave while copies may still land in this CTA's shared memory
+                for (int j = k; j < count && j < k + p.nstage; ++j)
+                    mbar_wait(&full[j % p.nstage], (j / p.nstage) & 1, nullptr, kSwWaitNs);
+            }
+            __syncthreads();
+            return;
+        }
+        const uint8_t *vt = smem + (size_t)(k % p.nstage) * p.stage_bytes;
+        const uint8_t *gt = vt + p.vbytes;
+        const int ntok = R * W;
+        for (int tk = static_cast<int>(threadIdx.x >> 3); tk < ntok; tk += kSwThreads / 8) {
+            const int r = tk / W, x = tk - r * W;
+            float acc[VEC];
+#pragma unroll
+            for (int e = 0; e < VEC; ++e) acc[e] = bs[e];
+            // value tile row r + i holds grid row y0 + r + i - 1, column x + j grid column x + j - 1
+#pragma unroll
+            for (int i = 0; i < 3; ++i) {
+#pragma unroll
+                for (int j = 0; j < 3; ++j) {
+                    float v[VEC];
+                    Vec16<E>::unpack(*reinterpret_cast<const uint4 *>(
+                                         vt + ((size_t)(r + i) * (W + 2) + (x + j)) * 128 + cg * 16),
+                                     v);
+#pragma unroll
+                    for (int e = 0; e < VEC; ++e) acc[e] = fmaf(w[3 * i + j][e], v[e], acc[e]);
+                }
+            }
+            if (live) {
+                float g[VEC], z[VEC];
+                Vec16<E>::unpack(*reinterpret_cast<const uint4 *>(gt + (size_t)tk * 128 + cg * 16), g);
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) z[e] = __fdividef(g[e], 1.f + __expf(-g[e])) * acc[e];
+                const long long tok = (long long)tp.b * T + (long long)(tp.y0 + r) * W + x;
+                *reinterpret_cast<uint4 *>(out + tok * p.F + fc) = Vec16<E>::pack(z);
+            }
+        }
+        __syncthreads();  // every thread is done with this stage
+        if (threadIdx.x == 0 && k + p.nstage < count) issue_tile<SLICE>(p, smem, full, first, step, k + p.nstage);
+    }
+}
+
+int elem_bytes(int dtype) { return dtype == 0 ? 4 : 2; }
+
+// Shared memory of one stage for `rows` grid rows: the value box (rows + 2) x (W + 2)
+// and the gate box rows x W, 128 bytes a token.
+size_t stage_bytes(int rows, int W) { return 128u * ((size_t)(rows + 2) * (W + 2) + (size_t)rows * W); }
+
+// Rows per tile: the most rows (up to kSwMaxRows and the grid's height) whose boxes
+// fit kSwStageBudget (two CTAs per SM), else, for grids too wide for one row there,
+// kSwSmemBudget (one CTA per SM).  One stage: the kernel also runs a CTA over
+// several tiles with two stages, which measured slower and is not launched.
+void tile_plan(const SwProblem &p, int *rows, int *nstage) {
+    for (int pass = 0; pass < 2; ++pass) {
+        const int ns = 1;
+        const size_t budget = pass == 0 ? kSwStageBudget : kSwSmemBudget;
+        int r = 0;
+        while (r < kSwMaxRows && r < p.grid_h && stage_bytes(r + 1, p.grid_w) <= budget) ++r;
+        if (r >= 1) {
+            *rows = r;
+            *nstage = ns;
+            return;
+        }
+    }
+    *rows = 0;
+    *nstage = 0;
+}
+
+template <typename E>
+cudaError_t launch_typed(const SwParams &sp, unsigned grid, size_t smem, cudaStream_t stream) {
+    static std::atomic<unsigned long long> set_on_devices(0);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (!(set_on_devices.load(std::memory_order_relaxed) & bit)) {
+        e = cudaFuncSetAttribute(sswiglu_kernel<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(kSwSmemBudget + 256));
+        if (e != cudaSuccess) return e;
+        set_on_devices.fetch_or(bit);
+    }
+    sswiglu_kernel<E><<<grid, kSwThreads, smem, stream>>>(sp);
+    return cudaGetLastError();
+}
+
+bool encode(CUtensorMap *m, const SwProblem &p, const void *base, int box_w, int box_h) {
+    auto enc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(tensor_map_encoder());
+    if (!enc) return false;
+    const int es = elem_bytes(p.dtype);
+    const cuuint64_t row = static_cast<cuuint64_t>(p.in_stride) * es;
+    const cuuint64_t T = static_cast<cuuint64_t>(p.grid_h) * p.grid_w;
+    cuuint64_t dims[4] = {static_cast<cuuint64_t>(p.F), static_cast<cuuint64_t>(p.grid_w),
+                          static_cast<cuuint64_t>(p.grid_h), static_cast<cuuint64_t>(p.B)};
+    cuuint64_t strides[3] = {row, row * p.grid_w, row * T};
+    cuuint32_t box[4] = {static_cast<cuuint32_t>(128 / es), static_cast<cuuint32_t>(box_w),
+                         static_cast<cuuint32_t>(box_h), 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUtensorMapDataType dt = p.dtype == 0 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32
+                                   : p.dtype == 1 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16
+                                                  : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    return enc(m, dt, 4, const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+bool sswiglu_supported(const SwProblem &p) {
+    // the value box spans the grid width plus the halo in one TMA dimension (at most
+    // 256 elements), and a stage of at least one row must fit the shared memory
+    int rows = 0, nstage = 0;
+    tile_plan(p, &rows, &nstage);
+    return p.grid_w + 2 <= 256 && rows >= 1 && tensor_map_encoder() != nullptr;
+}
+
+cudaError_t launch_sswiglu(const SwProblem &p, cudaStream_t stream) {
+    if (!sswiglu_supported(p)) return cudaErrorInvalidValue;
+    const int slice = 128 / elem_bytes(p.dtype);
+    SwParams sp;
+    std::memset(&sp, 0, sizeof(sp));
+    tile_plan(p, &sp.rows, &sp.nstage);
+    sp.out = p.out;
+    sp.weight = p.weight;
+    sp.bias = p.bias;
+    sp.grid_h = p.grid_h;
+    sp.grid_w = p.grid_w;
+    sp.F = p.F;
+    sp.ntile_y = (p.grid_h + sp.rows - 1) / sp.rows;
+    sp.ntile_f = (p.F + slice - 1) / slice;
+    const long long tiles = (long long)p.B * sp.ntile_y * sp.ntile_f;
+    if (tiles <= 0 || tiles > 0x7fffffffLL) return cudaErrorInvalidValue;
+    sp.ntiles = static_cast<int>(tiles);
+    sp.vbytes = static_cast<uint32_t>(128u * (size_t)(sp.rows + 2) * (p.grid_w + 2));
+    sp.gbytes = static_cast<uint32_t>(128u * (size_t)sp.rows * p.grid_w);
+    sp.stage_bytes = (sp.vbytes + sp.gbytes + 127u) & ~127u;
+    if (!encode(&sp.vmap, p, p.value, p.grid_w + 2, sp.rows + 2) || !encode(&sp.gmap, p, p.gate, p.grid_w, sp.rows))
+        return cudaErrorInvalidValue;
+    const unsigned grid = static_cast<unsigned>(tiles);  // one CTA per tile
+    const size_t smem = (size_t)sp.nstage * sp.stage_bytes + 128;
+    if (p.dtype == 0) return launch_typed<float>(sp, grid, smem, stream);
+    if (p.dtype == 1) return launch_typed<__half>(sp, grid, smem, stream);
+    return launch_typed<__nv_bfloat16>(sp, grid, smem, stream);
+}
+
+cudaError_t read_and_clear_sswiglu_status(unsigned int *status) {
+    cudaError_t e = cudaMemcpyFromSymbol(status, g_sswiglu_status, sizeof(unsigned int));
+    if (e != cudaSuccess) return e;
+    const unsigned int zero = 0;
+    return cudaMemcpyToSymbol(g_sswiglu_status, &zero, sizeof(unsigned int));
+}
+
+}  // namespace gtr

@@ -55,6 +55,8 @@ def load(path: Optional[str] = None):
         lib.gtr_gla_tc_supported.argtypes = [ci] * 8
         lib.gtr_gla_workspace_bytes.restype = st
         lib.gtr_gla_workspace_bytes.argtypes = [ci] * 7
+        lib.gtr_sswiglu_dwconv.restype = ci
+        lib.gtr_sswiglu_dwconv.argtypes = [vp, vp, ctypes.c_longlong, vp, vp] + [ci] * 5 + [vp, vp]
         lib.gtr_gla_chunk_boxes.restype = ci
         lib.gtr_gla_chunk_boxes.argtypes = [ci] * 4 + [ctypes.POINTER(ci), ci]
         lib.gtr_gla_split_plan.restype = ci
@@ -159,6 +161,40 @@ def split_plan(B: int, H: int, grid_h: int, grid_w: int, Dk: int, Dv: int, n_sm:
                                     ctypes.byref(seg_len))
     _check(status, "gtr_gla_split_plan", lib)
     return nseg.value, seg_len.value
+
+
+def sswiglu_dwconv(gate: torch.Tensor, value: torch.Tensor, weight: torch.Tensor, bias: Optional[torch.Tensor],
+                   grid_h: int, grid_w: int, out: Optional[torch.Tensor] = None,
+                   stream: Optional[torch.cuda.Stream] = None) -> torch.Tensor:
+    """Spatial SwiGLU between its projections through ``gtr_sswiglu_dwconv``:
+    out = SiLU(gate) * DWConv3x3(value) on the grid.  gate, value: [B, T, F] CUDA
+    tensors of one dtype whose last dimension is contiguous and whose token
+    stride is shared (e.g. the two halves of one [B, T, 2F] tensor); weight:
+    [F, 3, 3] float32, bias: [F] float32 or None (CUDA).  Returns out [B, T, F]."""
+    lib = load()
+    if gate.dim() != 3 or gate.shape != value.shape or gate.dtype != value.dtype:
+        raise ValueError("gate and value must be [B, T, F] tensors of one dtype")
+    if gate.dtype not in _DTYPES:
+        raise ValueError(f"unsupported dtype {gate.dtype}")
+    B, T, F = gate.shape
+    if T != grid_h * grid_w:
+        raise ValueError("T must equal grid_h * grid_w")
+    if gate.stride(2) != 1 or value.stride(2) != 1 or gate.stride(1) != value.stride(1) or \
+            gate.stride(0) != T * gate.stride(1) or value.stride(0) != T * value.stride(1):
+        raise ValueError("gate and value need contiguous channels and one shared token stride")
+    if not gate.is_cuda or not value.is_cuda or not weight.is_cuda:
+        raise ValueError("inputs must be CUDA tensors")
+    if weight.dtype != torch.float32 or not weight.is_contiguous() or tuple(weight.shape) != (F, 3, 3):
+        raise ValueError("weight must be a contiguous [F, 3, 3] float32 tensor")
+    if bias is not None and (bias.dtype != torch.float32 or not bias.is_contiguous() or tuple(bias.shape) != (F,)):
+        raise ValueError("bias must be a contiguous [F] float32 tensor")
+    if out is None:
+        out = torch.empty((B, T, F), dtype=gate.dtype, device=gate.device)
+    status = lib.gtr_sswiglu_dwconv(gate.data_ptr(), value.data_ptr(), gate.stride(1), weight.data_ptr(),
+                                    bias.data_ptr() if bias is not None else None, B, grid_h, grid_w, F,
+                                    _DTYPES[gate.dtype], out.data_ptr(), _stream_ptr(stream))
+    _check(status, "gtr_sswiglu_dwconv", lib)
+    return out
 
 
 def chunk_boxes(grid_h: int, grid_w: int, order: int, c: int):

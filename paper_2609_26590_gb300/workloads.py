@@ -147,3 +147,62 @@ def workload_inputs(w: Workload, B: Optional[int] = None, seed: Optional[int] = 
     s = (1234 + w.wid) if seed is None else seed
     return make_inputs(w.B if B is None else B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, w.dtype,
                        s, tau=w.tau, z_mean=w.z_mean, frac_nodecay=w.frac_nodecay)
+
+
+# ---------------------------------------------------------------- Spatial SwiGLU (Sec. 3.1)
+#
+# Inputs of the step between the two projections of Eq. (spatial_swiglu): the
+# projection output X [W_g | W_v] as one [B, T, 2F] tensor (gate channels first),
+# the depthwise 3 x 3 taps [F, 3, 3] and the bias [F] (fp32).  F is the model
+# width times the S-SwiGLU expansion ratio (App. B.3: widths 192 / 384, ratio 4,
+# 6 for GTR-X).  Seeds are 2609 + id.
+#
+# ====  ======  ====  ===============  =====  =====================================
+#  id   dtype    B     grid (T)         F      model
+# ====  ======  ====  ===============  =====  =====================================
+#  0    f32      1     8x12 (96)          64   small correctness case
+#  1    f16      1     40x40 (1600)      768   GTR-S at 640^2
+#  2    bf16    32     40x40 (1600)     1536   GTR-L at 640^2, batch 32
+#  3    f16      8     80x80 (6400)     2304   GTR-X at 1280^2, batch 8
+# ====  ======  ====  ===============  =====  =====================================
+#
+# gate and value pre-activations ~ N(0, 1), taps ~ N(0, 1/9), bias ~ N(0, 0.1^2),
+# all rounded to the storage dtype (taps and bias to fp32).
+
+@dataclasses.dataclass(frozen=True)
+class SwigluWorkload:
+    wid: int
+    name: str
+    dtype: str
+    B: int
+    grid_h: int
+    grid_w: int
+    F: int
+
+    @property
+    def T(self) -> int:
+        return self.grid_h * self.grid_w
+
+    def algorithmic_bytes(self) -> int:
+        """Gate and value read once, the output written once, plus the taps and bias."""
+        return self.B * self.T * 3 * self.F * ELEM_SIZE[self.dtype] + self.F * 10 * 4
+
+
+SWIGLU_WORKLOADS: Dict[int, SwigluWorkload] = {
+    0: SwigluWorkload(0, "sswiglu_tiny_8x12", "f32", 1, 8, 12, 64),
+    1: SwigluWorkload(1, "sswiglu_gtr_s_640", "f16", 1, 40, 40, 768),
+    2: SwigluWorkload(2, "sswiglu_gtr_l_640_b32", "bf16", 32, 40, 40, 1536),
+    3: SwigluWorkload(3, "sswiglu_gtr_x_1280_b8", "f16", 8, 80, 80, 2304),
+}
+
+
+def sswiglu_inputs(B: int, grid_h: int, grid_w: int, F: int, dtype: str, seed: int,
+                   with_bias: bool = True) -> Dict[str, np.ndarray]:
+    """Seeded [B, T, 2F] projection output (gate channels, then value channels) in
+    the storage dtype, fp32 taps [F, 3, 3] and bias [F] (None without bias)."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    T = grid_h * grid_w
+    h = round_to_storage(rng.standard_normal((B, T, 2 * F)), dtype)
+    w = (rng.standard_normal((F, 3, 3)) / 3.0).astype(np.float32)
+    b = (0.1 * rng.standard_normal(F)).astype(np.float32) if with_bias else None
+    return {"h": h, "weight": w, "bias": b}

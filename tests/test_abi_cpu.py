@@ -149,3 +149,23 @@ def test_gated_ws_entry_point_validates_before_any_launch(lib):
     assert call(gate=(1 << 26) + 64) == 1         # overlaps the output
     assert fwd(None, None, None, None, None, None, 1e-6, 0, 2, 8, 8, 64, 64, 0, 1, None, None, None, 0,
                None) == 0
+
+
+def test_sswiglu_entry_point_validates_before_any_launch(lib):
+    fwd = lib.gtr_sswiglu_dwconv
+    fwd.restype = ctypes.c_int
+    fwd.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_longlong, ctypes.c_void_p, ctypes.c_void_p] + \
+        [ctypes.c_int] * 5 + [ctypes.c_void_p, ctypes.c_void_p]
+    g, v, w, o = 1 << 24, (1 << 24) + 128, 1 << 25, 1 << 26
+
+    def call(gate=g, value=v, stride=128, weight=w, B=1, gh=4, gw=4, F=64, dtype=1, out=o):
+        return fwd(gate, value, stride, weight, None, B, gh, gw, F, dtype, out, None)
+    assert call(F=12) == 1                 # not a multiple of 8 elements
+    assert call(stride=60) == 1            # token stride below F
+    assert call(stride=68) == 1            # token stride not a multiple of 16 bytes
+    assert call(gate=g + 8) == 1           # not 16-byte aligned
+    assert call(weight=None) == 1
+    assert call(gh=0) == 1
+    assert call(dtype=7) == 1
+    assert call(out=g + 1024) == 1         # the output overlaps the inputs
+    assert call(B=0, gate=None, value=None, weight=None, out=None) == 0   # empty batch: nothing to do
