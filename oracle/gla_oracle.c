@@ -15,7 +15,8 @@
  *     with the value-side decay fixed to one (Sec. 3.1 and App. C.3), and
  *     gamma_t = exp(g_t), g_t the learned log-decay the operator consumes
  *     (Sec. 3.3).  The d_k^{-1/2} factor of the paper's o_t is NOT applied
- *     here: the caller folds it into k (reading recorded in the design doc).
+ *     here: the caller folds it into k, which gives the same o_t (the scale
+ *     multiplies every k_t^T v_t term of S_t alike).
  *   - Sec. 3.1 "Directional scanning": four raster orders over the grid
  *     (left-to-right, right-to-left, top-to-bottom, bottom-to-top), one
  *     sequence per image with the state carried across rows/columns, outputs
