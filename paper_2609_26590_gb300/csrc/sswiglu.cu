@@ -7,7 +7,7 @@
 // (64 channels at 16 bits, 32 at fp32) of one image, one CTA of 256 threads per
 // tile, two CTAs per SM (up to 108 KB of shared memory each), so that one CTA's
 // TMA loads overlap the other's arithmetic.  (A persistent CTA per SM with two
-// stages, or two persistent CTAs per SM, measured 4-25 % slower on a GB300: a
+// stages, or two persistent CTAs per SM, measured 3-29 % slower on a GB300: a
 // CTA-wide barrier per tile idles its warps.)  A tile's value box covers rows y0-1 ..
 // y0+R and columns -1 .. W of the slice: it starts at -1 on both grid axes and
 // runs one past the last row and column, where the tensor map returns zeros,
