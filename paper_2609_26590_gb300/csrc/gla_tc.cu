@@ -30,7 +30,8 @@
 // written in place (Q^ or Qtil over q, K^ or Kbar over k, the masked scores P
 // over g, bf16 v converted to fp16 in place), so four chunks can be in flight.
 // Only the tf32 score operands use separate buffers, one per gen warpgroup, so
-// that tf32-mode chunks of the two groups never wait for each other.  Row orders load one 64-row TMA box per tensor and chunk; column orders
+// that tf32-mode chunks of the two groups never wait for each other.  Row orders
+// load one 64-row TMA box per tensor and chunk; column orders
 // one box per column segment of the chunk, of the segment's exact height (a
 // tensor map per height).  The scan permutation lives in the box coordinates of
 // the loads and in the addresses of the output stores.
@@ -44,7 +45,8 @@
 //                chunk, then masks the chunk's scores P into fp16.
 //   warps 6-9    gen warpgroup 1 (odd chunks).
 //   warps 10-13  epi: carries the fp32 state S in registers, writes Diag(c1) S,
-//                and stores each chunk's outputs at the tokens' spatial positions.
+//                and stores each chunk's outputs at the tokens' spatial positions
+//                (GENOUT launches: the gen warpgroup that built the chunk stores them).
 //   warp 14      issuer of P(c) and U(c).
 //   warp 15      issuer of O(c).
 // Each issuer waits only for the inputs of its own product, so the issue overhead
@@ -52,6 +54,11 @@
 // A warp reads the TMEM lanes of sub-partition (warp % 4); an M = 64 accumulator
 // keeps rows 16q..16q+15 in lanes 32q..32q+15, and each thread takes one row and
 // 32 of its 64 columns.
+//
+// Few, long sequences are split into segments (MODE kSummary computes each
+// segment's end state from zero and its total decay, MODE kSplitFull starts every
+// segment from the fold of the earlier ones); the last segment may run past the
+// sequence over all-zero padding chunks, which leave the state unchanged.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
