@@ -20,6 +20,9 @@ Prediction"):
 * :func:`gated_output` -- Sec. 3.1, the output gate applied to the mixer's
   output: ``u_t = SiLU(r_t) * RMSNorm(o_t)`` (the epilogue the paper's deployed
   kernel fuses, App. C.3).
+* :func:`gate_producer` -- Sec. 3.1, the key-wise retention gate from its
+  low-rank projection: ``g = log gamma = logsigmoid(x W1 W2 + b) / tau`` (the
+  log-decay the mixer consumes), from ``a = x W1``.
 * :func:`sswiglu_dwconv` -- Sec. 3.1, "Spatial SwiGLU", Eq. (spatial_swiglu):
   the part between its two projections, ``SiLU(X W_g) * DWConv3x3(X W_v)``
   on the patch grid (the part the deployed S-SwiGLU kernel fuses, Sec. 4).
@@ -252,3 +255,24 @@ def sswiglu_dwconv(gate_pre, value_pre, weight, bias, grid_h: int, grid_w: int) 
     with np.errstate(over="ignore"):
         silu = g / (1.0 + np.exp(-g))
     return silu * conv.reshape(B, T, F)
+
+
+def gate_producer(a_low, w2, bias, tau: float) -> np.ndarray:
+    """Sec. 3.1, the retention gate: ``gamma_t = sigmoid(x_t W1 W2 + b)^(1/tau)``,
+    so the log-decay the mixer consumes is ``g_t = logsigmoid(x_t W1 W2 + b) / tau``.
+
+    a_low = x W1: [B, T, r] (the rank-r projection, r = 16 in the paper); w2:
+    [H, r, Dk] (the second factor, one block of key channels per head); bias:
+    [H, Dk]; tau > 0 (16 in the paper).  Returns g: [B, T, H, Dk] in float64.
+    logsigmoid(z) = -log(1 + e^{-z}), evaluated as min(z, 0) - log1p(e^{-|z|})
+    so that neither sign of z overflows.
+    """
+    a = np.asarray(a_low, dtype=np.float64)
+    w = np.asarray(w2, dtype=np.float64)
+    b = np.asarray(bias, dtype=np.float64)
+    if a.ndim != 3 or w.ndim != 3 or w.shape[1] != a.shape[2] or b.shape != (w.shape[0], w.shape[2]):
+        raise ValueError("a_low [B, T, r], w2 [H, r, Dk], bias [H, Dk]")
+    if not tau > 0:
+        raise ValueError("tau must be positive")
+    z = np.einsum("btr,hrd->bthd", a, w) + b
+    return (np.minimum(z, 0.0) - np.log1p(np.exp(-np.abs(z)))) / float(tau)

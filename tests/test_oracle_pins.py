@@ -373,3 +373,44 @@ def test_sswiglu_special_cases():
     w = rng.standard_normal((F, 3, 3))
     np.testing.assert_allclose(oracle.sswiglu_dwconv(g[:, :1], v[:, :1], w, None, 1, 1),
                                silu[:, :1] * v[:, :1] * w[:, 1, 1], rtol=1e-14)
+
+
+# ---------------------------------------------------------------- retention gate from its projection (Sec. 3.1)
+
+def test_gate_producer_hand_worked():
+    with open(os.path.join(GOLDEN, "gate_producer_2tok.json")) as f:
+        d = json.load(f)
+    a = np.array(d["a_low"], dtype=np.float64) * np.log(3.0)
+    g = oracle.gate_producer(a, np.array(d["w2"]), np.array(d["bias"]), d["tau"])
+    expect = np.array([[np.log(v) for _, v in tok] for tok in d["g"]]).reshape(1, 2, 1, 2)
+    np.testing.assert_allclose(g, expect, rtol=1e-14, atol=1e-15)
+
+
+def test_gate_producer_matches_scipy_log_expit():
+    special = pytest.importorskip("scipy.special")
+    rng = np.random.Generator(np.random.PCG64(11))
+    B, T, r, H, Dk, tau = 2, 5, 16, 3, 8, 16.0
+    a = rng.standard_normal((B, T, r)) * 3
+    w2 = rng.standard_normal((H, r, Dk))
+    b = rng.standard_normal((H, Dk))
+    g = oracle.gate_producer(a, w2, b, tau)
+    for h in range(H):
+        z = a @ w2[h] + b[h]                              # [B, T, Dk]
+        np.testing.assert_allclose(g[:, :, h, :], special.log_expit(z) / tau, rtol=1e-12, atol=1e-300)
+
+
+def test_gate_producer_special_cases():
+    rng = np.random.Generator(np.random.PCG64(12))
+    a = rng.standard_normal((1, 4, 16))
+    b = rng.standard_normal((2, 8))
+    # W2 = 0: every token gets logsigmoid(b) / tau
+    g = oracle.gate_producer(a, np.zeros((2, 16, 8)), b, 4.0)
+    np.testing.assert_allclose(g, np.broadcast_to(-np.log1p(np.exp(-b)) / 4.0, g.shape), rtol=1e-14)
+    # tau scales g; g <= 0 always (gamma in (0, 1]); extreme pre-activations stay finite
+    w2 = rng.standard_normal((2, 16, 8)) * 100
+    g1, g2 = oracle.gate_producer(a, w2, b, 1.0), oracle.gate_producer(a, w2, b, 16.0)
+    np.testing.assert_allclose(g2, g1 / 16.0, rtol=1e-14)
+    assert np.all(g1 <= 0) and np.all(np.isfinite(g1))
+    # z = 0: gamma^tau = 1/2
+    g0 = oracle.gate_producer(np.zeros((1, 1, 16)), w2, np.zeros((2, 8)), 2.0)
+    np.testing.assert_allclose(g0, np.full(g0.shape, -np.log(2.0) / 2.0), rtol=1e-15)
