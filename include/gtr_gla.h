@@ -114,10 +114,12 @@ gtr_status_t gtr_gla_fwd_sched(const void *q, const void *k, const void *v,
                                cudaStream_t stream);
 
 /* Bytes of workspace gtr_gla_fwd_ws needs for these arguments on the current
- * device (segment summaries of the split schedule: B*H*(segments-1)*(Dk*Dv +
- * Dk) floats); 0 when the call does not split sequences (the SIMT schedule,
- * or enough sequences to fill the device) or the arguments are invalid.  The
- * number of segments depends on the device's SM count. */
+ * device: the segment summaries of the split schedule (B*H*(segments-1)*(Dk'*Dv'
+ * + Dk') floats, Dk' and Dv' rounded up to multiples of 64), or, for the
+ * balanced schedule (gtr_gla_balanced_plan), one 64 x 64 fp32 hand-off state and
+ * one 64-bit flag per SM; 0 when the call needs neither (the SIMT schedule, or
+ * whole sequences dealt round-robin) or the arguments are invalid.  Both depend
+ * on the device's SM count. */
 size_t gtr_gla_workspace_bytes(int B, int H, int grid_h, int grid_w, int Dk, int Dv,
                                gtr_dtype_t dtype);
 
@@ -132,6 +134,16 @@ size_t gtr_gla_workspace_bytes(int B, int H, int grid_h, int grid_w, int Dk, int
  * NULL outputs (the outputs are then not written). */
 gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm,
                                 int *nseg, int *seg_len);
+
+/* 1 when the tensor-core schedule balances these shapes on a device with n_sm SMs,
+ * else 0 (also for invalid shapes or n_sm < 1).  Balanced: Dk <= 64, no sequence
+ * split, more (sequence, 64-column value slice) units than SMs, and a round-robin
+ * deal of whole units would give the busiest SM at least 1.25 times the chunks of an
+ * even split; every
+ * CTA then takes an equal contiguous range of the units' chunks, and a unit cut by
+ * a range boundary continues from the state (Eq. chunk_boundary_main) the CTA
+ * before it handed over through the workspace.  Host arithmetic only. */
+int gtr_gla_balanced_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm);
 
 /* Introspection of the scan-order gather (Sec. 3.1, directional scanning): the
  * TMA boxes the tensor-core schedule loads for 64-token chunk c of a sequence

@@ -241,6 +241,13 @@ gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, in
     return GTR_OK;
 }
 
+int gtr_gla_balanced_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm) {
+    if (n_sm < 1 || check_shape(B, H, grid_h, grid_w, Dk, Dv, 0, GTR_F16) != GTR_OK || B == 0 || H == 0) return 0;
+    gtr::Problem p{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, B, H, grid_h, grid_w,
+                   Dk, Dv, 0, GTR_F16, (long long)grid_h * grid_w};
+    return gtr::tc_balanced_plan(p, n_sm);
+}
+
 gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const void *log_gate, int B,
                             int H, int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
                             gtr_dtype_t dtype, void *out, float *final_state, void *workspace,

@@ -42,10 +42,16 @@ int tc_chunk_boxes(int order, int T, int grid_h, int grid_w, int c, int *boxes, 
 // this problem on a device with n_sm SMs (host arithmetic only; nseg 1: unsplit).
 void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len);
 // Scratch the tensor-core schedule uses for this problem on the current device:
-// per-segment summaries when it splits sequences (few, long ones), else 0.
+// per-segment summaries when it splits sequences (few, long ones), hand-off states and
+// flags when it balances chunk ranges (tc_balanced_plan), else 0.
 size_t tc_workspace_bytes(const Problem &p);
-// Launches the schedule; it splits sequences only when `workspace` holds at least
-// tc_workspace_bytes(p) bytes (256-byte aligned), else it runs unsplit.
+// 1 when the tensor-core schedule gives every CTA an equal contiguous range of chunks
+// (more units than SMs, a round-robin deal at least 1.25 times an even split's share) on a device
+// with n_sm SMs; its workspace then holds one hand-off state and flag per SM.
+int tc_balanced_plan(const Problem &p, int n_sm);
+// Launches the schedule; it splits sequences or balances ranges only when `workspace`
+// holds at least tc_workspace_bytes(p) bytes (256-byte aligned), else it deals whole
+// sequences round-robin.
 cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes);
 
 // Device status word of the current device (set by bounded device waits).

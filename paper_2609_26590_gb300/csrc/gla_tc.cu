@@ -58,13 +58,18 @@
 // Few, long sequences are split into segments (MODE kSummary computes each
 // segment's end state from zero and its total decay, MODE kSplitFull starts every
 // segment from the fold of the earlier ones); the last segment may run past the
-// sequence over all-zero padding chunks, which leave the state unchanged.
+// sequence over all-zero padding chunks, which leave the state unchanged.  When the
+// units outnumber the SMs unevenly (MODE kBalanced), every CTA takes an equal
+// contiguous range of the units' chunks: the head of the unit its range ends in comes
+// first and hands its end state to the next CTA through global memory, the tail of
+// the unit its range starts in comes last, from the state the CTA before handed over.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
 #include <atomic>
+#include <chrono>
 #include <cstdlib>
 #include <cstring>
 #include <list>
@@ -98,9 +103,11 @@ constexpr float kMaxRefF16 = 8.0f;        // fp16 score operands: factors within
 constexpr float kMaxRefTF32 = 100.0f;     // tf32 score operands: factors within 2^{+-100}
 
 enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
-// Kernel passes: kFull (sequences whole), kSplitFull (outputs of segments that
-// start from the fold of the earlier segments' summaries), kSummary (the summaries).
-enum : int { kFull = 0, kSplitFull = 1, kSummary = 2 };
+// Kernel passes: kFull (sequences whole, dealt round-robin), kSplitFull (outputs of
+// segments that start from the fold of the earlier segments' summaries), kSummary (the
+// summaries), kBalanced (equal contiguous chunk ranges per CTA, the state of a unit cut
+// by a range boundary handed from one CTA to the next; one key half).
+enum : int { kFull = 0, kSplitFull = 1, kSummary = 2, kBalanced = 3 };
 constexpr int kMinSegChunks = 2;          // a split segment keeps at least this many chunks
 
 // Shared-memory map (byte offsets from a 1024-aligned base).
@@ -158,6 +165,9 @@ struct TcParams {
                                            // [Dk][Dv] and total decay [Dk], fp32
     int drop_load;                         // test hook: CTA 0 withholds its first chunk's load, so the
                                            // bounded waits run out and the call reports a timeout
+    unsigned long long *flags;             // kBalanced: per CTA, == epoch once its hand-off state (in
+                                           // summary, [64][64] fp32 per CTA) is written; cleared when read
+    unsigned long long epoch;              // kBalanced: nonzero, new for every launch
 };
 
 // ---------------------------------------------------------------- helpers
@@ -228,12 +238,15 @@ __host__ __device__ __forceinline__ int chunk_w0(int order, int T, int c) {
 // key channels (o = sum over halves of Qtil_a S_a + P_a V), so the halves go through
 // the same per-chunk pipeline and only their O products share one accumulator.
 struct StreamPos {
-    int bh;   // sequence b * H + h
-    int vb;   // value slice
-    int c;    // chunk of the sequence
-    int a;    // key half
-    int seg;  // segment of the sequence
-    int cl;   // chunk within the segment
+    int bh;      // sequence b * H + h
+    int vb;      // value slice
+    int c;       // chunk of the sequence
+    int a;       // key half
+    int seg;     // segment of the sequence
+    int cl;      // chunk within the segment
+    bool start;  // a run of the unit starts here: its state is set
+    bool hin;    // kBalanced: the run starts from the previous CTA's hand-off state
+    bool hout;   // kBalanced: after this chunk the state goes to the next CTA
 };
 // Units are (sequence, segment, value slice), the value slice fastest (the two
 // slices of a sequence read the same q, k and gates); a unit covers seg_len chunks.
@@ -245,7 +258,52 @@ __device__ __forceinline__ StreamPos stream_pos(int v, int L, int nh, int lognv,
     const int seg = nsu == 1 ? 0 : rest % nsu;
     const int bh = nsu == 1 ? rest : rest / nsu;
     const int cl = rem / nh;
-    return {bh, unit & ((1 << lognv) - 1), seg * L + cl, rem - cl * nh, seg, cl};
+    const int a = rem - cl * nh;
+    return {bh, unit & ((1 << lognv) - 1), seg * L + cl, a, seg, cl, cl == 0 && a == 0, false, false};
+}
+
+// kBalanced: the units' chunks in order, unit by unit, cut into gridDim.x equal contiguous
+// ranges (each at least one unit long, so no range lies inside one unit), decoded once per
+// CTA.  A CTA first runs the head [0, c_hi) of the unit its range ends in (from zero; its
+// end state goes to the next CTA), then its whole units, then the tail [c_lo, N) of the
+// unit its range starts in, from the state the previous CTA handed over at the start of
+// its own run (long before).
+struct BalRange {
+    int u_lo, c_lo, u_hi, c_hi, u_first, n_full, G;
+};
+__device__ __forceinline__ BalRange bal_range(int N, int n_units) {
+    const long long tot = static_cast<long long>(n_units) * N;
+    const long long lo = tot * blockIdx.x / gridDim.x, hi = tot * (blockIdx.x + 1) / gridDim.x;
+    BalRange r;
+    r.u_lo = static_cast<int>(lo / N);
+    r.c_lo = static_cast<int>(lo - static_cast<long long>(r.u_lo) * N);
+    r.u_hi = static_cast<int>(hi / N);
+    r.c_hi = static_cast<int>(hi - static_cast<long long>(r.u_hi) * N);
+    r.u_first = r.c_lo ? r.u_lo + 1 : r.u_lo;
+    r.n_full = (r.u_hi - r.u_first) * N;
+    r.G = static_cast<int>(hi - lo);
+    return r;
+}
+__device__ __forceinline__ StreamPos stream_pos_bal(int v, int N, int lognv, const BalRange &r) {
+    int unit, c;
+    bool start, hin = false, hout = false;
+    if (v < r.c_hi) {
+        unit = r.u_hi;
+        c = v;
+        start = v == 0;
+        hout = v == r.c_hi - 1;
+    } else if (v - r.c_hi < r.n_full) {
+        const int w = v - r.c_hi, k = w / N;
+        unit = r.u_first + k;
+        c = w - k * N;
+        start = c == 0;
+    } else {
+        const int w = v - r.c_hi - r.n_full;
+        unit = r.u_lo;
+        c = r.c_lo + w;
+        start = hin = w == 0;
+    }
+    return {unit >> lognv, unit & ((1 << lognv) - 1), c, 0, 0, c, start, hin, hout};
 }
 
 // Visit the TMA load boxes of one chunk: calls f(map height index, smem row, c2, c3).
@@ -441,7 +499,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     // the state folded from the segment summaries).  MODE kSummary: per segment only
     // the end state from zero and the total decay (k, v and gates; no scores or outputs).
     constexpr bool kSum = MODE == kSummary;
-    constexpr bool kSplit = MODE != kFull;
+    constexpr bool kSplit = MODE == kSplitFull || MODE == kSummary;
+    constexpr bool kBal = MODE == kBalanced;
+    static_assert(!kBal || NH == 1, "balanced ranges hand over one key half's state");
     // GENOUT (one key half, outputs): the gen warpgroup that built a chunk also reads its
     // outputs back from TMEM and stores them, while it waits for the P of its next chunk,
     // which takes that work off the epi's serial per-chunk chain.  The host selects it where
@@ -455,9 +515,16 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     // this CTA's stream of virtual chunks: every barrier phase, stage slot and TMEM
     // buffer below follows the stream index (O: the real chunk's index), so
     // consecutive units flow through one pipeline
-    const int G = L * nh *
-                  ((p.n_units - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
-                   static_cast<int>(gridDim.x));
+    BalRange br{};
+    if constexpr (kBal) br = bal_range(N, p.n_units);
+    const int G = kBal ? br.G
+                       : L * nh *
+                             ((p.n_units - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
+                              static_cast<int>(gridDim.x));
+    auto pos = [&](int v) -> StreamPos {
+        if constexpr (kBal) return stream_pos_bal(v, N, lognv, br);
+        else return stream_pos(v, L, nh, lognv, kSplit ? p.nsu : 1);
+    };
     const int rev = p.order & 1;
 
     if (threadIdx.x == 0) {
@@ -512,7 +579,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             int issued = 0;
             for (int g = 0; g < G; ++g) {
                 const int sl = g % kSlots;
-                const StreamPos ps = stream_pos(g, L, nh, lognv, kSplit ? p.nsu : 1);
+                const StreamPos ps = pos(g);
                 const int b = ps.bh / p.H, h = ps.bh % p.H, c = ps.c;
                 const int xk = 64 * ps.a, xv = 64 * ps.vb;  // channel offsets of the key half, value slice
                 if (!mbar_wait(&bars[BAR_EMPTY + sl], ((g / kSlots) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
@@ -669,7 +736,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             uint32_t ow[16];
 #pragma unroll
             for (int j = 0; j < 16; ++j) ow[j] = Elem<E>::pack(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
-            const StreamPos po = stream_pos(co, L, nh, lognv, kSplit ? p.nsu : 1);
+            const StreamPos po = pos(co);
             const int b = po.bh / p.H, h = po.bh % p.H;
             const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
             if (t >= 0) {  // the row's columns inside Dv (padded columns stay behind)
@@ -885,9 +952,36 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             if (c < G) {
                 const int sl = c % kSlots, bb = c & 1;
                 const uint32_t ph = (c >> 1) & 1;
-                const StreamPos ps = stream_pos(c, L, nh, lognv, kSplit ? p.nsu : 1);
-                if (ps.cl == 0 && ps.a == 0) {  // a unit starts: its state (every key half)
-                    if (!kSplit || kSum || ps.seg == 0) {
+                const StreamPos ps = pos(c);
+                if (ps.start) {  // a run of a unit starts: its state (every key half)
+                    if (kBal && ps.hin) {
+                        // the previous CTA's hand-off (a bounded wait on its flag), then the flag
+                        // is cleared for the next launch
+                        const volatile unsigned long long *f = p.flags + blockIdx.x - 1;
+                        bool got = *f == p.epoch;
+                        const uint64_t t0 = global_timer_ns();
+                        while (!got && !*abort_flag && global_timer_ns() - t0 < kWaitLimitNs) {
+                            __nanosleep(64);
+                            got = *f == p.epoch;
+                        }
+                        if (named_barrier_or(3, 128, !got)) {  // the epi gives up together
+                            ok = false;
+                            break;
+                        }
+                        __threadfence();
+                        const float4 *x = reinterpret_cast<const float4 *>(p.summary + (size_t)(blockIdx.x - 1) * kD * kD +
+                                                                           (size_t)row * kD + ch0);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) {
+                            const float4 w = x[j];
+                            S[4 * j] = w.x;
+                            S[4 * j + 1] = w.y;
+                            S[4 * j + 2] = w.z;
+                            S[4 * j + 3] = w.w;
+                        }
+                        named_barrier_sync(3, 128);  // the epi's four warps read their rows
+                        if (threadIdx.x == 10 * 32) *const_cast<volatile unsigned long long *>(f) = 0ull;
+                    } else if (!kSplit || kSum || ps.seg == 0) {
 #pragma unroll
                         for (int j = 0; j < 32; ++j) S[j] = 0.f;
                         if constexpr (NH == 2) {
@@ -960,6 +1054,14 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
                         if (ps.vb == 0 && hc == 0) base[(size_t)kDk * kDv + 64 * ps.a + row] = dp;
                     }
+                } else if (kBal && ps.hout) {  // the state at the end of the head run -> the next CTA
+                    float4 *dst = reinterpret_cast<float4 *>(p.summary + (size_t)blockIdx.x * kD * kD + (size_t)row * kD + ch0);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
+                    __threadfence();
+                    named_barrier_sync(3, 128);  // the epi's four warps wrote their rows
+                    if (threadIdx.x == 10 * 32)
+                        *reinterpret_cast<volatile unsigned long long *>(p.flags + blockIdx.x) = p.epoch;
                 } else if (ps.c == N - 1 && p.final_state != nullptr && 64 * ps.a + row < p.Dk) {
                     // the sequence's final state [Dk][Dv] (padded channels and columns stay behind)
                     const int col0 = 64 * ps.vb + ch0;
@@ -1001,7 +1103,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     for (int j = 0; j < 8; ++j) ow[8 * hf + j] = Elem<E>::pack(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
                 }
                 tc_fence_before();
-                const StreamPos po = stream_pos(co, L, nh, lognv, kSplit ? p.nsu : 1);
+                const StreamPos po = pos(co);
                 const int b = po.bh / p.H, h = po.bh % p.H;
                 const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
                 if (t >= 0) {  // the row's columns inside Dv (padded columns stay behind)
@@ -1147,6 +1249,44 @@ cudaError_t launch_shape(dim3 grid, const TcParams &tp, cudaStream_t stream, boo
     return tp.nv == 1 ? launch_kernel<E, 2, 1, MODE>(grid, tp, stream) : launch_kernel<E, 2, 2, MODE>(grid, tp, stream);
 }
 
+// kBalanced CTAs wait for their neighbour's hand-off: a cooperative launch guarantees
+// that every CTA of the grid is resident at once.
+template <typename E, int NV>
+cudaError_t launch_balanced(dim3 grid, const TcParams &tp, cudaStream_t stream) {
+    static std::atomic<unsigned long long> set_on_devices(0);
+    auto kernel = gla_tc_kernel<E, 1, NV, kBalanced, false>;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const unsigned long long bit = 1ull << (dev & 63);
+    if (!(set_on_devices.load(std::memory_order_relaxed) & bit)) {
+        e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e != cudaSuccess) return e;
+        set_on_devices.fetch_or(bit);
+    }
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeCooperative;
+    attr.val.cooperative = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = stream;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, tp);
+}
+
+// Launch epochs of the balanced schedule: nonzero and never repeated within a process,
+// so a flag left by an earlier launch (or garbage in a fresh workspace) is not taken for
+// this launch's hand-off; flags are also cleared once read, which keeps graph replays of
+// one captured launch correct.
+unsigned long long next_epoch() {
+    static std::atomic<unsigned long long> ctr(
+        (static_cast<unsigned long long>(std::chrono::steady_clock::now().time_since_epoch().count()) << 16) | 1ull);
+    return ctr.fetch_add(2ull);  // odd, so never 0
+}
+
 cudaError_t sm_count(int *n_sm) {  // cached per device
     static std::atomic<int> cache[64] = {};
     int dev = 0;
@@ -1204,6 +1344,26 @@ Split choose_split(const Problem &p, int n_sm) {
     return best;
 }
 
+// Balanced ranges (one key half, unsplit): when the units are more than the SMs and a
+// round-robin deal would take at least 1.25 times the chunks per CTA of an even split,
+// every CTA takes an equal contiguous range of chunks instead.  Measured on a GB300
+// (graph-replayed, interleaved): B = 16, H = 12, 80 x 80, bf16 (192 units, ratio 1.58)
+// ran 1.23x faster balanced; B = 32, H = 12, 40 x 40 (384 units, ratio 1.19) 3 % slower
+// in bf16 and 4 % faster in fp16.  Units scattered over the CTAs cost about 8 % by
+// themselves (neighbouring CTAs no longer read the same token rows at the same time).
+bool choose_balanced(const Problem &p, int n_sm) {
+    if (pad64(p.Dk) != 64) return false;
+    const long long units = (long long)p.B * p.H * (pad64(p.Dv) / 64);
+    if (units <= n_sm) return false;
+    const long long waves = (units + n_sm - 1) / n_sm;
+    return waves * n_sm * 4 >= units * 5;  // ceil(U / SMs) >= 1.25 U / SMs
+}
+
+// hand-off states ([64][64] fp32 per CTA) and flags (one 64-bit word per CTA)
+size_t handoff_bytes(int n_sm) {
+    return (size_t)n_sm * 64 * 64 * sizeof(float) + (size_t)n_sm * sizeof(unsigned long long);
+}
+
 size_t summary_bytes(const Problem &p, int nseg) {
     if (nseg <= 1) return 0;
     return (size_t)p.B * p.H * (nseg - 1) * ((size_t)pad64(p.Dk) * pad64(p.Dv) + pad64(p.Dk)) * sizeof(float);
@@ -1234,8 +1394,12 @@ void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len) {
 size_t tc_workspace_bytes(const Problem &p) {
     int n_sm = 0;
     if (sm_count(&n_sm) != cudaSuccess) return 0;
-    return summary_bytes(p, choose_split(p, n_sm).nseg);
+    const int nseg = choose_split(p, n_sm).nseg;
+    if (nseg > 1) return summary_bytes(p, nseg);
+    return choose_balanced(p, n_sm) ? handoff_bytes(n_sm) : 0;
 }
+
+int tc_balanced_plan(const Problem &p, int n_sm) { return choose_split(p, n_sm).nseg == 1 && choose_balanced(p, n_sm); }
 
 bool tc_supported(const Problem &p) {
     if (p.dtype != 1 && p.dtype != 2) return false;       // fp16 / bf16 operands only
@@ -1270,6 +1434,8 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     tp.nseg = nseg;
     tp.seg_len = sp.len;
     tp.summary = static_cast<float *>(workspace);
+    tp.flags = nullptr;
+    tp.epoch = 0;
     // test hook for the timeout path (no fault: the data of one chunk simply never arrives)
     const char *drop = std::getenv("GTR_GLA_TEST_DROP_LOAD");
     tp.drop_load = (drop != nullptr && drop[0] == '1') ? 1 : 0;
@@ -1286,6 +1452,19 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     }
     tp.nsu = nseg;
     tp.n_units = seqs * nseg;
+    if (nseg == 1 && choose_balanced(p, n_sm) && workspace != nullptr && workspace_bytes >= handoff_bytes(n_sm)) {
+        // equal contiguous chunk ranges, one CTA per SM
+        tp.flags = reinterpret_cast<unsigned long long *>(static_cast<char *>(workspace) + (size_t)n_sm * 64 * 64 * sizeof(float));
+        tp.epoch = next_epoch();
+        const dim3 bgrid(static_cast<unsigned>(n_sm));
+        if (half)
+            e = tp.nv == 1 ? launch_balanced<__half, 1>(bgrid, tp, stream) : launch_balanced<__half, 2>(bgrid, tp, stream);
+        else
+            e = tp.nv == 1 ? launch_balanced<__nv_bfloat16, 1>(bgrid, tp, stream)
+                           : launch_balanced<__nv_bfloat16, 2>(bgrid, tp, stream);
+        if (e != cudaSuccess) return e;
+        return cudaGetLastError();
+    }
     const dim3 grid(static_cast<unsigned>(tp.n_units < n_sm ? tp.n_units : n_sm));
     // outputs from the gen warpgroups: fp16 launches of at most one wave (measured on a GB300:
     // +3 to +6 % there; with several units per CTA, or bf16, the epi storing them was faster)

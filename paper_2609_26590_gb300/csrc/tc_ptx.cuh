@@ -129,6 +129,13 @@ __device__ __forceinline__ void tma_load_5d(void *dst, const CUtensorMap *m, uin
         "r"(smem_u32(bar))
         : "memory");
 }
+// 5-D tiled prefetch global -> L2 (no shared memory, no completion to wait for).
+__device__ __forceinline__ void tma_prefetch_5d(const CUtensorMap *m, int c0, int c1, int c2, int c3, int c4) {
+    asm volatile("cp.async.bulk.prefetch.tensor.5d.L2.global.tile [%0, {%1, %2, %3, %4, %5}];" ::"l"(
+                     reinterpret_cast<uint64_t>(m)),
+                 "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4)
+                 : "memory");
+}
 // 5-D tiled store shared -> global (bulk async-group completion).
 __device__ __forceinline__ void tma_store_5d(const CUtensorMap *m, const void *src, int c0, int c1,
                                              int c2, int c3, int c4) {
@@ -258,6 +265,20 @@ __device__ __forceinline__ void tmem_ld_16x32bx2_x16(uint32_t taddr, uint32_t (&
 }
 __device__ __forceinline__ void tmem_ld_wait() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// ---------------------------------------------------------------- register budget
+// Per-warpgroup register limits (every warp of the warpgroup executes the same
+// instruction).  A decrease returns registers to the CTA's pool; an increase waits
+// until the pool holds them, so the limits of all warpgroups must add up to at most
+// the registers the block was launched with.
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+template <uint32_t N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
 }
 
 // ---------------------------------------------------------------- descriptors

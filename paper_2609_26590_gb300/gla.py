@@ -61,6 +61,8 @@ def load(path: Optional[str] = None):
         lib.gtr_gla_chunk_boxes.argtypes = [ci] * 4 + [ctypes.POINTER(ci), ci]
         lib.gtr_gla_split_plan.restype = ci
         lib.gtr_gla_split_plan.argtypes = [ci] * 7 + [ctypes.POINTER(ci)] * 2
+        lib.gtr_gla_balanced_plan.restype = ci
+        lib.gtr_gla_balanced_plan.argtypes = [ci] * 7
         lib.gtr_gla_fwd_ws.restype = ci
         lib.gtr_gla_fwd_ws.argtypes = [vp] * 4 + [ci] * 8 + [vp, vp, vp, st, vp]
         lib.gtr_gla_fwd_gated.restype = ci
@@ -161,6 +163,13 @@ def split_plan(B: int, H: int, grid_h: int, grid_w: int, Dk: int, Dv: int, n_sm:
                                     ctypes.byref(seg_len))
     _check(status, "gtr_gla_split_plan", lib)
     return nseg.value, seg_len.value
+
+
+def balanced_plan(B: int, H: int, grid_h: int, grid_w: int, Dk: int, Dv: int, n_sm: int) -> bool:
+    """Whether the tensor-core schedule gives every CTA an equal contiguous range of
+    chunks on a device with ``n_sm`` SMs, through ``gtr_gla_balanced_plan`` (host
+    arithmetic only)."""
+    return bool(load().gtr_gla_balanced_plan(B, H, grid_h, grid_w, Dk, Dv, n_sm))
 
 
 def sswiglu_dwconv(gate: torch.Tensor, value: torch.Tensor, weight: torch.Tensor, bias: Optional[torch.Tensor],

@@ -316,14 +316,73 @@ def test_explicit_schedule_rejects_unsupported():
 
 
 def test_workspace_matches_split_plan():
-    """The summaries the schedule allocates are those of the split gtr_gla_split_plan
-    reports for this device's SM count: (segments - 1) per sequence of padded
-    (Dk x Dv + Dk) floats."""
+    """The workspace the schedule asks for is that of the plan gtr_gla_split_plan and
+    gtr_gla_balanced_plan report for this device's SM count: (segments - 1) per
+    sequence of padded (Dk x Dv + Dk) floats for a split, one 64 x 64 fp32 state and
+    one 64-bit flag per SM for balanced ranges, else nothing."""
     n_sm = torch.cuda.get_device_properties(0).multi_processor_count
     pad = lambda d: (d + 63) // 64 * 64
     for B, H, gh, gw, Dk, Dv in [(1, 6, 40, 40, 64, 64), (1, 6, 44, 44, 64, 64), (2, 8, 128, 128, 128, 128),
-                                 (32, 12, 40, 40, 64, 64), (1, 3, 40, 36, 32, 64), (1, 1, 16, 20, 64, 64)]:
+                                 (32, 12, 40, 40, 64, 64), (1, 3, 40, 36, 32, 64), (1, 1, 16, 20, 64, 64),
+                                 (8, 16, 80, 80, 64, 64), (1, 160, 8, 16, 64, 64)]:
         nseg, seg_len = gla.split_plan(B, H, gh, gw, Dk, Dv, n_sm)
-        expect = 0 if nseg == 1 else B * H * (nseg - 1) * (pad(Dk) * pad(Dv) + pad(Dk)) * 4
+        bal = gla.balanced_plan(B, H, gh, gw, Dk, Dv, n_sm)
+        assert not (bal and nseg > 1)
+        if nseg > 1:
+            expect = B * H * (nseg - 1) * (pad(Dk) * pad(Dv) + pad(Dk)) * 4
+        else:
+            expect = n_sm * (64 * 64 * 4 + 8) if bal else 0
         for dt in (torch.float16, torch.bfloat16):
-            assert gla.workspace_bytes(B, H, gh, gw, Dk, Dv, dt) == expect, (B, H, gh, gw, Dk, Dv, nseg, seg_len)
+            assert gla.workspace_bytes(B, H, gh, gw, Dk, Dv, dt) == expect, (B, H, gh, gw, Dk, Dv, nseg, seg_len, bal)
+
+
+# More (sequence, value slice) units than SMs, not a multiple of them: the tensor-core
+# schedule gives every CTA an equal contiguous range of chunks, and a unit cut by a range
+# boundary continues on the next CTA from the state handed over through the workspace
+# (its end state after the head of the range before).  H is set from the device's SM
+# count so that the units exceed it by a few; (Dv, dtype, grid_h, grid_w, extra units).
+BALANCED = [(64, "bf16", 8, 16, 8), (64, "f16", 24, 8, 40), (128, "bf16", 16, 12, 10), (32, "f16", 5, 13, 3)]
+
+
+@pytest.mark.parametrize("case", BALANCED, ids=[f"dv{c[0]}_{c[1]}-{c[2]}x{c[3]}+{c[4]}" for c in BALANCED])
+def test_balanced_ranges(case):
+    Dv, dtype, gh, gw, extra = case
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    nv = (Dv + 63) // 64
+    H = (n_sm + extra + nv - 1) // nv
+    B, Dk = 1, 64
+    assert gla.balanced_plan(B, H, gh, gw, Dk, Dv, n_sm), "the schedule should balance these units"
+    ws_bytes = gla.workspace_bytes(B, H, gh, gw, Dk, Dv, TORCH_DT[dtype])
+    assert ws_bytes == n_sm * (64 * 64 * 4 + 8)
+    inp = wl.make_inputs(B, H, gh, gw, Dk, Dv, dtype, seed=7100 + BALANCED.index(case))
+    f = inputs_f64(inp, dtype)
+    t = {n: to_torch(inp[n], dtype) for n in ("q", "k", "v", "g")}
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device="cuda")
+    for order in wl.ALL_ORDERS:
+        ref_o, ref_s = oracle.recurrence(f["q"], f["k"], f["v"], f["g"], gh, gw, order)
+        out, fs = _run(inp, dtype, gh, gw, order, "tc")  # internal workspace
+        assert_within_bar(_np(out), ref_o, dtype, f"out order {order}")
+        assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, dtype, f"state {order}")
+        for rep in range(2):  # a caller workspace twice: flags of the call before are not taken
+            out2, fs2 = torch.empty_like(t["v"]), torch.empty_like(fs)
+            gla.forward_ws(t["q"], t["k"], t["v"], t["g"], gh, gw, order, out2, fs2, ws)
+            torch.cuda.synchronize()
+            assert gla.sync_status() == 0
+            assert torch.equal(out2, out) and torch.equal(fs2, fs)  # same schedule, same bits
+    # one captured launch replayed: each replay hands its states over afresh
+    order = wl.COL_REV
+    out_ref, fs_ref = _run(inp, dtype, gh, gw, order, "tc")
+    out3, fs3 = torch.empty_like(t["v"]), torch.empty_like(fs_ref)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(g, stream=side):
+            gla.forward_ws(t["q"], t["k"], t["v"], t["g"], gh, gw, order, out3, fs3, ws, stream=side)
+    torch.cuda.current_stream().wait_stream(side)
+    for rep in range(3):
+        out3.zero_()
+        g.replay()
+        torch.cuda.synchronize()
+        assert gla.sync_status() == 0
+        assert torch.equal(out3, out_ref) and torch.equal(fs3, fs_ref)
