@@ -56,6 +56,8 @@ def parse():
                     help="mixer: the chunkwise GLA token mixer (default); sswiglu: the Spatial SwiGLU "
                          "gate-and-depthwise-conv step (Eq. spatial_swiglu) on --sw-workload")
     ap.add_argument("--sw-workload", type=int, default=2)
+    ap.add_argument("--no-secondary", action="store_true",
+                    help="skip the 6400-token workload the default run also times")
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch size (smaller cases for profiling)")
     return ap.parse_args()
@@ -98,13 +100,43 @@ def load_peaks():
     return FALLBACK_HBM_GBS, "fallback"
 
 
-def workload_config(w: wl.Workload, world: int, extra=None):
+# GB300 L2 size.  The buffer-rotation plan below is computed from this constant in
+# both arms, so that they print the same config; the GPU arm also records the size
+# the device reports.
+L2_NOMINAL_BYTES = 129_000_000
+
+
+def rotation_sets(step_bytes: int) -> int:
+    """Input/output buffer sets a timed loop rotates through: enough that their
+    total exceeds twice the L2 size, so that every step reads its inputs from HBM
+    rather than from the L2 copy the previous step left behind."""
+    if step_bytes >= 2 * L2_NOMINAL_BYTES:
+        return 1
+    return -(-2 * L2_NOMINAL_BYTES // step_bytes)
+
+
+def l2_note(w: wl.Workload, n_sets: int) -> str:
+    mb = w.algorithmic_bytes() / 1e6
+    if n_sets == 1:
+        return "inputs larger than L2 (%.0f MB per step > 2 x 129 MB)" % mb
+    return ("rotating %d input/output buffer sets (%.2f MB per step, %.0f MB in all > 2 x 129 MB L2)"
+            % (n_sets, mb, n_sets * mb))
+
+
+def workload_config(w: wl.Workload, world: int, args=None, extra=None):
+    """The `config` object of a JSON line; both arms print the same keys and values
+    for the same command-line arguments."""
     cfg = {"workload": w.name, "B": w.B, "H": w.H, "grid": [w.grid_h, w.grid_w], "T": w.T,
            "Dk": w.Dk, "Dv": w.Dv, "tokens_per_step_per_gpu": w.B * w.T,
            "scan_orders": "alternating " + "/".join(wl.ORDER_NAMES[o] for o in w.orders),
            "final_state": w.final_state,
-           "l2": "inputs larger than L2 (%.0f MB per step > 129 MB)" % (w.algorithmic_bytes() / 1e6),
+           "l2": l2_note(w, rotation_sets(w.algorithmic_bytes())),
            "parallelism": f"replicas x{world} (independent batches, no collective)"}
+    if args is not None:
+        cfg["schedule"] = args.schedule
+        cfg["launch"] = "cuda-graph replay" if args.graph else "eager"
+        if args.gated:
+            cfg["epilogue"] = "output gate u = SiLU(r) * RMSNorm(o), second kernel right after the mixer"
     if extra:
         cfg.update(extra)
     return cfg
@@ -230,7 +262,8 @@ def run_reference(args, w: wl.Workload, rank: int, world: int):
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": per_step * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded, workload recipe)",
-            "config": workload_config(w, 1, {"reference": "fp64 CPU oracle (oracle/), as it stands"}),
+            "config": workload_config(w, world, args),
+            "reference": "fp64 CPU oracle (oracle/), as it stands",
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": oracle.max_threads(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
@@ -360,6 +393,264 @@ def run_sswiglu(args, rank: int, world: int, local: int):
           flush=True)
 
 
+def to_device(a: np.ndarray, dtype: str, dev):
+    import torch
+    if dtype == "bf16":
+        return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(dev)
+    return torch.from_numpy(a).to(dev)
+
+
+def device_l2_bytes(dev) -> int:
+    import torch
+    return int(getattr(torch.cuda.get_device_properties(dev), "L2_cache_size", 0))
+
+
+def mixer_sets(w: wl.Workload, inp, dev, n_sets: int, gated: bool, seed: int):
+    """n_sets device copies of the step's inputs and outputs (the same values at
+    different addresses); the timed loop rotates through them."""
+    import torch
+    base = {n: to_device(inp[n], w.dtype, dev) for n in ("q", "k", "v", "g")}
+    extra = {}
+    if gated:
+        rng = np.random.Generator(np.random.PCG64(seed + 17))
+        extra["r"] = to_device(wl.round_to_storage(rng.standard_normal((w.B, w.T, w.H, w.Dv)) * 1.5, w.dtype),
+                               w.dtype, dev)
+        extra["w"] = torch.from_numpy((1.0 + 0.2 * rng.standard_normal(w.Dv)).astype(np.float32)).to(dev)
+    sets = []
+    for j in range(n_sets):
+        s = {n: (t if j == 0 else t.clone()) for n, t in base.items()}
+        if gated:
+            s["r"] = extra["r"] if j == 0 else extra["r"].clone()
+            s["w"] = extra["w"]
+        s["out"] = torch.empty_like(s["v"])
+        s["fs"] = (torch.empty((w.B, w.H, w.Dk, w.Dv), dtype=torch.float32, device=dev)
+                   if w.final_state else None)
+        sets.append(s)
+    return sets
+
+
+def timed_loop(run, steps: int, stream, clocks_enabled: bool, local: int, pg=None):
+    """Time `steps` calls of run(i) on `stream` with CUDA events (one pair per step and
+    one around the loop), bracketed by a barrier and a synchronize on both sides;
+    nvidia-smi clocks are sampled during the loop."""
+    import torch
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local, enabled=clocks_enabled) as clk:
+        t_begin = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_begin.record(stream)
+        for i in range(steps):
+            starts[i].record(stream)
+            run(i)
+            ends[i].record(stream)
+        t_end.record(stream)
+        torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    per_launch = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    return t_begin.elapsed_time(t_end), per_launch, clk.summary()
+
+
+TORCH_DT_NAMES = {"f32": "float32", "f16": "float16", "bf16": "bfloat16"}
+SECONDARY_WORKLOAD = 3   # the 6400-token workload, timed after the headline in the same run
+
+
+def time_mixer(args, w: wl.Workload, rank: int, world: int, local: int, dev, pg):
+    """Device-resident timing of one mixer workload: warm-up, `args.steps` timed steps
+    rotating through enough buffer sets to defeat the L2, the roofline of the step's
+    kernel(s) and the clocks seen.  Returns a dict (the sets and host inputs stay in it
+    for the end-to-end leg)."""
+    import math
+
+    import torch
+    from paper_2609_26590_gb300 import gla
+
+    dt = getattr(torch, TORCH_DT_NAMES[w.dtype])
+    seed = rank_seed(w, rank)
+    inp = wl.workload_inputs(w, B=w.B, seed=seed)
+    n_sets = rotation_sets(w.algorithmic_bytes())
+    sets = mixer_sets(w, inp, dev, n_sets, args.gated, seed)
+    stream = torch.cuda.current_stream(dev)
+    orders = w.orders
+    schedule = args.schedule
+    tc = gla.tc_supported(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, orders[0], dt)
+    kernel_name = "tensor-core chunkwise (tcgen05/TMEM/TMA)" if (tc and schedule != "simt") else "simt recurrence"
+    ws_n = gla.workspace_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt) if tc and schedule != "simt" else 0
+    split = ws_n > 0 and gla.split_plan(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv,
+                                         torch.cuda.get_device_properties(dev).multi_processor_count)[0] > 1
+    launches_per_step = 2 if split else 1
+    if split:
+        kernel_name += ", segment-summary pass + output pass"
+    if args.gated:  # the output gate runs as one more kernel right after the mixer
+        launches_per_step += 1
+        kernel_name += " + output-gate kernel"
+
+    def call(s, order, strm=None, ws=None, graph=False):
+        if args.gated:
+            gla.forward_gated(s["q"], s["k"], s["v"], s["g"], s["r"], s["w"], 1e-5, w.grid_h, w.grid_w, order,
+                              out=s["out"], final_state=s["fs"], stream=strm, workspace=ws)
+        elif graph:
+            gla.forward_ws(s["q"], s["k"], s["v"], s["g"], w.grid_h, w.grid_w, order, s["out"], s["fs"], ws,
+                           stream=strm)
+        else:
+            gla.forward(s["q"], s["k"], s["v"], s["g"], w.grid_h, w.grid_w, order, out=s["out"],
+                        final_state=s["fs"], schedule=schedule)
+
+    def step(i):
+        call(sets[i % n_sets], orders[i % len(orders)])
+
+    for i in range(max(3, args.warmup)):
+        step(i)
+    torch.cuda.synchronize()
+    if gla.sync_status() != 0:
+        raise RuntimeError("device status word set during warm-up")
+
+    run = step
+    if args.graph:
+        # one graph per (buffer set, scan order) pair of the rotation, captured through the
+        # caller-workspace entry points (no allocation, no synchronisation)
+        if schedule != "auto":
+            raise SystemExit("--graph times the automatic schedule only")
+        ws = torch.empty(ws_n, dtype=torch.uint8, device=dev) if ws_n else None
+        n_graph = n_sets * len(orders) // math.gcd(n_sets, len(orders))
+        cap = torch.cuda.Stream(dev)
+        cap.wait_stream(stream)
+        graphs = []
+        with torch.cuda.stream(cap):
+            for j in range(n_graph):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=cap):
+                    call(sets[j % n_sets], orders[j % len(orders)], strm=cap, ws=ws, graph=True)
+                graphs.append(g)
+        stream.wait_stream(cap)
+        for j in range(max(3, args.warmup)):
+            graphs[j % n_graph].replay()
+        torch.cuda.synchronize()
+        if gla.sync_status() != 0:
+            raise RuntimeError("device status word set during graph warm-up")
+
+        def run(i):
+            graphs[i % n_graph].replay()
+
+    total_ms, per_launch_ms, clocks = timed_loop(run, args.steps, stream, not args.no_clocks, local, pg)
+    if gla.sync_status() != 0:
+        raise RuntimeError("device status word set during the timed region")
+    total_ms = max_over_ranks(total_ms, pg, dev)
+    ms_per_step = total_ms / args.steps
+    value = job_tokens_per_s(w.B * w.T, world, ms_per_step)
+
+    hbm_peak, peak_src = load_peaks()
+    alg_bytes = w.algorithmic_bytes()
+    if args.gated:  # the gate's pre-activation is read once more per token-head (u replaces o)
+        alg_bytes += w.B * w.T * w.H * w.Dv * wl.ELEM_SIZE[w.dtype]
+    kernel_ms = sum(per_launch_ms) / len(per_launch_ms)
+    achieved = alg_bytes / (kernel_ms * 1e-3) / 1e9
+    traffic, traffic_note = None, None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath) and not args.gated and args.batch is None:
+        with open(tpath) as f:
+            tj = json.load(f)
+        entry = tj.get(f"{w.name}:{'tc' if (tc and schedule != 'simt') else 'simt'}")
+        if isinstance(entry, dict):
+            traffic, traffic_note = entry.get("dram_bytes"), entry.get("note")
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                "frac": achieved / hbm_peak, "traffic": traffic,
+                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback",
+                "kernel": kernel_name, "kernel_ms": kernel_ms, "algorithmic_bytes_per_launch": alg_bytes,
+                "timing": "CUDA events around each step on the launching stream"}
+    if traffic_note:
+        roofline["traffic_note"] = traffic_note
+    return {"w": w, "inp": inp, "sets": sets, "value": value, "ms_per_step": ms_per_step,
+            "roofline": roofline, "clocks": clocks, "launches": args.steps * launches_per_step,
+            "n_sets": n_sets, "dt": dt, "tc": tc}
+
+
+def time_e2e(args, res, world: int, dev, pg):
+    """End to end through gtr_gla_fwd_host: pinned host inputs in, outputs back to
+    pinned host memory, every step inside the timed region.  Beside it, the host
+    link's own rate: plain pinned copies of the same bytes, each direction alone and
+    both at once, so that the e2e number can be read against what the link gives."""
+    import torch
+    from paper_2609_26590_gb300 import gla
+
+    w, inp, dt = res["w"], res["inp"], res["dt"]
+    stream = torch.cuda.current_stream(dev)
+    orders = w.orders
+    host = {n: (torch.from_numpy(inp[n].view(np.int16)).view(torch.bfloat16) if w.dtype == "bf16"
+                else torch.from_numpy(inp[n])).pin_memory() for n in ("q", "k", "v", "g")}
+    hout = torch.empty(host["v"].shape, dtype=host["v"].dtype).pin_memory()
+    hfs = torch.empty((w.B, w.H, w.Dk, w.Dv), dtype=torch.float32).pin_memory() if w.final_state else None
+    nbytes = gla.host_buffer_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt, w.final_state)
+    dbuf = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    for i in range(2):
+        gla.forward_host(host["q"], host["k"], host["v"], host["g"], w.grid_h, w.grid_w,
+                         orders[i % len(orders)], hout, hfs, dbuf)
+    torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(args.e2e_steps):
+        gla.forward_host(host["q"], host["k"], host["v"], host["g"], w.grid_h, w.grid_w,
+                         orders[i % len(orders)], hout, hfs, dbuf)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if gla.sync_status() != 0:
+        raise RuntimeError("device status word set during the end-to-end leg")
+    e_ms = max_over_ranks(e0.elapsed_time(e1), pg, dev) / args.e2e_steps
+    h2d = sum(host[n].numel() * host[n].element_size() for n in ("q", "k", "v", "g"))
+    d2h = hout.numel() * hout.element_size() + (hfs.numel() * 4 if hfs is not None else 0)
+
+    # the link alone: one cudaMemcpyAsync per tensor (torch copy_ of pinned memory)
+    s0 = res["sets"][0]
+    dins = [s0[n] for n in ("q", "k", "v", "g")]
+    douts = [(hout, s0["out"])] + ([(hfs, s0["fs"])] if hfs is not None else [])
+    side = torch.cuda.Stream(dev)
+    reps = 3
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+
+    def up():
+        for d, n in zip(dins, ("q", "k", "v", "g")):
+            d.copy_(host[n], non_blocking=True)
+
+    def down():
+        for h, d in douts:
+            h.copy_(d, non_blocking=True)
+
+    def both():  # uploads on the launching stream, downloads on a second one at the same time
+        side.wait_stream(stream)
+        up()
+        with torch.cuda.stream(side):
+            down()
+        stream.wait_stream(side)
+
+    up_ms, down_ms, both_ms = timed(up), timed(down), timed(both)
+    tokens = w.B * w.T
+    return {"value": job_tokens_per_s(tokens, world, e_ms), "unit": "tokens/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e_ms,
+            "api": "gtr_gla_fwd_host (pinned host buffers)",
+            "link": {"e2e_gbs": (h2d + d2h) / (e_ms * 1e-3) / 1e9,
+                     "h2d_alone_gbs": h2d / (up_ms * 1e-3) / 1e9,
+                     "d2h_alone_gbs": d2h / (down_ms * 1e-3) / 1e9,
+                     "both_at_once_gbs": (h2d + d2h) / (both_ms * 1e-3) / 1e9,
+                     "copies_only_ms_per_step": both_ms,
+                     "how": "plain pinned cudaMemcpyAsync of the step's bytes, one per tensor, in the same run"}}
+
+
 def main():
     args = parse()
     rank, world, local = dist_env()
@@ -384,183 +675,45 @@ def main():
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
         pg = dist
-
     gla.load()
-    dt = {"f32": torch.float32, "f16": torch.float16, "bf16": torch.bfloat16}[w.dtype]
 
-    # inputs: rank r draws batch r of the workload (same distributions, own seed)
-    inp = wl.workload_inputs(w, B=w.B, seed=rank_seed(w, rank))
-
-    def to_dev(a):
-        if w.dtype == "bf16":
-            return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(dev)
-        return torch.from_numpy(a).to(dev)
-
-    t = {n: to_dev(inp[n]) for n in ("q", "k", "v", "g")}
-    out = torch.empty_like(t["v"])
-    fs = torch.empty((w.B, w.H, w.Dk, w.Dv), dtype=torch.float32, device=dev) if w.final_state else None
-    stream = torch.cuda.current_stream(dev)
-    orders = w.orders
-    schedule = args.schedule
-    tc = gla.tc_supported(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, orders[0], dt)
-    kernel_name = "tensor-core chunkwise (tcgen05/TMEM/TMA)" if (tc and schedule != "simt") else "simt recurrence"
-    # a split schedule runs a summary pass before the output pass: two launches a step
-    split = tc and schedule != "simt" and gla.workspace_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt) > 0
-    launches_per_step = 2 if split else 1
-    if split:
-        kernel_name += ", segment-summary pass + output pass"
-    if args.gated:  # the output gate runs as one more kernel right after the mixer
-        launches_per_step += 1
-        kernel_name += " + output-gate kernel"
-
-    if args.gated:
-        rng = np.random.Generator(np.random.PCG64(rank_seed(w, rank) + 17))
-        gate_r = to_dev(wl.round_to_storage(rng.standard_normal((w.B, w.T, w.H, w.Dv)) * 1.5, w.dtype))
-        gate_w = torch.from_numpy((1.0 + 0.2 * rng.standard_normal(w.Dv)).astype(np.float32)).to(dev)
-
-    def step(i):
-        if args.gated:
-            gla.forward_gated(t["q"], t["k"], t["v"], t["g"], gate_r, gate_w, 1e-5, w.grid_h, w.grid_w,
-                              orders[i % len(orders)], out=out, final_state=fs if fs is not None else None)
-        else:
-            gla.forward(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, orders[i % len(orders)],
-                        out=out, final_state=fs if fs is not None else None, schedule=schedule)
-
-    for i in range(max(3, args.warmup)):
-        step(i)
-    torch.cuda.synchronize()
-    if gla.sync_status() != 0:
-        raise RuntimeError("device status word set during warm-up")
-
-    run = step
-    if args.graph:
-        # one graph per scan order, captured through the caller-workspace entry points
-        # (no allocation, no synchronisation; the split schedule stays on)
-        if schedule != "auto":
-            raise SystemExit("--graph times the automatic schedule only")
-        ws_n = gla.workspace_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt)
-        ws = torch.empty(ws_n, dtype=torch.uint8, device=dev) if ws_n else None
-        cap = torch.cuda.Stream(dev)
-        cap.wait_stream(stream)
-        graphs = []
-        with torch.cuda.stream(cap):
-            for j in range(len(orders)):
-                g = torch.cuda.CUDAGraph()
-                with torch.cuda.graph(g, stream=cap):
-                    if args.gated:
-                        gla.forward_gated(t["q"], t["k"], t["v"], t["g"], gate_r, gate_w, 1e-5, w.grid_h,
-                                          w.grid_w, orders[j], out=out, final_state=fs, stream=cap, workspace=ws)
-                    else:
-                        gla.forward_ws(t["q"], t["k"], t["v"], t["g"], w.grid_h, w.grid_w, orders[j], out, fs, ws,
-                                       stream=cap)
-                graphs.append(g)
-        stream.wait_stream(cap)
-        for j in range(max(3, args.warmup)):
-            graphs[j % len(graphs)].replay()
-        torch.cuda.synchronize()
-        if gla.sync_status() != 0:
-            raise RuntimeError("device status word set during graph warm-up")
-
-        def run(i):
-            graphs[i % len(graphs)].replay()
-
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    if pg:
-        pg.barrier()
-    torch.cuda.synchronize()
-    with ClockSampler(local, enabled=not args.no_clocks) as clk:
-        t_begin = torch.cuda.Event(enable_timing=True)
-        t_end = torch.cuda.Event(enable_timing=True)
-        t_begin.record(stream)
-        for i in range(args.steps):
-            starts[i].record(stream)
-            run(i)
-            ends[i].record(stream)
-        t_end.record(stream)
-        torch.cuda.synchronize()
-    if pg:
-        pg.barrier()
-    total_ms = t_begin.elapsed_time(t_end)
-    per_launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    if gla.sync_status() != 0:
-        raise RuntimeError("device status word set during the timed region")
-    total_ms = max_over_ranks(total_ms, pg, dev)
-    ms_per_step = total_ms / args.steps
-    value = job_tokens_per_s(w.B * w.T, world, ms_per_step)
-
-    # roofline of the (single) kernel of a step
-    hbm_peak, peak_src = load_peaks()
-    alg_bytes = w.algorithmic_bytes()
-    if args.gated:  # the gate's pre-activation is read once more per token-head (u replaces o)
-        alg_bytes += w.B * w.T * w.H * w.Dv * wl.ELEM_SIZE[w.dtype]
-    kernel_ms = sum(per_launch_ms) / len(per_launch_ms)
-    achieved = alg_bytes / (kernel_ms * 1e-3) / 1e9
-    traffic = None
-    tpath = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tpath):
-        with open(tpath) as f:
-            tj = json.load(f)
-        key = f"{w.name}:{'tc' if (tc and schedule != 'simt') else 'simt'}"
-        traffic = tj.get(key)
-    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                "frac": achieved / hbm_peak, "traffic": traffic,
-                "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback",
-                "kernel": kernel_name, "kernel_ms": kernel_ms,
-                "algorithmic_bytes_per_launch": alg_bytes}
-
-    # end to end through the host-memory entry point (pinned host buffers)
-    e2e = None
-    if args.e2e_steps > 0 and not args.gated:
-        host = {n: (torch.from_numpy(inp[n].view(np.int16)).view(torch.bfloat16) if w.dtype == "bf16"
-                    else torch.from_numpy(inp[n])).pin_memory() for n in ("q", "k", "v", "g")}
-        hout = torch.empty(host["v"].shape, dtype=host["v"].dtype).pin_memory()
-        hfs = torch.empty((w.B, w.H, w.Dk, w.Dv), dtype=torch.float32).pin_memory() if w.final_state else None
-        nbytes = gla.host_buffer_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt, w.final_state)
-        dbuf = torch.empty(nbytes, dtype=torch.uint8, device=dev)
-        for i in range(2):
-            gla.forward_host(host["q"], host["k"], host["v"], host["g"], w.grid_h, w.grid_w,
-                             orders[i % len(orders)], hout, hfs, dbuf)
-        torch.cuda.synchronize()
-        if pg:
-            pg.barrier()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for i in range(args.e2e_steps):
-            gla.forward_host(host["q"], host["k"], host["v"], host["g"], w.grid_h, w.grid_w,
-                             orders[i % len(orders)], hout, hfs, dbuf)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        e_ms = e0.elapsed_time(e1)
-        e_ms = max_over_ranks(e_ms, pg, dev)
-        es = job_tokens_per_s(w.B * w.T, world, e_ms / args.e2e_steps)
-        h2d = sum(host[n].numel() * host[n].element_size() for n in ("q", "k", "v", "g"))
-        d2h = hout.numel() * hout.element_size() + (hfs.numel() * 4 if hfs is not None else 0)
-        e2e = {"value": es, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": e_ms / args.e2e_steps,
-               "api": "gtr_gla_fwd_host (pinned host buffers)"}
+    res = time_mixer(args, w, rank, world, local, dev, pg)
+    head = {k: res[k] for k in ("value", "ms_per_step", "roofline", "clocks", "launches")}
+    e2e = time_e2e(args, res, world, dev, pg) if args.e2e_steps > 0 and not args.gated else None
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        inp64 = {n: wl.storage_to_f64(inp[n], w.dtype) for n in ("q", "k", "v", "g")}
-        val, el, n_pairs, cores = time_oracle(w, inp64, orders[0], budget_s=10.0)
+        inp64 = {n: wl.storage_to_f64(res["inp"][n], w.dtype) for n in ("q", "k", "v", "g")}
+        val, el, n_pairs, cores = time_oracle(w, inp64, w.orders[0], budget_s=10.0)
         cpu = {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                "sample": f"{n_pairs} (b,h) sequences x {w.T} tokens ({el:.1f} s wall), "
-                         f"order {wl.ORDER_NAMES[orders[0]]}"}
+                         f"order {wl.ORDER_NAMES[w.orders[0]]}"}
+        del inp64
 
+    secondary = None
+    if (args.workload == DEFAULT_WORKLOAD and args.batch is None and not args.gated and not args.no_secondary
+            and args.schedule == "auto"):
+        # the 6400-token workload in the same run (the second length of the target)
+        del res
+        torch.cuda.empty_cache()
+        w2 = wl.WORKLOADS[SECONDARY_WORKLOAD]
+        r2 = time_mixer(args, w2, rank, world, local, dev, pg)
+        secondary = {"workload": w2.name, "metric": "GLA-forward tokens/s (GB300, device-timed) and % of roofline "
+                                                    "at 6400 tokens",
+                     "value": r2["value"], "unit": "tokens/s", "ms_per_step": r2["ms_per_step"],
+                     "steps": args.steps, "dtype": w2.dtype, "roofline": r2["roofline"], "clocks": r2["clocks"],
+                     "gpu_launches": r2["launches"],
+                     "config": workload_config(w2, world, args), "token_heads_per_s": r2["value"] * w2.H}
     if rank == 0:
-        line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
-                "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        line = {"metric": METRIC, "value": head["value"], "unit": "tokens/s", "n_gpus": world,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": head["ms_per_step"],
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
                 "dtype": w.dtype, "data": "synthetic (seeded, workload recipe in workloads.py)",
-                "config": workload_config(w, world, dict({"schedule": schedule,
-                                                          "launch": "cuda-graph replay" if args.graph else "eager"},
-                                                         **({"epilogue": "output gate u = SiLU(r) * RMSNorm(o), "
-                                                             "second kernel right after the mixer"}
-                                                            if args.gated else {}))),
-                "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-                "gpu_launches": args.steps * launches_per_step, "clocks": clk.summary(),
-                "token_heads_per_s": value * w.H}
+                "config": workload_config(w, world, args),
+                "roofline": head["roofline"], "cpu_baseline": cpu, "e2e": e2e,
+                "gpu_launches": head["launches"], "clocks": head["clocks"],
+                "token_heads_per_s": head["value"] * w.H, "l2_device_bytes": device_l2_bytes(dev),
+                "secondary": secondary}
         print(json.dumps(line), flush=True)
     if pg:
         pg.destroy_process_group()

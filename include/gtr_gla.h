@@ -48,8 +48,19 @@
  *     Launch failures return GTR_ERR_CUDA.  Conditions the device detects
  *     (a bounded wait that gave up) are recorded in a per-device status word
  *     and reported by gtr_gla_sync_status().
- *   - No call allocates device memory, synchronises, or reads device data on
- *     the host, so gtr_gla_fwd can be captured in a CUDA graph.
+ *   - Allocation and synchronisation: gtr_gla_fwd, gtr_gla_fwd_sched and
+ *     gtr_gla_fwd_gated keep an internal per-device workspace for the split
+ *     and balanced schedules.  The first call that needs it, and any later
+ *     call that needs more, allocates it with cudaMalloc (and frees the
+ *     smaller one with cudaFree, which synchronises the device); calls made
+ *     while their stream is being captured never touch it and run the
+ *     round-robin schedule instead (gtr_gla_last_schedule reports both the
+ *     schedule that ran and the one that was planned).  gtr_gla_fwd_host
+ *     creates two streams and a set of events on its first call per device.
+ *     Every other entry point allocates no device memory and does not
+ *     synchronise: the _ws and _noalloc forms are the ones to capture in a
+ *     CUDA graph with every schedule.  No entry point reads device data on the
+ *     host except gtr_gla_sync_status.
  */
 #ifndef GTR_GLA_H
 #define GTR_GLA_H
@@ -97,8 +108,9 @@ typedef enum { GTR_SCHED_AUTO = 0, GTR_SCHED_SIMT = 1, GTR_SCHED_TC = 2 } gtr_sc
  * across segments).  Those summaries live in an internal per-device workspace
  * that this call allocates (cudaMalloc) the first time a problem needs it and
  * grows outside stream capture; under capture the call never touches it and
- * runs the schedule unsplit.  Callers that manage memory themselves use
- * gtr_gla_fwd_ws. */
+ * runs the schedule unsplit (gtr_gla_last_schedule then reports GTR_RAN_TC
+ * against a planned GTR_RAN_TC_SPLIT).  Callers that manage memory themselves
+ * use gtr_gla_fwd_ws. */
 gtr_status_t gtr_gla_fwd(const void *q, const void *k, const void *v, const void *log_gate,
                          int B, int H, int grid_h, int grid_w, int Dk, int Dv,
                          gtr_scan_t scan_order, gtr_dtype_t dtype,
@@ -222,9 +234,16 @@ gtr_status_t gtr_sswiglu_dwconv(const void *gate, const void *value, long long i
 
 /* Size of the fixed device scratch array behind gtr_gla_fwd_noalloc.  The
  * library holds one such array on every GPU where it is loaded, from the
- * module's load until the process exits.  The split schedule needs at most
- * B*H*(segments-1) summaries of (Dk*Dv + Dk) floats, with segments bounded by
- * the SM count: about 5 MB on a 152-SM device. */
+ * module's load until the process exits.  What a call keeps there is bounded by
+ * the device's SM count n_sm:
+ *   - split schedule: B*H*(segments-1) summaries of (Dk'*Dv' + Dk') floats
+ *     (Dk', Dv' rounded up to 64), and the split keeps B*H*nv*segments <= n_sm
+ *     with nv = Dv'/64, so at most floor(n_sm/nv) * (Dk'*Dv' + Dk') * 4 bytes,
+ *     which is largest for Dk = 128, Dv <= 64: n_sm * 33,280 bytes;
+ *   - balanced schedule: n_sm * (64*64*4 + 8) = n_sm * 16,392 bytes.
+ * So 8 MiB covers every problem on devices of up to 252 SMs (a 152-SM GB300
+ * needs at most 5.06 MB); on larger devices a problem over the limit returns
+ * GTR_ERR_WORKSPACE. */
 #define GTR_GLA_NOALLOC_SCRATCH_BYTES (8u << 20)
 
 /* gtr_gla_fwd for callers that must not allocate device memory on the call
@@ -298,6 +317,25 @@ gtr_status_t gtr_gla_fwd_host(const void *q_host, const void *k_host, const void
  * the tensor-core schedule withholds one chunk's load in its first CTA, so the
  * call reports GTR_ERR_TIMEOUT (no fault is involved). */
 gtr_status_t gtr_gla_sync_status(cudaStream_t stream);
+
+/* Schedules a forward call can run (gtr_gla_last_schedule). */
+typedef enum {
+    GTR_RAN_NONE = 0,         /* nothing launched (no call yet on this thread, or B*H == 0)      */
+    GTR_RAN_SIMT = 1,         /* fp32 CUDA-core recurrence                                        */
+    GTR_RAN_TC = 2,           /* tensor cores, whole sequences dealt round-robin to the SMs       */
+    GTR_RAN_TC_SPLIT = 3,     /* tensor cores, sequences split into segments (two launches)       */
+    GTR_RAN_TC_BALANCED = 4   /* tensor cores, equal chunk ranges per SM with state hand-offs     */
+} gtr_ran_t;
+
+/* What the last successful forward call (gtr_gla_fwd, _sched, _ws, _gated,
+ * _gated_ws, _noalloc; gtr_gla_fwd_host: its last piece) of this host thread
+ * enqueued: *ran receives the schedule that was launched and *planned the one
+ * the library would have chosen with enough workspace.  They differ when the
+ * split or balanced schedule was dropped for lack of workspace, for example
+ * gtr_gla_fwd under stream capture before its internal workspace had grown to
+ * the size the problem needs.  Either pointer may be NULL.  Host state only:
+ * nothing is launched or synchronised. */
+gtr_status_t gtr_gla_last_schedule(int *ran, int *planned);
 
 /* Static, NUL-terminated description of a status code. */
 const char *gtr_status_string(gtr_status_t status);

@@ -18,6 +18,12 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[GTR_GLA_NOALLOC
 namespace {
 
 thread_local int t_last_cuda_error = 0;
+thread_local gtr::Ran t_last_ran;  // schedule of this thread's last successful forward call
+
+gtr_status_t nothing_launched() {
+    t_last_ran = gtr::Ran{};
+    return GTR_OK;
+}
 
 constexpr size_t kAlign = 16;
 constexpr int kMaxHeadDim = 128;
@@ -181,14 +187,17 @@ gtr_status_t dispatch(const gtr::Problem &p, gtr_schedule_t schedule, void *ws, 
                       cudaStream_t stream) {
     cudaError_t e;
     const bool tc = gtr::tc_supported(p);
+    gtr::Ran r;
     if (schedule == GTR_SCHED_SIMT || (schedule == GTR_SCHED_AUTO && !tc)) {
         e = gtr::launch_simt(p, stream);
+        r.ran = r.planned = gtr::kRanSimt;
     } else {
         if (!tc) return GTR_ERR_UNSUPPORTED;
         if (!own_ws) ws = internal_workspace(gtr::tc_workspace_bytes(p), stream, &ws_bytes);
-        e = gtr::launch_tc(p, stream, ws, ws_bytes);
+        e = gtr::launch_tc(p, stream, ws, ws_bytes, &r);
     }
     if (e != cudaSuccess) return cuda_fail(e);
+    t_last_ran = r;
     return GTR_OK;
 }
 
@@ -205,7 +214,7 @@ gtr_status_t gtr_gla_fwd_sched(const void *q, const void *k, const void *v, cons
                                    dtype, out, final_state, &p);
     if (st != GTR_OK) return st;
     if (schedule < GTR_SCHED_AUTO || schedule > GTR_SCHED_TC) return GTR_ERR_INVALID_ARG;
-    if (B == 0 || H == 0) return GTR_OK;
+    if (B == 0 || H == 0) return nothing_launched();
     return dispatch(p, schedule, nullptr, 0, false, stream);
 }
 
@@ -257,7 +266,7 @@ gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const v
                                    dtype, out, final_state, &p);
     if (st != GTR_OK) return st;
     if ((reinterpret_cast<uintptr_t>(workspace) % 256) != 0) return GTR_ERR_INVALID_ARG;
-    if (B == 0 || H == 0) return GTR_OK;
+    if (B == 0 || H == 0) return nothing_launched();
     const size_t need = gtr_gla_workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype);
     if (need > 0 && (workspace == nullptr || workspace_bytes < need)) return GTR_ERR_WORKSPACE;
     return dispatch(p, GTR_SCHED_AUTO, workspace, workspace_bytes, true, stream);
@@ -278,7 +287,7 @@ gtr_status_t gated(const void *q, const void *k, const void *v, const void *log_
                                    dtype, out, final_state, &p);
     if (st != GTR_OK) return st;
     if (!(eps >= 0.f) || !(eps < 3.0e38f)) return GTR_ERR_INVALID_ARG;  // also rejects NaN
-    if (B == 0 || H == 0) return GTR_OK;
+    if (B == 0 || H == 0) return nothing_launched();
     if (!gate || !norm_weight || !aligned(gate) || !aligned(norm_weight)) return GTR_ERR_INVALID_ARG;
     const size_t nv = (size_t)B * p.T * H * Dv * elem_size(dtype);
     if (overlaps(out, nv, gate, nv)) return GTR_ERR_INVALID_ARG;
@@ -322,7 +331,7 @@ gtr_status_t gtr_gla_fwd_noalloc(const void *q, const void *k, const void *v, co
     gtr_status_t st = make_problem(q, k, v, log_gate, B, H, grid_h, grid_w, Dk, Dv, scan_order,
                                    dtype, out, final_state, &p);
     if (st != GTR_OK) return st;
-    if (B == 0 || H == 0) return GTR_OK;
+    if (B == 0 || H == 0) return nothing_launched();
     if (gtr_gla_workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype) > GTR_GLA_NOALLOC_SCRATCH_BYTES)
         return GTR_ERR_WORKSPACE;
     void *scratch = nullptr;
@@ -370,7 +379,7 @@ gtr_status_t gtr_gla_fwd_host(const void *q_host, const void *k_host, const void
     const size_t need = gtr_gla_host_buffer_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype, with_fs);
     if (dev_buffer == nullptr || dev_buffer_bytes < need) return GTR_ERR_WORKSPACE;
     if ((reinterpret_cast<uintptr_t>(dev_buffer) % 256) != 0) return GTR_ERR_INVALID_ARG;
-    if (B == 0 || H == 0) return GTR_OK;
+    if (B == 0 || H == 0) return nothing_launched();
     const size_t T = (size_t)grid_h * grid_w, es = elem_size(dtype);
     const size_t bk = (size_t)B * T * H * Dk * es, bv = (size_t)B * T * H * Dv * es;
     char *base = static_cast<char *>(dev_buffer);
@@ -468,6 +477,12 @@ const char *gtr_status_string(gtr_status_t status) {
 }
 
 int gtr_last_cuda_error(void) { return t_last_cuda_error; }
+
+gtr_status_t gtr_gla_last_schedule(int *ran, int *planned) {
+    if (ran) *ran = t_last_ran.ran;
+    if (planned) *planned = t_last_ran.planned;
+    return GTR_OK;
+}
 
 int gtr_version(void) { return 100; }
 

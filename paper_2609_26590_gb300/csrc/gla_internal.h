@@ -49,10 +49,17 @@ size_t tc_workspace_bytes(const Problem &p);
 // (more units than SMs, a round-robin deal at least 1.25 times an even split's share) on a device
 // with n_sm SMs; its workspace then holds one hand-off state and flag per SM.
 int tc_balanced_plan(const Problem &p, int n_sm);
+// Which schedule a launch ran, and which one it would have run with enough workspace
+// (values of gtr_ran_t in include/gtr_gla.h).
+struct Ran {
+    int ran = 0, planned = 0;
+};
+enum : int { kRanNone = 0, kRanSimt = 1, kRanTc = 2, kRanTcSplit = 3, kRanTcBalanced = 4 };
 // Launches the schedule; it splits sequences or balances ranges only when `workspace`
 // holds at least tc_workspace_bytes(p) bytes (256-byte aligned), else it deals whole
-// sequences round-robin.
-cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes);
+// sequences round-robin.  *ran (may be null) receives what was launched and planned.
+cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes,
+                      Ran *ran = nullptr);
 
 // Device status word of the current device (set by bounded device waits).
 cudaError_t read_and_clear_device_status(unsigned int *status);

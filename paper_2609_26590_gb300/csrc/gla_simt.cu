@@ -6,12 +6,14 @@
 // cannot hold a 1e-5 relative error) and the path for shapes the tensor-core
 // schedule does not take.
 //
-// Mapping: one CTA of 64 threads per (b, h, block of 64 value columns).  Thread
-// j owns column j of S (all Dk rows) in registers, so the state update and the
-// readout o_t[j] = sum_i q_t[i] S[i][j] are thread-local; q_t, k_t and gamma_t
-// are staged in shared memory for 16 tokens at a time and read as broadcasts.
-// The permutation is applied when staging (gather) and when storing o_t
-// (scatter back to the spatial position).
+// Mapping: one CTA of 256 threads per (b, h, block of 64 value columns).  Thread
+// (r, j) owns column j of S over the r-th quarter of the Dk rows in registers, so
+// the state update is thread-local and the readout o_t[j] = sum_i q_t[i] S[i][j] is
+// four partial sums, added after every block of 16 tokens through shared memory
+// (one barrier per block, not per token).  q_t, k_t, gamma_t and v_t of the next
+// block are loaded into registers while the current block runs, then staged in
+// shared memory and read as broadcasts.  The permutation is applied when loading
+// (gather) and when storing o_t (scatter back to the spatial position).
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -20,8 +22,10 @@
 namespace gtr {
 namespace {
 
-constexpr int kTok = 16;    // tokens staged per step
-constexpr int kCols = 64;   // value columns per CTA (= threads per CTA)
+constexpr int kTok = 16;       // tokens staged per block
+constexpr int kCols = 64;      // value columns per CTA
+constexpr int kGroups = 4;     // row quarters of S per column
+constexpr int kSimtThreads = kCols * kGroups;
 
 __device__ __forceinline__ float to_f32(float x) { return x; }
 __device__ __forceinline__ float to_f32(__half x) { return __half2float(x); }
@@ -49,18 +53,22 @@ __device__ __forceinline__ long long scan_token(int order, long long gh, long lo
 }
 
 template <int DKM, typename E>
-__global__ void __launch_bounds__(kCols) gla_simt_kernel(Problem p) {
+__global__ void __launch_bounds__(kSimtThreads) gla_simt_kernel(Problem p) {
+    constexpr int RPT = DKM / kGroups;                 // rows of S per thread
+    constexpr int NQ = kTok * DKM / kSimtThreads;      // staged q / k / gamma values per thread
+    constexpr int NV = kTok * kCols / kSimtThreads;    // staged v values per thread
     __shared__ __align__(16) float sq[kTok][DKM];
     __shared__ __align__(16) float sk[kTok][DKM];
     __shared__ __align__(16) float sgam[kTok][DKM];
     __shared__ float sv[kTok][kCols];
+    __shared__ float po[kGroups][kTok][kCols];          // partial readouts of the block
     __shared__ long long stok[kTok];
 
     const int bh = blockIdx.x;
     const int b = bh / p.H, h = bh % p.H;
     const int c0 = blockIdx.y * kCols;
     const int tid = threadIdx.x;
-    const int col = c0 + tid;
+    const int cj = tid % kCols, grp = tid / kCols;     // column and row quarter owned
     const long long T = p.T;
     const int Dk = p.Dk, Dv = p.Dv, H = p.H;
     const E *q = static_cast<const E *>(p.q);
@@ -69,53 +77,91 @@ __global__ void __launch_bounds__(kCols) gla_simt_kernel(Problem p) {
     const E *g = static_cast<const E *>(p.g);
     E *out = static_cast<E *>(p.out);
 
-    float S[DKM];
-#pragma unroll
-    for (int i = 0; i < DKM; ++i) S[i] = 0.f;
-
-    for (long long s0 = 0; s0 < T; s0 += kTok) {
+    // one block's inputs in registers (zeros / gamma = 1 past the sequence and past Dk, Dv:
+    // padding contributes nothing)
+    float rq[NQ], rk[NQ], rg[NQ], rv[NV];
+    long long rt = 0;
+    auto load_block = [&](long long s0) {
         const int n = (int)((T - s0) < kTok ? (T - s0) : kTok);
-        __syncthreads();  // readers of the previous step are done
-        if (tid < kTok) stok[tid] = tid < n ? scan_token(p.order, p.grid_h, p.grid_w, T, s0 + tid) : 0;
-        __syncthreads();
-        for (int idx = tid; idx < kTok * DKM; idx += kCols) {
-            const int j = idx / DKM, i = idx % DKM;
-            float qv = 0.f, kv = 0.f, gam = 1.f;  // padding rows/channels contribute nothing
+#pragma unroll
+        for (int m = 0; m < NQ; ++m) {
+            const int idx = tid + m * kSimtThreads, j = idx / DKM, i = idx % DKM;
+            float qv = 0.f, kv = 0.f, gam = 1.f;
             if (j < n && i < Dk) {
-                const long long off = (((long long)b * T + stok[j]) * H + h) * Dk + i;
+                const long long off = (((long long)b * T + scan_token(p.order, p.grid_h, p.grid_w, T, s0 + j)) * H + h) * Dk + i;
                 qv = to_f32(q[off]);
                 kv = to_f32(k[off]);
                 float lg = to_f32(g[off]);
                 lg = lg < -1.0e4f ? -1.0e4f : lg;  // gamma = 0 below -1e4; NaN stays NaN
                 gam = expf(lg);
             }
-            sq[j][i] = qv;
-            sk[j][i] = kv;
-            sgam[j][i] = gam;
+            rq[m] = qv;
+            rk[m] = kv;
+            rg[m] = gam;
         }
-        for (int idx = tid; idx < kTok * kCols; idx += kCols) {
-            const int j = idx / kCols, c = idx % kCols;
+#pragma unroll
+        for (int m = 0; m < NV; ++m) {
+            const int idx = tid + m * kSimtThreads, j = idx / kCols, c = idx % kCols;
             float vv = 0.f;
-            if (j < n && c0 + c < Dv) vv = to_f32(v[(((long long)b * T + stok[j]) * H + h) * Dv + c0 + c]);
-            sv[j][c] = vv;
+            if (j < n && c0 + c < Dv)
+                vv = to_f32(v[(((long long)b * T + scan_token(p.order, p.grid_h, p.grid_w, T, s0 + j)) * H + h) * Dv + c0 + c]);
+            rv[m] = vv;
+        }
+        rt = tid < n ? scan_token(p.order, p.grid_h, p.grid_w, T, s0 + tid) : 0;
+    };
+
+    float S[RPT];
+#pragma unroll
+    for (int i = 0; i < RPT; ++i) S[i] = 0.f;
+
+    load_block(0);
+    for (long long s0 = 0; s0 < T; s0 += kTok) {
+        const int n = (int)((T - s0) < kTok ? (T - s0) : kTok);
+        __syncthreads();  // the previous block's shared values and partials are consumed
+#pragma unroll
+        for (int m = 0; m < NQ; ++m) {
+            const int idx = tid + m * kSimtThreads;
+            sq[idx / DKM][idx % DKM] = rq[m];
+            sk[idx / DKM][idx % DKM] = rk[m];
+            sgam[idx / DKM][idx % DKM] = rg[m];
+        }
+#pragma unroll
+        for (int m = 0; m < NV; ++m) {
+            const int idx = tid + m * kSimtThreads;
+            sv[idx / kCols][idx % kCols] = rv[m];
+        }
+        if (tid < kTok) stok[tid] = rt;
+        __syncthreads();
+        if (s0 + kTok < T) load_block(s0 + kTok);  // in flight while this block runs
+        for (int j = 0; j < n; ++j) {
+            const float vj = sv[j][cj];
+            float o0 = 0.f, o1 = 0.f;
+#pragma unroll
+            for (int i = 0; i < RPT; i += 2) {
+                const int r = grp * RPT + i;
+                S[i] = fmaf(sgam[j][r], S[i], sk[j][r] * vj);
+                S[i + 1] = fmaf(sgam[j][r + 1], S[i + 1], sk[j][r + 1] * vj);
+                o0 = fmaf(sq[j][r], S[i], o0);
+                o1 = fmaf(sq[j][r + 1], S[i + 1], o1);
+            }
+            po[grp][j][cj] = o0 + o1;
         }
         __syncthreads();
-        for (int j = 0; j < n; ++j) {
-            const float vj = sv[j][tid];
-            float o = 0.f;
-#pragma unroll
-            for (int i = 0; i < DKM; ++i) {
-                S[i] = fmaf(sgam[j][i], S[i], sk[j][i] * vj);
-                o = fmaf(sq[j][i], S[i], o);
+        // the block's outputs: sum of the four quarters, scattered to the spatial tokens
+        for (int idx = tid; idx < n * kCols; idx += kSimtThreads) {
+            const int j = idx / kCols, c = idx % kCols;
+            if (c0 + c < Dv) {
+                const float o = po[0][j][c] + po[1][j][c] + po[2][j][c] + po[3][j][c];
+                out[(((long long)b * T + stok[j]) * H + h) * Dv + c0 + c] = from_f32<E>(o);
             }
-            if (col < Dv) out[(((long long)b * T + stok[j]) * H + h) * Dv + col] = from_f32<E>(o);
         }
     }
+    const int col = c0 + cj;
     if (p.final_state != nullptr && col < Dv) {
         float *fs = p.final_state + ((long long)b * H + h) * Dk * Dv;
 #pragma unroll
-        for (int i = 0; i < DKM; ++i)
-            if (i < Dk) fs[(long long)i * Dv + col] = S[i];
+        for (int i = 0; i < RPT; ++i)
+            if (grp * RPT + i < Dk) fs[(long long)(grp * RPT + i) * Dv + col] = S[i];
     }
 }
 
@@ -123,11 +169,11 @@ template <typename T>
 cudaError_t launch_typed(const Problem &p, cudaStream_t stream) {
     dim3 grid((unsigned)(p.B * p.H), (unsigned)((p.Dv + kCols - 1) / kCols));
     if (p.Dk <= 32) {
-        gla_simt_kernel<32, T><<<grid, kCols, 0, stream>>>(p);
+        gla_simt_kernel<32, T><<<grid, kSimtThreads, 0, stream>>>(p);
     } else if (p.Dk <= 64) {
-        gla_simt_kernel<64, T><<<grid, kCols, 0, stream>>>(p);
+        gla_simt_kernel<64, T><<<grid, kSimtThreads, 0, stream>>>(p);
     } else {
-        gla_simt_kernel<128, T><<<grid, kCols, 0, stream>>>(p);
+        gla_simt_kernel<128, T><<<grid, kSimtThreads, 0, stream>>>(p);
     }
     return cudaGetLastError();
 }

@@ -1409,7 +1409,7 @@ bool tc_supported(const Problem &p) {
     return get_encode() != nullptr;
 }
 
-cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes) {
+cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes, Ran *ran) {
     TcParams tp;
     if (!get_maps(p, tp.maps)) return cudaErrorInvalidValue;
     int n_sm = 0;
@@ -1428,8 +1428,12 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     tp.nh = pad64(p.Dk) / 64;
     tp.nv = pad64(p.Dv) / 64;
     Split sp = choose_split(p, n_sm);
+    Ran r;
+    r.planned = sp.nseg > 1 ? kRanTcSplit : (choose_balanced(p, n_sm) ? kRanTcBalanced : kRanTc);
+    r.ran = kRanTc;
     if (sp.nseg > 1 && (workspace == nullptr || workspace_bytes < summary_bytes(p, sp.nseg)))
         sp = Split{1, tp.n_chunks};
+    if (sp.nseg > 1) r.ran = kRanTcSplit;
     const int nseg = sp.nseg;
     tp.nseg = nseg;
     tp.seg_len = sp.len;
@@ -1454,6 +1458,8 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     tp.n_units = seqs * nseg;
     if (nseg == 1 && choose_balanced(p, n_sm) && workspace != nullptr && workspace_bytes >= handoff_bytes(n_sm)) {
         // equal contiguous chunk ranges, one CTA per SM
+        r.ran = kRanTcBalanced;
+        if (ran) *ran = r;
         tp.flags = reinterpret_cast<unsigned long long *>(static_cast<char *>(workspace) + (size_t)n_sm * 64 * 64 * sizeof(float));
         tp.epoch = next_epoch();
         const dim3 bgrid(static_cast<unsigned>(n_sm));
@@ -1465,6 +1471,7 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
         if (e != cudaSuccess) return e;
         return cudaGetLastError();
     }
+    if (ran) *ran = r;
     const dim3 grid(static_cast<unsigned>(tp.n_units < n_sm ? tp.n_units : n_sm));
     // outputs from the gen warpgroups: fp16 launches of at most one wave (measured on a GB300:
     // +3 to +6 % there; with several units per CTA, or bf16, the epi storing them was faster)

@@ -53,8 +53,8 @@ struct SwParams {
     void *out;
     const float *weight;
     const float *bias;
-    int grid_h, grid_w, F, rows, ntile_y, ntile_f, ntiles, nstage;
-    uint32_t vbytes, gbytes, stage_bytes;  // box bytes, and the stride of the stages
+    int grid_h, grid_w, F, rows, ntile_y, ntile_f, ntiles;
+    uint32_t vbytes, gbytes;  // bytes of the value box and of the gate box
 };
 
 struct TilePos {
@@ -66,17 +66,13 @@ __device__ __forceinline__ TilePos tile_pos(const SwParams &p, int t) {
     return {tf * SLICE, (rest % p.ntile_y) * p.rows, rest / p.ntile_y};
 }
 
-// TMA loads of the CTA's k-th tile into stage k % nstage (one thread).  Always
-// inlined: the tensor maps are addressed in the kernel's parameter space.
-template <int SLICE>
-__device__ __forceinline__ void issue_tile(const SwParams &p, uint8_t *smem, uint64_t *full, int first, int step,
-                                           int k) {
-    const TilePos tp = tile_pos<SLICE>(p, first + k * step);
-    uint8_t *st = smem + (size_t)(k % p.nstage) * p.stage_bytes;
-    uint64_t *bar = &full[k % p.nstage];
-    mbar_arrive_expect_tx(bar, p.vbytes + p.gbytes);
-    tma_load_4d(st, &p.vmap, bar, tp.f0, -1, tp.y0 - 1, tp.b);
-    tma_load_4d(st + p.vbytes, &p.gmap, bar, tp.f0, 0, tp.y0, tp.b);
+// TMA loads of the CTA's tile (one thread): the value box with its halo, then the
+// gate box.  Always inlined: the tensor maps are addressed in the kernel's
+// parameter space.
+__device__ __forceinline__ void issue_tile(const SwParams &p, uint8_t *smem, uint64_t *full, const TilePos &tp) {
+    mbar_arrive_expect_tx(full, p.vbytes + p.gbytes);
+    tma_load_4d(smem, &p.vmap, full, tp.f0, -1, tp.y0 - 1, tp.b);
+    tma_load_4d(smem + p.vbytes, &p.gmap, full, tp.f0, 0, tp.y0, tp.b);
 }
 
 template <typename E> struct Vec8;
@@ -121,22 +117,20 @@ __global__ void __launch_bounds__(kSwThreads, 2) sswiglu_kernel(const __grid_con
     constexpr int RB = 4;                   // rows per strip piece
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 127) & ~uintptr_t(127));
-    __shared__ uint64_t full[2];
+    __shared__ uint64_t full;
     const int W = p.grid_w;
-    const int first = static_cast<int>(blockIdx.x), step = static_cast<int>(gridDim.x);
-    const int count = first < p.ntiles ? (p.ntiles - 1 - first) / step + 1 : 0;
+    // one tile per CTA (the grid has one CTA per tile)
+    const TilePos tp = tile_pos<SLICE>(p, static_cast<int>(blockIdx.x));
     if (threadIdx.x == 0) {
-        mbar_init(&full[0], 1);
-        mbar_init(&full[1], 1);
+        mbar_init(&full, 1);
         fence_mbar_init();
-        for (int k = 0; k < p.nstage && k < count; ++k) issue_tile<SLICE>(p, smem, full, first, step, k);
+        issue_tile(p, smem, &full, tp);
     }
     __syncthreads();
     const int cg = static_cast<int>(threadIdx.x & 15u);
     E *out = static_cast<E *>(p.out);
     const long long T = (long long)p.grid_h * W;
-    for (int k = 0; k < count; ++k) {
-        const TilePos tp = tile_pos<SLICE>(p, first + k * step);
+    {
         const int fc = tp.f0 + cg * N;
         const bool live = fc < p.F;
         const int R = p.grid_h - tp.y0 < p.rows ? p.grid_h - tp.y0 : p.rows;
@@ -147,17 +141,16 @@ __global__ void __launch_bounds__(kSwThreads, 2) sswiglu_kernel(const __grid_con
             for (int q = 0; q < 9; ++q) w[q][e] = live ? p.weight[(size_t)(fc + e) * 9 + q] : 0.f;
             bs[e] = (live && p.bias != nullptr) ? p.bias[fc + e] : 0.f;
         }
-        const bool ok = mbar_wait(&full[k % p.nstage], (k / p.nstage) & 1, nullptr, kSwWaitNs);
+        const bool ok = mbar_wait(&full, 0, nullptr, kSwWaitNs);
         if (__syncthreads_or(!ok)) {
-            if (threadIdx.x == 0) {
+            if (threadIdx.x == 0) {  // never leave while the copies may still land
                 atomicOr(&g_sswiglu_status, kStatusTimeout);
-                for (int j = k; j < count && j < k + p.nstage; ++j)
-                    mbar_wait(&full[j % p.nstage], (j / p.nstage) & 1, nullptr, kSwWaitNs);
+                mbar_wait(&full, 0, nullptr, kSwWaitNs);
             }
             __syncthreads();
             return;
         }
-        const uint8_t *vt = smem + (size_t)(k % p.nstage) * p.stage_bytes;
+        const uint8_t *vt = smem;
         const uint8_t *gt = vt + p.vbytes;
         const int nrb = (R + RB - 1) / RB;
         // items: (column x, row block) pairs; each walks RB rows down its column with a
@@ -201,8 +194,6 @@ __global__ void __launch_bounds__(kSwThreads, 2) sswiglu_kernel(const __grid_con
                 }
             }
         }
-        __syncthreads();
-        if (threadIdx.x == 0 && k + p.nstage < count) issue_tile<SLICE>(p, smem, full, first, step, k + p.nstage);
     }
 }
 
@@ -214,22 +205,15 @@ size_t stage_bytes(int rows, int W) { return 128u * ((size_t)(rows + 2) * (W + 2
 
 // Rows per tile: the most rows (up to kSwMaxRows and the grid's height) whose boxes
 // fit kSwStageBudget (two CTAs per SM), else, for grids too wide for one row there,
-// kSwSmemBudget (one CTA per SM).  One stage: the kernel also runs a CTA over
-// several tiles with two stages, which measured slower and is not launched.
-void tile_plan(const SwProblem &p, int *rows, int *nstage) {
+// kSwSmemBudget (one CTA per SM); 0 when not even one row fits.
+int tile_rows(const SwProblem &p) {
     for (int pass = 0; pass < 2; ++pass) {
-        const int ns = 1;
         const size_t budget = pass == 0 ? kSwStageBudget : kSwSmemBudget;
         int r = 0;
         while (r < kSwMaxRows && r < p.grid_h && stage_bytes(r + 1, p.grid_w) <= budget) ++r;
-        if (r >= 1) {
-            *rows = r;
-            *nstage = ns;
-            return;
-        }
+        if (r >= 1) return r;
     }
-    *rows = 0;
-    *nstage = 0;
+    return 0;
 }
 
 template <typename E>
@@ -274,9 +258,7 @@ bool encode(CUtensorMap *m, const SwProblem &p, const void *base, int box_w, int
 bool sswiglu_supported(const SwProblem &p) {
     // the value box spans the grid width plus the halo in one TMA dimension (at most
     // 256 elements), and a stage of at least one row must fit the shared memory
-    int rows = 0, nstage = 0;
-    tile_plan(p, &rows, &nstage);
-    return p.grid_w + 2 <= 256 && rows >= 1 && tensor_map_encoder() != nullptr;
+    return p.grid_w + 2 <= 256 && tile_rows(p) >= 1 && tensor_map_encoder() != nullptr;
 }
 
 cudaError_t launch_sswiglu(const SwProblem &p, cudaStream_t stream) {
@@ -284,7 +266,7 @@ cudaError_t launch_sswiglu(const SwProblem &p, cudaStream_t stream) {
     const int slice = 128 / elem_bytes(p.dtype);
     SwParams sp;
     std::memset(&sp, 0, sizeof(sp));
-    tile_plan(p, &sp.rows, &sp.nstage);
+    sp.rows = tile_rows(p);
     sp.out = p.out;
     sp.weight = p.weight;
     sp.bias = p.bias;
@@ -298,11 +280,10 @@ cudaError_t launch_sswiglu(const SwProblem &p, cudaStream_t stream) {
     sp.ntiles = static_cast<int>(tiles);
     sp.vbytes = static_cast<uint32_t>(128u * (size_t)(sp.rows + 2) * (p.grid_w + 2));
     sp.gbytes = static_cast<uint32_t>(128u * (size_t)sp.rows * p.grid_w);
-    sp.stage_bytes = (sp.vbytes + sp.gbytes + 127u) & ~127u;
     if (!encode(&sp.vmap, p, p.value, p.grid_w + 2, sp.rows + 2) || !encode(&sp.gmap, p, p.gate, p.grid_w, sp.rows))
         return cudaErrorInvalidValue;
     const unsigned grid = static_cast<unsigned>(tiles);  // one CTA per tile
-    const size_t smem = (size_t)sp.nstage * sp.stage_bytes + 128;
+    const size_t smem = (size_t)sp.vbytes + sp.gbytes + 128;
     if (p.dtype == 0) return launch_typed<float>(sp, grid, smem, stream);
     if (p.dtype == 1) return launch_typed<__half>(sp, grid, smem, stream);
     return launch_typed<__nv_bfloat16>(sp, grid, smem, stream);

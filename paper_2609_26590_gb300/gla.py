@@ -83,6 +83,8 @@ def load(path: Optional[str] = None):
         lib.gtr_last_cuda_error.argtypes = []
         lib.gtr_version.restype = ci
         lib.gtr_version.argtypes = []
+        lib.gtr_gla_last_schedule.restype = ci
+        lib.gtr_gla_last_schedule.argtypes = [ctypes.POINTER(ci)] * 2
         if path is None:
             _lib = lib
         return lib
@@ -308,6 +310,19 @@ def forward_host(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: to
         final_state.data_ptr() if final_state is not None else None, dev_buffer.data_ptr(),
         dev_buffer.numel() * dev_buffer.element_size(), _stream_ptr(stream))
     _check(status, "gtr_gla_fwd_host", lib)
+
+
+RAN = {0: "none", 1: "simt", 2: "tc", 3: "tc_split", 4: "tc_balanced"}
+
+
+def last_schedule() -> Tuple[str, str]:
+    """(schedule launched, schedule planned) of this thread's last successful forward
+    call, through ``gtr_gla_last_schedule``; they differ when the split or balanced
+    schedule was dropped for lack of workspace."""
+    lib = load()
+    ran, planned = ctypes.c_int(-1), ctypes.c_int(-1)
+    _check(lib.gtr_gla_last_schedule(ctypes.byref(ran), ctypes.byref(planned)), "gtr_gla_last_schedule", lib)
+    return RAN[ran.value], RAN[planned.value]
 
 
 def sync_status(stream: Optional[torch.cuda.Stream] = None) -> int:

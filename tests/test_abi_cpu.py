@@ -79,6 +79,15 @@ def test_validation_rejects_before_launch(lib):
     assert _fwd(lib, B=0, q=1 << 20, k=2 << 20, v=3 << 20, g=4 << 20, out=5 << 20) == 0
 
 
+def test_last_schedule_after_an_empty_call(lib):
+    # an empty call launches nothing and says so; NULL outputs are allowed
+    assert _fwd(lib, B=0, q=1 << 20, k=2 << 20, v=3 << 20, g=4 << 20, out=5 << 20) == 0
+    ran, planned = ctypes.c_int(-1), ctypes.c_int(-1)
+    assert lib.gtr_gla_last_schedule(ctypes.byref(ran), ctypes.byref(planned)) == 0
+    assert (ran.value, planned.value) == (0, 0)
+    assert lib.gtr_gla_last_schedule(None, None) == 0
+
+
 def test_host_buffer_bytes(lib):
     n = lib.gtr_gla_host_buffer_bytes(2, 3, 4, 5, 64, 32, 1, 1)
     T = 20
