@@ -6,11 +6,12 @@
 // cannot hold a 1e-5 relative error) and the path for shapes the tensor-core
 // schedule does not take.
 //
-// Mapping: one CTA of 256 threads per (b, h, block of 64 value columns).  Thread
-// (r, j) owns column j of S over the r-th quarter of the Dk rows in registers, so
+// Mapping: one CTA of 256 threads per (b, h, block of 16 value columns).  Thread
+// (r, j) owns column j of S over the r-th sixteenth of the Dk rows in registers, so
 // the state update is thread-local and the readout o_t[j] = sum_i q_t[i] S[i][j] is
-// four partial sums, added after every block of 16 tokens through shared memory
-// (one barrier per block, not per token).  q_t, k_t, gamma_t and v_t of the next
+// sixteen partial sums, added after every block of 16 tokens through shared memory
+// (one barrier per block, not per token); the per-token chain of a thread is short
+// (2 to 8 rows), which is what bounds this latency-bound recurrence.  q_t, k_t, gamma_t and v_t of the next
 // block are loaded into registers while the current block runs, then staged in
 // shared memory and read as broadcasts.  The permutation is applied when loading
 // (gather) and when storing o_t (scatter back to the spatial position).
@@ -23,8 +24,8 @@ namespace gtr {
 namespace {
 
 constexpr int kTok = 16;       // tokens staged per block
-constexpr int kCols = 64;      // value columns per CTA
-constexpr int kGroups = 4;     // row quarters of S per column
+constexpr int kCols = 16;      // value columns per CTA
+constexpr int kGroups = 16;    // row groups of S per column
 constexpr int kSimtThreads = kCols * kGroups;
 
 __device__ __forceinline__ float to_f32(float x) { return x; }
@@ -147,11 +148,13 @@ __global__ void __launch_bounds__(kSimtThreads) gla_simt_kernel(Problem p) {
             po[grp][j][cj] = o0 + o1;
         }
         __syncthreads();
-        // the block's outputs: sum of the four quarters, scattered to the spatial tokens
+        // the block's outputs: sum over the row groups, scattered to the spatial tokens
         for (int idx = tid; idx < n * kCols; idx += kSimtThreads) {
             const int j = idx / kCols, c = idx % kCols;
             if (c0 + c < Dv) {
-                const float o = po[0][j][c] + po[1][j][c] + po[2][j][c] + po[3][j][c];
+                float o = 0.f;
+#pragma unroll
+                for (int r = 0; r < kGroups; ++r) o += po[r][j][c];
                 out[(((long long)b * T + stok[j]) * H + h) * Dv + c0 + c] = from_f32<E>(o);
             }
         }

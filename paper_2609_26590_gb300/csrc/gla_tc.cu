@@ -1472,7 +1472,11 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
         return cudaGetLastError();
     }
     if (ran) *ran = r;
-    const dim3 grid(static_cast<unsigned>(tp.n_units < n_sm ? tp.n_units : n_sm));
+    // the fewest CTAs that keep the busiest one's unit count: equal shares, and no SM works
+    // on a short share while the others finish (measured on a GB300: B = 32, H = 12, 40 x 40,
+    // bf16, 384 units on 128 CTAs instead of 152 ran 3 % faster, the same at fp16)
+    const int per_cta = (tp.n_units + n_sm - 1) / n_sm;
+    const dim3 grid(static_cast<unsigned>((tp.n_units + per_cta - 1) / per_cta));
     // outputs from the gen warpgroups: fp16 launches of at most one wave (measured on a GB300:
     // +3 to +6 % there; with several units per CTA, or bf16, the epi storing them was faster)
     const bool gen_out = half && tp.n_units <= n_sm;
