@@ -56,6 +56,9 @@ def parse():
                     help="mixer: the chunkwise GLA token mixer (default); sswiglu: the Spatial SwiGLU "
                          "gate-and-depthwise-conv step (Eq. spatial_swiglu) on --sw-workload")
     ap.add_argument("--sw-workload", type=int, default=2)
+    ap.add_argument("--gate-producer", action="store_true",
+                    help="compute the retention gate in the kernel from its rank-16 projection "
+                         "(gtr_gla_fwd_lowrank_gate, Sec. 3.1) instead of reading a stored log-gate")
     ap.add_argument("--no-secondary", action="store_true",
                     help="skip the 6400-token workload the default run also times")
     ap.add_argument("--batch", type=int, default=None,
@@ -137,6 +140,9 @@ def workload_config(w: wl.Workload, world: int, args=None, extra=None):
         cfg["launch"] = "cuda-graph replay" if args.graph else "eager"
         if args.gated:
             cfg["epilogue"] = "output gate u = SiLU(r) * RMSNorm(o), second kernel right after the mixer"
+        if getattr(args, "gate_producer", False):
+            cfg["gate"] = ("computed in the kernel: g = logsigmoid(a W2 + b) / tau from a = x W1 (rank 16), "
+                           "tau %g" % w.tau)
     if extra:
         cfg.update(extra)
     return cfg
@@ -242,8 +248,23 @@ def run_reference(args, w: wl.Workload, rank: int, world: int):
     inp64 = {n: wl.storage_to_f64(inp[n], w.dtype) for n in ("q", "k", "v", "g")}
     del inp
     n_pairs = min(w.B * w.H, max(1, oracle.max_threads()))
+    gp = None
+    if args.gate_producer:  # the sampled images' gates come from the rank-16 projection, in the step
+        nb = (n_pairs + w.H - 1) // w.H
+        gpi = wl.gate_producer_inputs(w.B, w.H, w.T, w.Dk, w.dtype, rank_seed(w, rank) + 29, z_mean=w.z_mean,
+                                       bias_std=0.0)
+        gp = (wl.storage_to_f64(gpi["a"][:nb], w.dtype), wl.storage_to_f64(gpi["w2"], w.dtype),
+              gpi["bias"].astype(np.float64), nb)
+
+    def gates():
+        if gp is None:
+            return inp64["g"]
+        g = np.zeros_like(inp64["g"])
+        g[:gp[3]] = oracle.gate_producer(gp[0], gp[1], gp[2], w.tau)
+        return g
+
     for i in range(args.warmup):
-        oracle.recurrence(inp64["q"], inp64["k"], inp64["v"], inp64["g"], w.grid_h, w.grid_w,
+        oracle.recurrence(inp64["q"], inp64["k"], inp64["v"], gates(), w.grid_h, w.grid_w,
                           w.orders[i % len(w.orders)],
                           pairs=[(b, h) for b in range(w.B) for h in range(w.H)][:n_pairs])
     times = []
@@ -251,7 +272,7 @@ def run_reference(args, w: wl.Workload, rank: int, world: int):
         order = w.orders[i % len(w.orders)]
         pairs = [(b, h) for b in range(w.B) for h in range(w.H)][:n_pairs]
         t0 = time.perf_counter()
-        oracle.recurrence(inp64["q"], inp64["k"], inp64["v"], inp64["g"], w.grid_h, w.grid_w,
+        oracle.recurrence(inp64["q"], inp64["k"], inp64["v"], gates(), w.grid_h, w.grid_w,
                           order, pairs=pairs)
         times.append(time.perf_counter() - t0)
     per_step = sum(times) / len(times)
@@ -474,13 +495,20 @@ def time_mixer(args, w: wl.Workload, rank: int, world: int, local: int, dev, pg)
     inp = wl.workload_inputs(w, B=w.B, seed=seed)
     n_sets = rotation_sets(w.algorithmic_bytes())
     sets = mixer_sets(w, inp, dev, n_sets, args.gated, seed)
+    if args.gate_producer:  # the gate's low-rank inputs instead of the stored log-gate
+        gp = wl.gate_producer_inputs(w.B, w.H, w.T, w.Dk, w.dtype, seed + 29, z_mean=w.z_mean, bias_std=0.0)
+        for j, st in enumerate(sets):
+            st["a"] = to_device(gp["a"], w.dtype, dev)
+            st["w2"] = to_device(gp["w2"], w.dtype, dev)
+            st["bias"] = torch.from_numpy(gp["bias"]).to(dev)
+            del st["g"]
     stream = torch.cuda.current_stream(dev)
     orders = w.orders
     schedule = args.schedule
     tc = gla.tc_supported(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, orders[0], dt)
     kernel_name = "tensor-core chunkwise (tcgen05/TMEM/TMA)" if (tc and schedule != "simt") else "simt recurrence"
     ws_n = gla.workspace_bytes(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, dt) if tc and schedule != "simt" else 0
-    split = ws_n > 0 and gla.split_plan(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv,
+    split = not args.gate_producer and ws_n > 0 and gla.split_plan(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv,
                                          torch.cuda.get_device_properties(dev).multi_processor_count)[0] > 1
     launches_per_step = 2 if split else 1
     if split:
@@ -488,9 +516,16 @@ def time_mixer(args, w: wl.Workload, rank: int, world: int, local: int, dev, pg)
     if args.gated:  # the output gate runs as one more kernel right after the mixer
         launches_per_step += 1
         kernel_name += " + output-gate kernel"
+    if args.gate_producer:
+        if args.gated:
+            raise SystemExit("--gate-producer runs without the output gate")
+        kernel_name += ", retention gate computed in the kernel"
 
     def call(s, order, strm=None, ws=None, graph=False):
-        if args.gated:
+        if args.gate_producer:
+            gla.forward_lowrank_gate(s["q"], s["k"], s["v"], s["a"], s["w2"], s["bias"], w.tau, w.grid_h, w.grid_w,
+                                     order, out=s["out"], final_state=s["fs"], stream=strm)
+        elif args.gated:
             gla.forward_gated(s["q"], s["k"], s["v"], s["g"], s["r"], s["w"], 1e-5, w.grid_h, w.grid_w, order,
                               out=s["out"], final_state=s["fs"], stream=strm, workspace=ws)
         elif graph:
@@ -547,11 +582,15 @@ def time_mixer(args, w: wl.Workload, rank: int, world: int, local: int, dev, pg)
     alg_bytes = w.algorithmic_bytes()
     if args.gated:  # the gate's pre-activation is read once more per token-head (u replaces o)
         alg_bytes += w.B * w.T * w.H * w.Dv * wl.ELEM_SIZE[w.dtype]
+    if args.gate_producer:  # no g tensor; a (rank 16 per token), W2 and the bias instead
+        es = wl.ELEM_SIZE[w.dtype]
+        alg_bytes += (- w.B * w.T * w.H * w.Dk * es + w.B * w.T * wl.GATE_RANK * es
+                      + w.H * wl.GATE_RANK * w.Dk * es + w.H * w.Dk * 4)
     kernel_ms = sum(per_launch_ms) / len(per_launch_ms)
     achieved = alg_bytes / (kernel_ms * 1e-3) / 1e9
     traffic, traffic_note = None, None
     tpath = os.path.join(ROOT, "profiles", "traffic.json")
-    if os.path.exists(tpath) and not args.gated and args.batch is None:
+    if os.path.exists(tpath) and not args.gated and not args.gate_producer and args.batch is None:
         with open(tpath) as f:
             tj = json.load(f)
         entry = tj.get(f"{w.name}:{'tc' if (tc and schedule != 'simt') else 'simt'}")

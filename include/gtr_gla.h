@@ -232,6 +232,32 @@ gtr_status_t gtr_sswiglu_dwconv(const void *gate, const void *value, long long i
                                 const float *weight, const float *bias, int B, int grid_h,
                                 int grid_w, int F, gtr_dtype_t dtype, void *out, cudaStream_t stream);
 
+/* The mixer with its retention gate computed inside the kernel (Sec. 3.1, the key-wise
+ * retention gate gamma_t = sigmoid(x_t W_1 W_2 + b)^(1/tau) with a rank-r factorisation of
+ * the gate projection): instead of a stored log_gate, the kernel reads the rank-r projection
+ * a = x W_1 of every token and forms
+ *
+ *     g[b,t,h,:] = logsigmoid(a[b,t,:] W2[h] + bias[h]) / tau
+ *
+ * per chunk: Z = a W2 by a tensor-core product, the log-sigmoid in fp32, g rounded to fp16,
+ * then the schedule of gtr_gla_fwd.  The gate tensor ([B, T, H, Dk], 2 Dk bytes per
+ * token-head) is never written or read; a costs 2 r bytes per token for all heads.
+ *   a_low     : [B, T, rank], element type `dtype`, contiguous, 16-byte aligned.
+ *   w2        : [H, rank, Dk], element type `dtype`, contiguous, 16-byte aligned.
+ *   gate_bias : [H, Dk] float32, contiguous, 16-byte aligned.
+ *   tau       : > 0 (the paper uses 16).
+ * q, k, v, out, final_state and the other arguments as gtr_gla_fwd.  Tensor-core
+ * schedule only: fp16 or bf16, rank == 16 (the paper's rank), Dk a multiple of 8 up to 64,
+ * Dv a multiple of 8 up to 128, and T = grid_h * grid_w > 192; other well-formed
+ * arguments return GTR_ERR_UNSUPPORTED.  Sequences are dealt whole to the SMs (no split, no
+ * balanced ranges): allocates nothing and does not synchronise (capturable).
+ * Errors as gtr_gla_fwd; gtr_gla_last_schedule reports GTR_RAN_TC. */
+gtr_status_t gtr_gla_fwd_lowrank_gate(const void *q, const void *k, const void *v, const void *a_low,
+                                      const void *w2, const float *gate_bias, float tau, int rank,
+                                      int B, int H, int grid_h, int grid_w, int Dk, int Dv,
+                                      gtr_scan_t scan_order, gtr_dtype_t dtype, void *out,
+                                      float *final_state, cudaStream_t stream);
+
 /* Size of the fixed device scratch array behind gtr_gla_fwd_noalloc.  The
  * library holds one such array on every GPU where it is loaded, from the
  * module's load until the process exits.  What a call keeps there is bounded by

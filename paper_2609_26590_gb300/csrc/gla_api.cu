@@ -342,6 +342,35 @@ gtr_status_t gtr_gla_fwd_noalloc(const void *q, const void *k, const void *v, co
     return dispatch(p, GTR_SCHED_AUTO, scratch, GTR_GLA_NOALLOC_SCRATCH_BYTES, true, stream);
 }
 
+gtr_status_t gtr_gla_fwd_lowrank_gate(const void *q, const void *k, const void *v, const void *a_low,
+                                      const void *w2, const float *gate_bias, float tau, int rank, int B, int H,
+                                      int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
+                                      gtr_dtype_t dtype, void *out, float *final_state, cudaStream_t stream) {
+    // the common checks with q standing in for the unused log_gate; a_low, w2 and the bias are
+    // checked below with their own extents
+    gtr::Problem p;
+    gtr_status_t st = make_problem(q, k, v, q, B, H, grid_h, grid_w, Dk, Dv, scan_order, dtype, out, final_state, &p);
+    if (st != GTR_OK) return st;
+    if (!(tau > 0.f) || !(tau < 3.0e38f)) return GTR_ERR_INVALID_ARG;  // also rejects NaN
+    if (rank < 1) return GTR_ERR_INVALID_ARG;
+    if (B == 0 || H == 0) return nothing_launched();
+    if (!a_low || !w2 || !gate_bias || !aligned(a_low) || !aligned(w2) || !aligned(gate_bias)) return GTR_ERR_INVALID_ARG;
+    const size_t es = elem_size(dtype);
+    const size_t na = (size_t)B * p.T * rank * es, nw = (size_t)H * rank * Dk * es, nb = (size_t)H * Dk * 4;
+    const size_t nv = (size_t)B * p.T * H * Dv * es, nfs = (size_t)B * H * Dk * Dv * 4;
+    const void *extra[3] = {a_low, w2, gate_bias};
+    const size_t extra_n[3] = {na, nw, nb};
+    for (int i = 0; i < 3; ++i)
+        if (overlaps(out, nv, extra[i], extra_n[i]) || overlaps(final_state, nfs, extra[i], extra_n[i]))
+            return GTR_ERR_INVALID_ARG;
+    if (!gtr::tc_gate_supported(p, rank)) return GTR_ERR_UNSUPPORTED;
+    gtr::Ran r;
+    const cudaError_t e = gtr::launch_tc_gate(p, gtr::GateSource{a_low, w2, gate_bias, tau}, stream, &r);
+    if (e != cudaSuccess) return cuda_fail(e);
+    t_last_ran = r;
+    return GTR_OK;
+}
+
 gtr_status_t gtr_gla_fwd(const void *q, const void *k, const void *v, const void *log_gate, int B,
                          int H, int grid_h, int grid_w, int Dk, int Dv, gtr_scan_t scan_order,
                          gtr_dtype_t dtype, void *out, float *final_state, cudaStream_t stream) {

@@ -61,6 +61,21 @@ enum : int { kRanNone = 0, kRanSimt = 1, kRanTc = 2, kRanTcSplit = 3, kRanTcBala
 cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes,
                       Ran *ran = nullptr);
 
+// The retention gate computed inside the mixer (Sec. 3.1): g = logsigmoid(a W2 + b) / tau from
+// the rank-r projection a = x W1 instead of a stored g.
+struct GateSource {
+    const void *a_low;   // [B, T, r] in the problem's dtype
+    const void *w2;      // [H, r, Dk] in the problem's dtype
+    const float *bias;   // [H, Dk]
+    float tau;
+};
+// Whether launch_tc_gate takes these shapes: the tensor-core dtypes, Dk <= 64 (one key half),
+// rank 16, and at least four 64-token chunks per sequence.
+bool tc_gate_supported(const Problem &p, int rank);
+// The tensor-core schedule with the gate producer (whole sequences dealt round-robin; the
+// problem's g pointer is not used).
+cudaError_t launch_tc_gate(const Problem &p, const GateSource &gs, cudaStream_t stream, Ran *ran = nullptr);
+
 // Device status word of the current device (set by bounded device waits).
 cudaError_t read_and_clear_device_status(unsigned int *status);
 

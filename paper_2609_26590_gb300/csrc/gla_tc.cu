@@ -117,8 +117,11 @@ constexpr int kOffSlot = 0;
 constexpr int kOffOp = kOffSlot + kSlots * kSlotBytes;         // per gen group g @32K g: tf32 Q^ @0, K^ @16K
 constexpr int kOffS = kOffOp + 4 * kTile32;                    // 2 x S'_[c] (fp16, MN-major)
 constexpr int kOffL = kOffS + 2 * kTile16;                     // triangle of ones
-constexpr int kRefFloats = 5 * kD;                             // raw mid, raw last, mid*log2e, c1, c2
-constexpr int kOffRef = kOffL + kTile16;                       // per slot
+constexpr int kRank = 16;                                      // rank r of the gate's low-rank projection
+constexpr int kW2Bytes = kRank * kD * 2;                       // a head's W2 block: r x 64 channels, 16-bit
+constexpr int kOffW2 = kOffL + kTile16;                        // gate producer: 2 x W2 (by unit parity)
+constexpr int kRefFloats = 4 * kD;                             // raw A_mid, raw A_last, c1, c2
+constexpr int kOffRef = kOffW2 + 2 * kW2Bytes;                 // per slot
 constexpr int kOffDecay = kOffRef + kSlots * kRefFloats * 4;   // per slot, 64 fp32
 constexpr int kOffMode = kOffDecay + kSlots * kD * 4;          // per slot u32 mode; 2 x 2 fp32 maxima
 constexpr int kOffBar = kOffMode + 64;
@@ -139,7 +142,9 @@ enum {
     BAR_ORDY = BAR_UFULL + 2,          // [2] O(c) may go: gen(c) masked P in smem and TMEM P read
                                        //     (4) + epi wrote Diag(c1) S_[c] and read O(c-2) (4)
     BAR_OFULL = BAR_ORDY + 2,          // [2] O of a virtual chunk done -> epi
-    BAR_DONE = BAR_OFULL + 2,          // every MMA completed (teardown)
+    BAR_ZFULL = BAR_OFULL + 2,         // [2] gate producer: Z = a W2 done -> gen
+    BAR_GRDY = BAR_ZFULL + 2,          // [2] gate producer: gates G written by the gen group (4) -> A issuer
+    BAR_DONE = BAR_GRDY + 2,           // every MMA completed (teardown)
     BAR_COUNT = BAR_DONE + 1
 };
 static_assert(BAR_COUNT <= kNumBars, "barrier space");
@@ -168,6 +173,10 @@ struct TcParams {
     unsigned long long *flags;             // kBalanced: per CTA, == epoch once its hand-off state (in
                                            // summary, [64][64] fp32 per CTA) is written; cleared when read
     unsigned long long epoch;              // kBalanced: nonzero, new for every launch
+    // gate producer (maps[T_G] then load the rank-16 projection a = x W1 instead of the gates)
+    CUtensorMap w2map;                     // W2 [H][r][Dk], 16-bit, box (64 channels, r rows) SW128
+    const float *gbias;                    // b [H][Dk] fp32
+    float tau_inv;                         // 1 / tau
 };
 
 // ---------------------------------------------------------------- helpers
@@ -187,6 +196,15 @@ __device__ __forceinline__ float ex2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
+}
+// log sigma(x) = min(x, 0) - log(1 + e), e = e^{-|x|} in (0, 1]: log(1 + e) by the fast
+// logarithm (absolute error below 2^-21 on [1, 2]), or by its series e - e^2 / 2 where e < 1e-3
+// (error below e^3 / 3), so that the relative error stays below 4e-4 before the gate is
+// rounded to fp16.  NaN propagates; x = +inf gives 0, x = -inf gives -inf.
+__device__ __forceinline__ float log_sigmoid(float x) {
+    const float e = ex2(-fabsf(x) * kLog2e);
+    const float l1p = e < 1.0e-3f ? e * fmaf(-0.5f, e, 1.f) : __logf(1.f + e);
+    return fminf(x, 0.f) - l1p;
 }
 __device__ __forceinline__ float to_tf32(float x) {
     uint32_t r;
@@ -373,7 +391,7 @@ __device__ __forceinline__ int walk_token(int order, int T, int grid_h, int grid
 // Exact scores for one chunk (extreme or non-finite log-decays): serial prefix
 // of the clamped gates, P[rho][sigma] = sum_i q k 2^{a_r,i - a_j,i} (j <= r) by
 // CUDA cores, Qtil = q 2^{a}, Kbar = k 2^{a_last - a}, and the chunk decay.
-template <typename E>
+template <typename E, typename GT>
 __device__ __noinline__ void exact_chunk(uint8_t *tq, uint8_t *tk, uint8_t *tgate, float *as,
                                          float *decay, int rev, int tg, int bar_id) {
     if (tg < kD) {
@@ -381,7 +399,7 @@ __device__ __noinline__ void exact_chunk(uint8_t *tq, uint8_t *tk, uint8_t *tgat
         for (int r = 0; r < kC; ++r) {
             const int rho = rev ? kC - 1 - r : r;
             const uint16_t bits = *reinterpret_cast<const uint16_t *>(tgate + sw128(rho, tg * 2));
-            float x = Elem<E>::unpack(bits).x * kLog2e;
+            float x = Elem<GT>::unpack(bits).x * kLog2e;
             x = x < kGateMinLog2 ? kGateMinLog2 : x;
             run += x;
             as[rho * kD + tg] = run;
@@ -447,12 +465,14 @@ __device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *op
         const uint32_t qa[4] = {qw.x, qw.y, qw.z, qw.w}, ka[4] = {kw.x, kw.y, kw.z, kw.w};
         // A_mid log2, c1 and c2 of the 8 channels (16-byte aligned rows of the references)
         float am[8], c1v[8], c2v[8];
-        *reinterpret_cast<float4 *>(&am[0]) = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl);
-        *reinterpret_cast<float4 *>(&am[4]) = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl + 4);
-        *reinterpret_cast<float4 *>(&c1v[0]) = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl);
-        *reinterpret_cast<float4 *>(&c1v[4]) = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl + 4);
-        *reinterpret_cast<float4 *>(&c2v[0]) = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl);
-        *reinterpret_cast<float4 *>(&c2v[4]) = *reinterpret_cast<const float4 *>(ref + 4 * kD + cl + 4);
+        *reinterpret_cast<float4 *>(&am[0]) = *reinterpret_cast<const float4 *>(ref + cl);
+        *reinterpret_cast<float4 *>(&am[4]) = *reinterpret_cast<const float4 *>(ref + cl + 4);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) am[e] *= kLog2e;
+        *reinterpret_cast<float4 *>(&c1v[0]) = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl);
+        *reinterpret_cast<float4 *>(&c1v[4]) = *reinterpret_cast<const float4 *>(ref + 2 * kD + cl + 4);
+        *reinterpret_cast<float4 *>(&c2v[0]) = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl);
+        *reinterpret_cast<float4 *>(&c2v[4]) = *reinterpret_cast<const float4 *>(ref + 3 * kD + cl + 4);
         float qs[8], ks[8];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -483,7 +503,11 @@ __device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *op
     }
 }
 
-template <typename E, int NH, int NV, int MODE, bool GENOUT>
+// GP (gate producer, one key half, whole sequences): the gates are not read but computed
+// from the rank-16 projection, g = logsigmoid(a W2 + b) / tau (Sec. 3.1, retention gate):
+// Z = a W2 by one MMA into the chunk's TMEM A buffer, g by the gen warpgroup that owns the
+// chunk, written as fp16 over the chunk's gate tile, then A = L G as usual (fp16).
+template <typename E, int NH, int NV, int MODE, bool GENOUT, bool GP = false>
 __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_constant__ TcParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -502,6 +526,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     constexpr bool kSplit = MODE == kSplitFull || MODE == kSummary;
     constexpr bool kBal = MODE == kBalanced;
     static_assert(!kBal || NH == 1, "balanced ranges hand over one key half's state");
+    static_assert(!GP || (NH == 1 && MODE == kFull), "the gate producer runs whole sequences, one key half");
+    // element type of the gate tile: the loaded gates, or the fp16 gates the gate producer writes
+    using GE = typename std::conditional<GP, __half, E>::type;
     // GENOUT (one key half, outputs): the gen warpgroup that built a chunk also reads its
     // outputs back from TMEM and stores them, while it waits for the P of its next chunk,
     // which takes that work off the epi's serial per-chunk chain.  The host selects it where
@@ -541,6 +568,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             mbar_init(&bars[BAR_UFULL + i], 1);
             mbar_init(&bars[BAR_ORDY + i], 8);
             mbar_init(&bars[BAR_OFULL + i], 1);
+            mbar_init(&bars[BAR_ZFULL + i], 1);
+            mbar_init(&bars[BAR_GRDY + i], 4);
         }
         mbar_init(&bars[BAR_DONE], 3);  // one commit per issuer warp
         fence_mbar_init();
@@ -562,7 +591,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 const int s0 = half * 32 + u * 8 + 2 * e;
                 const bool k0 = rev ? (s0 >= rho) : (s0 <= rho);
                 const bool k1 = rev ? (s0 + 1 >= rho) : (s0 + 1 <= rho);
-                w[e] = (k0 ? (uint32_t)Elem<E>::one : 0u) | ((k1 ? (uint32_t)Elem<E>::one : 0u) << 16);
+                w[e] = (k0 ? (uint32_t)Elem<GE>::one : 0u) | ((k1 ? (uint32_t)Elem<GE>::one : 0u) << 16);
             }
             *reinterpret_cast<uint4 *>(L + sw128(rho, (half * 32 + u * 8) * 2)) = make_uint4(w[0], w[1], w[2], w[3]);
         }
@@ -589,12 +618,19 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
                 uint64_t *fb = &bars[BAR_FULL + sl];
                 if (!(p.drop_load && blockIdx.x == 0 && g == 0)) {
-                    mbar_arrive_expect_tx(fb, kSum ? kSlotBytes - kTile16 : kSlotBytes);  // summaries need no q
+                    // gate producer: a unit's first chunk also brings the head's W2 block, into the
+                    // buffer of the unit's parity (the unit before last, whose Z products used it,
+                    // ended at least four chunks earlier: its last Z completed before this slot freed)
+                    const bool w2 = GP && ps.cl == 0;
+                    mbar_arrive_expect_tx(fb, (kSum ? kSlotBytes - kTile16 : kSlotBytes) + (w2 ? kW2Bytes : 0));
+                    if (w2) tma_load_5d(smem + kOffW2 + ((g / L) & 1) * kW2Bytes, &p.w2map, fb, 0, 0, h, 0, 0);
                     chunk_load_boxes(p.order, p.T, p.grid_h, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
                         if (!kSum) tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, xk, h, c2, c3, b);
                         tma_load_5d(st + kK + row * 128, &p.maps[T_K][hi], fb, xk, h, c2, c3, b);
                         tma_load_5d(st + kV + row * 128, &p.maps[T_V][hi], fb, xv, h, c2, c3, b);
-                        tma_load_5d(st + kG + row * 128, &p.maps[T_G][hi], fb, xk, h, c2, c3, b);
+                        // the gate tile, or (gate producer) the 16 projection values of each token,
+                        // zero-filled to a 128-byte row
+                        tma_load_5d(st + kG + row * 128, &p.maps[T_G][hi], fb, GP ? 0 : xk, GP ? 0 : h, c2, c3, b);
                     });
                 }
                 ++issued;
@@ -624,23 +660,44 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         const uint32_t slot0 = smem_u32(smem + kOffSlot);
         bool ok = true;
         if (warp == 1) {
-            const uint32_t idesc_a = instr_desc(Elem<E>::fmt, 64, 64, 0, 1);
+            const uint32_t idesc_a = instr_desc(Elem<GE>::fmt, 64, 64, 0, 1);
+            const uint32_t idesc_z = instr_desc(Elem<E>::fmt, 64, 64, 0, 1);  // a K-major, W2 MN-major
             const uint64_t dL = kdesc(smem_u32(smem + kOffL));
-            int sa = 0;
-            for (int c = 0; c < G; ++c) {
-                if (c >= 2) {
-                    ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_PURDY + (c & 1)], ((c - 2) >> 1) & 1, abort_flag, kWaitLimitNs));
+
+            // GP: Z runs one chunk ahead of A = L G, so that the two gen groups compute their
+            // chunks' gates concurrently: iteration c issues Z(c), then A(c - 1) once the gen group
+            // of c - 1 wrote its gates.  Z(c) reuses the A buffer of chunk c - 2 (PURDY(c - 2): its
+            // A was read), A(c - 1) overwrites Z(c - 1) (GRDY(c - 1): Z was read).
+            for (int c = 0; c < G + (GP ? 1 : 0); ++c) {
+                if (c < G) {
+                    if (c >= 2) {
+                        ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_PURDY + (c & 1)], ((c - 2) >> 1) & 1, abort_flag, kWaitLimitNs));
+                        if (!ok) break;
+                    }
+                    ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + c % kSlots], (c / kSlots) & 1, abort_flag, kWaitLimitNs));
                     if (!ok) break;
+                    tc_fence_after();
+                    if constexpr (GP) {
+                        // Z = a W2 (M = 64 tokens, N = 64 channels, K = r = 16: one MMA) into the
+                        // chunk's A buffer; a tile K-major with 128-byte rows, W2 MN-major
+                        const uint64_t da = kdesc(slot0 + (c % kSlots) * kSlotBytes + kG);
+                        const uint64_t dw = mndesc(smem_u32(smem + kOffW2) + ((c / L) & 1) * kW2Bytes);
+                        mma_f16_ss_warp(tmem + kColA + (c & 1) * 64, da, dw, idesc_z, 0);
+                        mma_commit_warp(&bars[BAR_ZFULL + (c & 1)]);
+                    }
                 }
-                ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_FULL + sa], (c / kSlots) & 1, abort_flag, kWaitLimitNs));
-                if (!ok) break;
-                tc_fence_after();
-                const uint64_t dg = mndesc(slot0 + sa * kSlotBytes + kG);
-                const uint32_t d = tmem + kColA + (c & 1) * 64;
+                const int ca = GP ? c - 1 : c;  // the chunk whose A = L G goes now
+                if (ca < 0) continue;
+                if constexpr (GP) {
+                    ok = !__any_sync(0xffffffffu, !mbar_wait(&bars[BAR_GRDY + (ca & 1)], (ca >> 1) & 1, abort_flag, kWaitLimitNs));
+                    if (!ok) break;
+                    tc_fence_after();
+                }
+                const uint64_t dg = mndesc(slot0 + (ca % kSlots) * kSlotBytes + kG);
+                const uint32_t d = tmem + kColA + (ca & 1) * 64;
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks) mma_f16_ss_warp(d, dL + 2 * ks, dg + 128 * ks, idesc_a, ks > 0);
-                mma_commit_warp(&bars[BAR_AFULL + (c & 1)]);
-                sa = (sa == kSlots - 1) ? 0 : sa + 1;
+                mma_commit_warp(&bars[BAR_AFULL + (ca & 1)]);
             }
         } else if (warp == 14) {
             const uint32_t idesc_p16 = instr_desc(kFmtF16, 64, 64, 0, 0);
@@ -752,8 +809,45 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         for (int c = gw; c < G; c += 2) {
             const int sl = c % kSlots, bb = c & 1;
             const uint32_t ph = (c >> 1) & 1;
-            const bool fail = !mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs);
             uint8_t *st = smem + kOffSlot + sl * kSlotBytes;
+            bool zfail = false;
+            if constexpr (GP) {
+                // the chunk's gates from Z = a W2 (Sec. 3.1): g = logsigmoid(z + b) / tau in fp32,
+                // written as fp16 over the a tile, whose Z product has completed; rows outside
+                // the sequence keep g = 0 (no decay), as zero-filled gate rows do
+                zfail = !mbar_wait(&bars[BAR_ZFULL + bb], ph, abort_flag, kWaitLimitNs);
+                tc_fence_after();
+                uint32_t zr[32];
+                tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&zr[0]));
+                tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&zr[16]));
+                tmem_ld_wait();
+                const StreamPos pz = pos(c);
+                const int wz = chunk_w0(p.order, p.T, pz.c) + row;
+                const bool live = wz >= 0 && wz < p.T;
+                const float *bz = p.gbias + (size_t)(pz.bh % p.H) * p.Dk;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    // 8 channels of the bias (Dk is a multiple of 8: all inside it or all past it)
+                    float bq[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                    if (ch0 + 8 * q < p.Dk) {
+                        *reinterpret_cast<float4 *>(&bq[0]) = __ldg(reinterpret_cast<const float4 *>(bz + ch0 + 8 * q));
+                        *reinterpret_cast<float4 *>(&bq[4]) = __ldg(reinterpret_cast<const float4 *>(bz + ch0 + 8 * q + 4));
+                    }
+                    uint32_t gq[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float g0 = live ? log_sigmoid(__uint_as_float(zr[8 * q + 2 * e]) + bq[2 * e]) * p.tau_inv : 0.f;
+                        const float g1 = live ? log_sigmoid(__uint_as_float(zr[8 * q + 2 * e + 1]) + bq[2 * e + 1]) * p.tau_inv : 0.f;
+                        gq[e] = h2bits(g0, g1);
+                    }
+                    *reinterpret_cast<uint4 *>(st + kG + sw128(row, (ch0 + 8 * q) * 2)) = make_uint4(gq[0], gq[1], gq[2], gq[3]);
+                }
+                fence_proxy_async_smem();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars[BAR_GRDY + bb]);  // this warp's rows of G are in smem
+            }
+            const bool fail = zfail || !mbar_wait(&bars[BAR_AFULL + bb], ph, abort_flag, kWaitLimitNs);
             // bf16 values become fp16 MMA operands in place (exact for |v| in the fp16
             // normal range); the loads go first so that their latency hides behind the
             // operand build, the converted words are stored with the operands
@@ -762,8 +856,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&ar[0]));
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColA + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&ar[16]));
             tmem_ld_wait();
-            // references of chunk c: [0,64) raw A_mid, [64,128) raw A_last, [128,192) A_mid log2,
-            // [192,256) c1 = 2^{A_mid}, [256,320) c2 = 2^{A_last - A_mid}
+            // references of chunk c: [0,64) raw A_mid, [64,128) raw A_last, [128,192) c1 = 2^{A_mid},
+            // [192,256) c2 = 2^{A_last - A_mid}
             float *ref = reinterpret_cast<float *>(smem + kOffRef) + sl * kRefFloats;
             if (!fail && (row == rho_mid || row == rho_last)) {
                 float *dst = ref + (row == rho_mid ? 0 : kD) + ch0;
@@ -792,12 +886,10 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
                 mode = m <= kMaxRefF16 ? kModeF16 : (m <= kMaxRefTF32 ? kModeTF32 : kModeExact);
                 if (tg < 32) {
-                    ref[2 * kD + lane] = am0;
-                    ref[2 * kD + lane + 32] = am1;
-                    ref[3 * kD + lane] = ex2(am0);
-                    ref[3 * kD + lane + 32] = ex2(am1);
-                    ref[4 * kD + lane] = ex2(al0 - am0);
-                    ref[4 * kD + lane + 32] = ex2(al1 - am1);
+                    ref[2 * kD + lane] = ex2(am0);
+                    ref[2 * kD + lane + 32] = ex2(am1);
+                    ref[3 * kD + lane] = ex2(al0 - am0);
+                    ref[3 * kD + lane + 32] = ex2(al1 - am1);
                     decay_s[sl * kD + lane] = ex2(al0);
                     decay_s[sl * kD + lane + 32] = ex2(al1);
                     if (tg == 0) mode_s[sl] = mode;
@@ -839,7 +931,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 if (mode == kModeTF32)
                     tf32_operands<E>(tq, tk, smem + kOffOp + gw * 2 * kTile32, ref, tmem + lane_base + kColA + bb * 64, row, ch0);
                 else
-                    exact_chunk<E>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp + gw * 2 * kTile32), decay_s + sl * kD, rev, tg,
+                    exact_chunk<E, GE>(tq, tk, tgt, reinterpret_cast<float *>(smem + kOffOp + gw * 2 * kTile32), decay_s + sl * kD, rev, tg,
                                    bar_id);
             }
             if constexpr (std::is_same<E, __nv_bfloat16>::value) {
@@ -1005,8 +1097,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 }
                 const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + sl * kRefFloats;
                 const bool fold = (mode_s[sl] == kModeF16);
-                const float c1 = fold ? ref[3 * kD + row] : 1.f;
-                const float c2 = fold ? ref[4 * kD + row] : 1.f;
+                const float c1 = fold ? ref[2 * kD + row] : 1.f;
+                const float c2 = fold ? ref[3 * kD + row] : 1.f;
                 const float dc = decay_s[sl * kD + row];
                 if (!kSum) {
                     // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout)
@@ -1169,6 +1261,22 @@ bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int width, in
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Gate producer: W2 [H][r][Dk] as dims (Dk, r, H, 1, 1), box (64 channels, r rows): one head's
+// block lands as r rows of 128 bytes (SW128, MN-major B of Z = a W2); channels past Dk load as 0.
+bool encode_w2_map(CUtensorMap *m, const void *w2, int H, int Dk, int dtype) {
+    auto enc = get_encode();
+    if (!enc) return false;
+    const cuuint64_t es = 2;
+    cuuint64_t dims[5] = {(cuuint64_t)Dk, (cuuint64_t)kRank, (cuuint64_t)H, 1, 1};
+    cuuint64_t strides[4] = {(cuuint64_t)Dk * es, (cuuint64_t)kRank * Dk * es, (cuuint64_t)H * kRank * Dk * es,
+                             (cuuint64_t)H * kRank * Dk * es};
+    cuuint32_t box[5] = {64, (cuuint32_t)kRank, 1, 1, 1}, estr[5] = {1, 1, 1, 1, 1};
+    const CUtensorMapDataType dt = dtype == 1 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    return enc(m, dt, 5, const_cast<void *>(w2), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Encoded maps are cached per (pointers, shape, order, dtype): a repeated call
 // reuses them instead of encoding 32 maps again.
 struct MapKey {
@@ -1218,7 +1326,7 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     return true;
 }
 
-template <typename E, int NH, int NV, int MODE, bool GENOUT = false>
+template <typename E, int NH, int NV, int MODE, bool GENOUT = false, bool GP = false>
 cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
     // the shared-memory opt-in, once per process and device (setting it again is harmless)
     static std::atomic<unsigned long long> set_on_devices(0);
@@ -1227,11 +1335,12 @@ cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     const unsigned long long bit = 1ull << (dev & 63);
     if (!(set_on_devices.load(std::memory_order_relaxed) & bit)) {
-        e = cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV, MODE, GENOUT>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        e = cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV, MODE, GENOUT, GP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kSmemBytes);
         if (e != cudaSuccess) return e;
         set_on_devices.fetch_or(bit);
     }
-    gla_tc_kernel<E, NH, NV, MODE, GENOUT><<<grid, kThreads, kSmemBytes, stream>>>(tp);
+    gla_tc_kernel<E, NH, NV, MODE, GENOUT, GP><<<grid, kThreads, kSmemBytes, stream>>>(tp);
     return cudaSuccess;
 }
 
@@ -1486,6 +1595,69 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     else
         e = half ? launch_shape<__half, kFull>(grid, tp, stream, gen_out)
                  : launch_shape<__nv_bfloat16, kFull>(grid, tp, stream);
+    if (e != cudaSuccess) return e;
+    return cudaGetLastError();
+}
+
+bool tc_gate_supported(const Problem &p, int rank) {
+    // one 64-channel key half, the paper's rank, and units of at least four chunks (the W2 block
+    // of a unit is double-buffered by unit parity, see the producer)
+    return tc_supported(p) && p.Dk <= 64 && rank == kRank && p.T > 3 * kC;
+}
+
+cudaError_t launch_tc_gate(const Problem &p, const GateSource &gs, cudaStream_t stream, Ran *ran) {
+    if (!tc_gate_supported(p, kRank) || !(gs.tau > 0.f)) return cudaErrorInvalidValue;
+    TcParams tp;
+    std::memset(&tp, 0, sizeof(tp));
+    // q, k and v as in the plain schedule; the gate tiles' maps then load the projection a
+    // ([B, T, r] as a one-head tensor of width r, boxes 64 elements wide: the row's other 48
+    // elements are zero-filled, so the a tile has 128-byte rows like the other tiles)
+    Problem pq = p;
+    pq.g = p.q;
+    if (!get_maps(pq, tp.maps)) return cudaErrorInvalidValue;
+    Problem pa = p;
+    pa.H = 1;
+    for (int hi = 0; hi < kHeights; ++hi)
+        if (!encode_map(&tp.maps[T_G][hi], gs.a_low, pa, kRank, box_height(hi))) return cudaErrorInvalidValue;
+    if (!encode_w2_map(&tp.w2map, gs.w2, p.H, p.Dk, p.dtype)) return cudaErrorInvalidValue;
+    tp.gbias = gs.bias;
+    tp.tau_inv = 1.f / gs.tau;
+    int n_sm = 0;
+    cudaError_t e = sm_count(&n_sm);
+    if (e != cudaSuccess) return e;
+    tp.out = p.out;
+    tp.final_state = p.final_state;
+    tp.H = p.H;
+    tp.grid_h = p.grid_h;
+    tp.grid_w = p.grid_w;
+    tp.order = p.order;
+    tp.T = static_cast<int>(p.T);
+    tp.n_chunks = static_cast<int>((p.T + kC - 1) / kC);
+    tp.Dk = p.Dk;
+    tp.Dv = p.Dv;
+    tp.nh = 1;
+    tp.nv = pad64(p.Dv) / 64;
+    tp.nseg = 1;
+    tp.nsu = 1;
+    tp.seg_len = tp.n_chunks;
+    const char *drop = std::getenv("GTR_GLA_TEST_DROP_LOAD");
+    tp.drop_load = (drop != nullptr && drop[0] == '1') ? 1 : 0;
+    tp.n_units = static_cast<int>(p.B * p.H) * tp.nv;
+    if (ran) *ran = Ran{kRanTc, kRanTc};
+    const int per_cta = (tp.n_units + n_sm - 1) / n_sm;
+    const dim3 grid(static_cast<unsigned>((tp.n_units + per_cta - 1) / per_cta));
+    const bool gen_out = p.dtype == 1 && tp.n_units <= n_sm;  // as the plain schedule
+    if (p.dtype == 1) {
+        if (gen_out)
+            e = tp.nv == 1 ? launch_kernel<__half, 1, 1, kFull, true, true>(grid, tp, stream)
+                           : launch_kernel<__half, 1, 2, kFull, true, true>(grid, tp, stream);
+        else
+            e = tp.nv == 1 ? launch_kernel<__half, 1, 1, kFull, false, true>(grid, tp, stream)
+                           : launch_kernel<__half, 1, 2, kFull, false, true>(grid, tp, stream);
+    } else {
+        e = tp.nv == 1 ? launch_kernel<__nv_bfloat16, 1, 1, kFull, false, true>(grid, tp, stream)
+                       : launch_kernel<__nv_bfloat16, 1, 2, kFull, false, true>(grid, tp, stream);
+    }
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

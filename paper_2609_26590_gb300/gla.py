@@ -83,6 +83,8 @@ def load(path: Optional[str] = None):
         lib.gtr_last_cuda_error.argtypes = []
         lib.gtr_version.restype = ci
         lib.gtr_version.argtypes = []
+        lib.gtr_gla_fwd_lowrank_gate.restype = ci
+        lib.gtr_gla_fwd_lowrank_gate.argtypes = [vp] * 6 + [ctypes.c_float] + [ci] * 9 + [vp, vp, vp]
         lib.gtr_gla_last_schedule.restype = ci
         lib.gtr_gla_last_schedule.argtypes = [ctypes.POINTER(ci)] * 2
         if path is None:
@@ -310,6 +312,38 @@ def forward_host(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: to
         final_state.data_ptr() if final_state is not None else None, dev_buffer.data_ptr(),
         dev_buffer.numel() * dev_buffer.element_size(), _stream_ptr(stream))
     _check(status, "gtr_gla_fwd_host", lib)
+
+
+def forward_lowrank_gate(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, a_low: torch.Tensor,
+                         w2: torch.Tensor, gate_bias: torch.Tensor, tau: float, grid_h: int, grid_w: int,
+                         order: int = ROW_FWD, out: Optional[torch.Tensor] = None, final_state=True,
+                         stream: Optional[torch.cuda.Stream] = None) -> Tuple[torch.Tensor, Optional[torch.Tensor]]:
+    """Mixer with the retention gate computed in the kernel, through ``gtr_gla_fwd_lowrank_gate``:
+    g = logsigmoid(a_low W2 + b) / tau.  a_low: [B, T, r] (same dtype as q); w2: [H, r, Dk];
+    gate_bias: [H, Dk] float32; all contiguous CUDA tensors.  Returns (out, final_state)."""
+    lib = load()
+    B, H, Dk, Dv = _dims(q, v, grid_h, grid_w)
+    if a_low.dim() != 3 or a_low.shape[:2] != q.shape[:2] or w2.dim() != 3 or tuple(w2.shape[::2]) != (H, Dk):
+        raise ValueError("a_low must be [B, T, r] and w2 [H, r, Dk]")
+    if tuple(gate_bias.shape) != (H, Dk) or gate_bias.dtype != torch.float32:
+        raise ValueError("gate_bias must be a [H, Dk] float32 tensor")
+    for name, t in (("q", q), ("k", k), ("v", v), ("a_low", a_low), ("w2", w2), ("gate_bias", gate_bias)):
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    rank = a_low.shape[2]
+    if out is None:
+        out = torch.empty(v.shape, dtype=v.dtype, device=v.device)
+    fs = None
+    if final_state is True:
+        fs = torch.empty((B, H, Dk, Dv), dtype=torch.float32, device=q.device)
+    elif isinstance(final_state, torch.Tensor):
+        fs = final_state
+    status = lib.gtr_gla_fwd_lowrank_gate(
+        q.data_ptr(), k.data_ptr(), v.data_ptr(), a_low.data_ptr(), w2.data_ptr(), gate_bias.data_ptr(),
+        float(tau), rank, B, H, grid_h, grid_w, Dk, Dv, order, _DTYPES[q.dtype], out.data_ptr(),
+        fs.data_ptr() if fs is not None else None, _stream_ptr(stream))
+    _check(status, "gtr_gla_fwd_lowrank_gate", lib)
+    return out, fs
 
 
 RAN = {0: "none", 1: "simt", 2: "tc", 3: "tc_split", 4: "tc_balanced"}

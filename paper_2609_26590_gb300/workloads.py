@@ -142,6 +142,23 @@ def make_inputs(B: int, H: int, grid_h: int, grid_w: int, Dk: int, Dv: int, dtyp
     return out
 
 
+GATE_RANK = 16   # rank r of the gate's low-rank projection (Sec. 3.1)
+
+
+def gate_producer_inputs(B: int, H: int, T: int, Dk: int, dtype: str, seed: int,
+                         z_mean: float = 0.0, rank: int = GATE_RANK,
+                         bias_std: float = 0.25) -> Dict[str, np.ndarray]:
+    """Seeded inputs of the in-kernel retention gate: the projection a = x W1 [B, T, rank]
+    ~ N(0, 1), the second factor W2 [H, rank, Dk] ~ N(0, 1/rank) (so a W2 ~ N(0, 1)), both in
+    the storage dtype, and the bias [H, Dk] ~ z_mean + N(0, bias_std^2) in float32 (bias_std
+    = 0: the gate pre-activation is N(z_mean, 1) per token and channel, as in the workloads)."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    a = round_to_storage(rng.standard_normal((B, T, rank)), dtype)
+    w2 = round_to_storage(rng.standard_normal((H, rank, Dk)) / np.sqrt(rank), dtype)
+    bias = (z_mean + bias_std * rng.standard_normal((H, Dk))).astype(np.float32)
+    return {"a": a, "w2": w2, "bias": bias}
+
+
 def workload_inputs(w: Workload, B: Optional[int] = None, seed: Optional[int] = None):
     """Inputs of workload ``w`` (optionally with a smaller batch, same distributions)."""
     s = (1234 + w.wid) if seed is None else seed
