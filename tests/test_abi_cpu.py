@@ -178,3 +178,30 @@ def test_sswiglu_entry_point_validates_before_any_launch(lib):
     assert call(dtype=7) == 1
     assert call(out=g + 1024) == 1         # the output overlaps the inputs
     assert call(B=0, gate=None, value=None, weight=None, out=None) == 0   # empty batch: nothing to do
+
+
+def test_lowrank_gate_validation_rejects_before_launch(lib):
+    # gtr_gla_fwd_lowrank_gate(q, k, v, a_low, w2, bias, tau, rank, B, H, gh, gw, Dk, Dv, order, dtype,
+    #                          out, final_state, stream): bad arguments never reach the GPU
+    q, k, v, out = 1 << 20, 2 << 20, 3 << 20, 4 << 20
+    a, w2, bias = 5 << 20, 6 << 20, 7 << 20
+
+    def call(a=a, w2=w2, bias=bias, tau=16.0, rank=16, B=1, Dk=64, q=q):
+        return lib.gtr_gla_fwd_lowrank_gate(q, k, v, a, w2, bias, tau, rank, B, 2, 16, 16, Dk, 64, 0, 1,
+                                            out, None, None)
+
+    assert call(tau=0.0) == 1
+    assert call(tau=-1.0) == 1
+    assert call(tau=float("nan")) == 1
+    assert call(rank=0) == 1
+    assert call(a=None) == 1
+    assert call(w2=None) == 1
+    assert call(bias=None) == 1
+    assert call(bias=bias + 4) == 1          # the bias must be 16-byte aligned
+    assert call(a=a + 8) == 1
+    assert call(q=None) == 1
+    # an empty batch is valid and launches nothing
+    assert call(B=0) == 0
+    ran, planned = ctypes.c_int(-1), ctypes.c_int(-1)
+    assert lib.gtr_gla_last_schedule(ctypes.byref(ran), ctypes.byref(planned)) == 0
+    assert (ran.value, planned.value) == (0, 0)
