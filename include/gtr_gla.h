@@ -186,11 +186,14 @@ gtr_status_t gtr_gla_fwd_ws(const void *q, const void *k, const void *v, const v
  * RMSNorm(o)_j = o_j / sqrt(mean over the head's Dv outputs of o^2 + eps) *
  * norm_weight[j] (`norm_weight`: Dv fp32 values on the device, shared by the
  * heads; eps >= 0).  App. C.3 fuses this epilogue into the mixer kernel's
- * output stores; here a second kernel applies it to `out` in place right after
- * the mixer (o is rounded to the dtype in between), reading o back while it is
- * still in L2 for outputs that fit there: on GB300 that was measured 1.45-1.7x
- * faster than the fused stores, whose extra work lands on the mixer's critical
- * path.  final_state is the mixer's state as in gtr_gla_fwd.  `gate` and `norm_weight` must be 16-byte
+ * output stores.  Here the tensor-core schedule does so (u rounded once, from
+ * the fp32 outputs) for launches of few sequences with Dk, Dv <= 64 (at most half
+ * as many B*H units as SMs), where it saves a launch; otherwise a second kernel
+ * applies it to `out` in place right after the mixer (o is rounded to the dtype
+ * in between), reading o back while it is still in L2: on GB300 that was measured
+ * 1.14-1.26x faster than the fused stores for large batches, whose extra work
+ * lands on the mixer's critical chain.  final_state is the mixer's state as in
+ * gtr_gla_fwd.  `gate` and `norm_weight` must be 16-byte
  * aligned and `gate` must not overlap `out`.  Allocation, workspace and errors
  * as gtr_gla_fwd. */
 gtr_status_t gtr_gla_fwd_gated(const void *q, const void *k, const void *v, const void *log_gate,

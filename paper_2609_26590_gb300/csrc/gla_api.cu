@@ -184,7 +184,8 @@ cudaError_t host_pipe(HostPipe **out) {  // caller holds g_pipe_mutex
 
 // Dispatch of one validated, non-empty problem; `ws` null means the internal workspace.
 gtr_status_t dispatch(const gtr::Problem &p, gtr_schedule_t schedule, void *ws, size_t ws_bytes, bool own_ws,
-                      cudaStream_t stream) {
+                      cudaStream_t stream, const gtr::Gate *gate = nullptr, bool *gate_fused = nullptr) {
+    if (gate_fused) *gate_fused = false;
     cudaError_t e;
     const bool tc = gtr::tc_supported(p);
     gtr::Ran r;
@@ -194,7 +195,7 @@ gtr_status_t dispatch(const gtr::Problem &p, gtr_schedule_t schedule, void *ws, 
     } else {
         if (!tc) return GTR_ERR_UNSUPPORTED;
         if (!own_ws) ws = internal_workspace(gtr::tc_workspace_bytes(p), stream, &ws_bytes);
-        e = gtr::launch_tc(p, stream, ws, ws_bytes, &r);
+        e = gtr::launch_tc(p, stream, ws, ws_bytes, &r, gate, gate_fused);
     }
     if (e != cudaSuccess) return cuda_fail(e);
     t_last_ran = r;
@@ -295,9 +296,14 @@ gtr_status_t gated(const void *q, const void *k, const void *v, const void *log_
         const size_t need = gtr_gla_workspace_bytes(B, H, grid_h, grid_w, Dk, Dv, dtype);
         if (need > 0 && (ws == nullptr || ws_bytes < need)) return GTR_ERR_WORKSPACE;
     }
-    st = dispatch(p, GTR_SCHED_AUTO, ws, ws_bytes, own_ws, stream);
+    // the tensor-core schedule applies the gate in its stores where a row's outputs stay in one
+    // CTA (Dk, Dv <= 64, not balanced); otherwise a second kernel applies it to `out` in place
+    const gtr::Gate g{gate, norm_weight, eps};
+    bool fused = false;
+    st = dispatch(p, GTR_SCHED_AUTO, ws, ws_bytes, own_ws, stream, &g, &fused);
     if (st != GTR_OK) return st;
-    const cudaError_t e = gtr::launch_gate_epilogue(p, gtr::Gate{gate, norm_weight, eps}, stream);
+    if (fused) return GTR_OK;
+    const cudaError_t e = gtr::launch_gate_epilogue(p, g, stream);
     if (e != cudaSuccess) return cuda_fail(e);
     return GTR_OK;
 }

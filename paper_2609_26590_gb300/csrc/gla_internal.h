@@ -57,9 +57,11 @@ struct Ran {
 enum : int { kRanNone = 0, kRanSimt = 1, kRanTc = 2, kRanTcSplit = 3, kRanTcBalanced = 4 };
 // Launches the schedule; it splits sequences or balances ranges only when `workspace`
 // holds at least tc_workspace_bytes(p) bytes (256-byte aligned), else it deals whole
-// sequences round-robin.  *ran (may be null) receives what was launched and planned.
+// sequences round-robin.  *ran (may be null) receives what was launched and planned.  With
+// `gate`, launches whose rows fit one thread pair (Dk, Dv <= 64) and are not balanced apply
+// the output gate in the kernel's stores and set *gate_fused; otherwise the caller applies it.
 cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes,
-                      Ran *ran = nullptr);
+                      Ran *ran = nullptr, const Gate *gate = nullptr, bool *gate_fused = nullptr);
 
 // The retention gate computed inside the mixer (Sec. 3.1): g = logsigmoid(a W2 + b) / tau from
 // the rank-r projection a = x W1 instead of a stored g.

@@ -177,6 +177,10 @@ struct TcParams {
     CUtensorMap w2map;                     // W2 [H][r][Dk], 16-bit, box (64 channels, r rows) SW128
     const float *gbias;                    // b [H][Dk] fp32
     float tau_inv;                         // 1 / tau
+    // output gate fused into the gen warpgroups' stores (GATED): u = SiLU(r) RMSNorm(o) w
+    const void *gate_r;                    // r = x W_r [B][T][H][Dv], the input dtype
+    const float *gate_w;                   // RMSNorm weight [Dv]
+    float gate_eps;
 };
 
 // ---------------------------------------------------------------- helpers
@@ -507,7 +511,10 @@ __device__ __noinline__ void tf32_operands(uint8_t *tq, uint8_t *tk, uint8_t *op
 // from the rank-16 projection, g = logsigmoid(a W2 + b) / tau (Sec. 3.1, retention gate):
 // Z = a W2 by one MMA into the chunk's TMEM A buffer, g by the gen warpgroup that owns the
 // chunk, written as fp16 over the chunk's gate tile, then A = L G as usual (fp16).
-template <typename E, int NH, int NV, int MODE, bool GENOUT, bool GP = false>
+// GATED (outputs stored by the gen warpgroups, one key half, one value slice): the stores
+// apply the output gate u = SiLU(r) * RMSNorm(o) * w of Sec. 3.1 to the row's fp32 outputs
+// (the deployed kernel's fused epilogue, App. C.3), so o is rounded once, as u.
+template <typename E, int NH, int NV, int MODE, bool GENOUT, bool GP = false, bool GATED = false>
 __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_constant__ TcParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -527,6 +534,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     constexpr bool kBal = MODE == kBalanced;
     static_assert(!kBal || NH == 1, "balanced ranges hand over one key half's state");
     static_assert(!GP || (NH == 1 && MODE == kFull), "the gate producer runs whole sequences, one key half");
+    static_assert(!GATED || (GENOUT && NH == 1 && NV == 1 && MODE != kSummary), "the fused gate normalises whole rows");
     // element type of the gate tile: the loaded gates, or the fp16 gates the gate producer writes
     using GE = typename std::conditional<GP, __half, E>::type;
     // GENOUT (one key half, outputs): the gen warpgroup that built a chunk also reads its
@@ -791,11 +799,43 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + (co & 1) * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
             tmem_ld_wait();
             uint32_t ow[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) ow[j] = Elem<E>::pack(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
             const StreamPos po = pos(co);
             const int b = po.bh / p.H, h = po.bh % p.H;
             const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
+            if constexpr (GATED) {
+                // u = SiLU(r) * o / sqrt(mean_j o_j^2 + eps) * w over the head's Dv outputs: this
+                // thread holds 32 of the row's columns, the lane 16 apart the other 32 (padded
+                // columns are 0 and count for nothing)
+                uint4 rq[4] = {};
+                const E *rrow = static_cast<const E *>(p.gate_r) + (((size_t)b * p.T + (t < 0 ? 0 : t)) * p.H + h) * p.Dv;
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    if (t >= 0 && ch0 + 8 * q < p.Dv) rq[q] = *reinterpret_cast<const uint4 *>(rrow + ch0 + 8 * q);
+                float ss = 0.f;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) ss = fmaf(__uint_as_float(r[j]), __uint_as_float(r[j]), ss);
+                ss += __shfl_xor_sync(0xffffffffu, ss, 16);
+                const float inv = rsqrtf(ss / static_cast<float>(p.Dv) + p.gate_eps);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    float wq[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                    if (ch0 + 8 * q < p.Dv) {
+                        *reinterpret_cast<float4 *>(&wq[0]) = __ldg(reinterpret_cast<const float4 *>(p.gate_w + ch0 + 8 * q));
+                        *reinterpret_cast<float4 *>(&wq[4]) = __ldg(reinterpret_cast<const float4 *>(p.gate_w + ch0 + 8 * q + 4));
+                    }
+                    const uint32_t rw[4] = {rq[q].x, rq[q].y, rq[q].z, rq[q].w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float2 z = Elem<E>::unpack(rw[e]);
+                        const float s0 = __fdividef(z.x, 1.f + __expf(-z.x)), s1 = __fdividef(z.y, 1.f + __expf(-z.y));
+                        const float o0 = __uint_as_float(r[8 * q + 2 * e]), o1 = __uint_as_float(r[8 * q + 2 * e + 1]);
+                        ow[4 * q + e] = Elem<E>::pack(s0 * o0 * inv * wq[2 * e], s1 * o1 * inv * wq[2 * e + 1]);
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) ow[j] = Elem<E>::pack(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
+            }
             if (t >= 0) {  // the row's columns inside Dv (padded columns stay behind)
                 const int col0 = 64 * po.vb + ch0;
                 uint4 *dst = reinterpret_cast<uint4 *>(static_cast<E *>(p.out) + (((size_t)b * p.T + t) * p.H + h) * p.Dv + col0);
@@ -1326,7 +1366,7 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     return true;
 }
 
-template <typename E, int NH, int NV, int MODE, bool GENOUT = false, bool GP = false>
+template <typename E, int NH, int NV, int MODE, bool GENOUT = false, bool GP = false, bool GATED = false>
 cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
     // the shared-memory opt-in, once per process and device (setting it again is harmless)
     static std::atomic<unsigned long long> set_on_devices(0);
@@ -1335,12 +1375,12 @@ cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     const unsigned long long bit = 1ull << (dev & 63);
     if (!(set_on_devices.load(std::memory_order_relaxed) & bit)) {
-        e = cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV, MODE, GENOUT, GP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(gla_tc_kernel<E, NH, NV, MODE, GENOUT, GP, GATED>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kSmemBytes);
         if (e != cudaSuccess) return e;
         set_on_devices.fetch_or(bit);
     }
-    gla_tc_kernel<E, NH, NV, MODE, GENOUT, GP><<<grid, kThreads, kSmemBytes, stream>>>(tp);
+    gla_tc_kernel<E, NH, NV, MODE, GENOUT, GP, GATED><<<grid, kThreads, kSmemBytes, stream>>>(tp);
     return cudaSuccess;
 }
 
@@ -1518,7 +1558,9 @@ bool tc_supported(const Problem &p) {
     return get_encode() != nullptr;
 }
 
-cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes, Ran *ran) {
+cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, size_t workspace_bytes, Ran *ran,
+                      const Gate *gate, bool *gate_fused) {
+    if (gate_fused) *gate_fused = false;
     TcParams tp;
     if (!get_maps(p, tp.maps)) return cudaErrorInvalidValue;
     int n_sm = 0;
@@ -1581,6 +1623,19 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
         return cudaGetLastError();
     }
     if (ran) *ran = r;
+    // output gate fused into the stores: one key half and one value slice (a row's Dv outputs in
+    // one thread pair), outputs stored by the gen warpgroups, for launches of few sequences (at
+    // most half as many units as SMs), where it saves a launch: measured on a GB300 (graph
+    // replays, interleaved) 3.5 % faster at B = 1, H = 6, 40 x 40, but 1.14-1.26x slower than
+    // the separate gate kernel at B = 32, H = 12, 40 x 40 and B = 8, H = 16, 80 x 80, where the
+    // gate's work lands on the gen warpgroups' share of the critical chain
+    const bool fuse = gate != nullptr && tp.nh == 1 && tp.nv == 1 && 2 * seqs <= n_sm;
+    if (fuse) {
+        tp.gate_r = gate->r;
+        tp.gate_w = gate->w;
+        tp.gate_eps = gate->eps;
+        if (gate_fused) *gate_fused = true;
+    }
     // the fewest CTAs that keep the busiest one's unit count: equal shares, and no SM works
     // on a short share while the others finish (measured on a GB300: B = 32, H = 12, 40 x 40,
     // bf16, 384 units on 128 CTAs instead of 152 ran 3 % faster, the same at fp16)
@@ -1589,6 +1644,16 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     // outputs from the gen warpgroups: fp16 launches of at most one wave (measured on a GB300:
     // +3 to +6 % there; with several units per CTA, or bf16, the epi storing them was faster)
     const bool gen_out = half && tp.n_units <= n_sm;
+    if (fuse) {
+        if (nseg > 1)
+            e = half ? launch_kernel<__half, 1, 1, kSplitFull, true, false, true>(grid, tp, stream)
+                     : launch_kernel<__nv_bfloat16, 1, 1, kSplitFull, true, false, true>(grid, tp, stream);
+        else
+            e = half ? launch_kernel<__half, 1, 1, kFull, true, false, true>(grid, tp, stream)
+                     : launch_kernel<__nv_bfloat16, 1, 1, kFull, true, false, true>(grid, tp, stream);
+        if (e != cudaSuccess) return e;
+        return cudaGetLastError();
+    }
     if (nseg > 1)
         e = half ? launch_shape<__half, kSplitFull>(grid, tp, stream, gen_out)
                  : launch_shape<__nv_bfloat16, kSplitFull>(grid, tp, stream);

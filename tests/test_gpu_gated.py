@@ -2,11 +2,13 @@
 kernel's stores) against the fp64 oracle: u = SiLU(r) * RMSNorm(o) per head with
 o the oracle's recurrence.
 
-Bars for 16-bit u: the library applies the gate to the stored (rounded) o, so
-u carries two roundings, and the gate multiplies each output by SiLU(r) w / rms,
-so an output error at the mixer's bar (max-abs 1e-2 max|o|) can grow relative to
-max|u| where that factor is largest: rel L2 <= 4e-3 and max-abs <= 4e-2 max|u|.
-fp32: rel L2 <= 1e-5."""
+Bars for 16-bit u: where the tensor-core schedule applies the gate in its stores
+(Dk, Dv <= 64, few sequences: 2 B H <= SMs) u is rounded once, from the fp32 outputs, and
+is held to the mixer's bar (rel L2 <= 2e-3, max-abs <= 1e-2 max|u|).  Elsewhere a
+second kernel applies the gate to the stored (rounded) o, so u carries two
+roundings, and the gate multiplies each output by SiLU(r) w / rms, so an output
+error at the mixer's bar can grow relative to max|u| where that factor is largest:
+rel L2 <= 4e-3 and max-abs <= 4e-2 max|u|.  fp32: rel L2 <= 1e-5."""
 import numpy as np
 import pytest
 import torch
@@ -59,7 +61,9 @@ def test_gated_output_all_orders(case):
     t = {n: to_torch(inp[n], dtype) for n in ("q", "k", "v", "g")}
     tr = to_torch(r, dtype)
     tw = torch.from_numpy(w).cuda()
-    scale = 1.0 if dtype == "f32" else 2.0
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    fused = dtype != "f32" and Dk <= 64 and Dv <= 64 and 2 * B * H <= n_sm
+    scale = 1.0 if (dtype == "f32" or fused) else 2.0
     for order in wl.ALL_ORDERS:
         ref_o, ref_s = oracle.recurrence(f["q"], f["k"], f["v"], f["g"], gh, gw, order)
         ref_u = oracle.gated_output(ref_o, r64, w.astype(np.float64), eps)
@@ -73,7 +77,7 @@ def test_gated_output_all_orders(case):
         bar_l2 = 1e-5 if dtype == "f32" else 2e-3 * scale
         assert e["rel_l2"] <= bar_l2, f"order {order}: {e}"
         if dtype != "f32":
-            assert e["max_abs"] <= 2e-2 * scale * e["max_ref"], f"order {order}: {e}"
+            assert e["max_abs"] <= (1e-2 if fused else 4e-2) * e["max_ref"], f"order {order}: {e}"
         assert_within_bar(fs.cpu().numpy().astype(np.float64), ref_s, dtype, f"state {order}")
 
 
