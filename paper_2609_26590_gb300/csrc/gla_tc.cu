@@ -31,10 +31,12 @@
 // over g, bf16 v converted to fp16 in place), so four chunks can be in flight.
 // Only the tf32 score operands use separate buffers, one per gen warpgroup, so
 // that tf32-mode chunks of the two groups never wait for each other.  Row orders
-// load one 64-row TMA box per tensor and chunk; column orders
-// one box per column segment of the chunk, of the segment's exact height (a
-// tensor map per height).  The scan permutation lives in the box coordinates of
-// the loads and in the addresses of the output stores.
+// load one 64-row TMA box per tensor and chunk; column orders one im2col load per
+// tensor (a map whose fastest spatial dimension is the grid row, so 64 pixels run
+// down a column and on into the next).  Chunks that reach past either end of the
+// sequence load one box per column segment instead, of the segment's exact height (a
+// tensor map per height), and zero-fill boxes for the rows outside.  The scan
+// permutation lives in the load coordinates and in the addresses of the output stores.
 //
 // Warp roles (512 threads, one CTA per SM; four warps per SM sub-partition, so a
 // thread keeps 128 registers).  Few roles with small loops keep the hot code
@@ -156,6 +158,7 @@ enum { T_Q = 0, T_K = 1, T_V = 2, T_G = 3, kTensors = 4 };
 
 struct TcParams {
     CUtensorMap maps[kTensors][kHeights];  // box height box_height(i)
+    CUtensorMap cmaps[kTensors];           // column orders: a chunk's 64-token walk as one im2col load
     void *out;
     float *final_state;
     int H, grid_h, grid_w, order, n_chunks, T;
@@ -632,7 +635,17 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     const bool w2 = GP && ps.cl == 0;
                     mbar_arrive_expect_tx(fb, (kSum ? kSlotBytes - kTile16 : kSlotBytes) + (w2 ? kW2Bytes : 0));
                     if (w2) tma_load_5d(smem + kOffW2 + ((g / L) & 1) * kW2Bytes, &p.w2map, fb, 0, 0, h, 0, 0);
-                    chunk_load_boxes(p.order, p.T, p.grid_h, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
+                    const int w0 = chunk_w0(p.order, p.T, c);
+                    if ((p.order >> 1) != 0 && w0 >= 0 && w0 + kC <= p.T) {
+                        // column orders, chunk inside the sequence: its 64 tokens (down a column and
+                        // on into the next ones) as one im2col load per tensor; boxes per column
+                        // segment cost the TMA unit one request each and ran up to 1.9x slower
+                        const int x0 = w0 / p.grid_h, y0 = w0 - x0 * p.grid_h;
+                        if (!kSum) tma_load_im2col_5d(st + kQ, &p.cmaps[T_Q], fb, xk, y0, x0, h, b);
+                        tma_load_im2col_5d(st + kK, &p.cmaps[T_K], fb, xk, y0, x0, h, b);
+                        tma_load_im2col_5d(st + kV, &p.cmaps[T_V], fb, xv, y0, x0, h, b);
+                        tma_load_im2col_5d(st + kG, &p.cmaps[T_G], fb, GP ? 0 : xk, y0, x0, GP ? 0 : h, b);
+                    } else chunk_load_boxes(p.order, p.T, p.grid_h, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
                         if (!kSum) tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, xk, h, c2, c3, b);
                         tma_load_5d(st + kK + row * 128, &p.maps[T_K][hi], fb, xk, h, c2, c3, b);
                         tma_load_5d(st + kV + row * 128, &p.maps[T_V][hi], fb, xv, h, c2, c3, b);
@@ -1301,6 +1314,39 @@ bool encode_map(CUtensorMap *m, const void *ptr, const Problem &p, int width, in
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+PFN_cuTensorMapEncodeIm2col_v12000 get_encode_im2col() {
+    static PFN_cuTensorMapEncodeIm2col_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        cudaDriverEntryPointQueryResult q;
+        void *f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeIm2col", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeIm2col_v12000>(f);
+    });
+    return fn;
+}
+
+// Column orders' walk map: the tensor [B][T][H][D] (T = Hg x W tokens, row-major) seen as the
+// im2col dims (D, Hg, W, H, B), grid rows fastest: an im2col load of 64 pixels from (y, x, h, b)
+// walks down column x and on into the next columns, exactly the column scan.  64 channels per
+// pixel at c0 = 0 or 64 (channels past D load as zero); no filter window (all corners 0).
+bool encode_col_map(CUtensorMap *m, const void *ptr, const Problem &p, int H, int width) {
+    auto enc = get_encode_im2col();
+    if (!enc) return false;
+    const cuuint64_t es = 2, D = static_cast<cuuint64_t>(width);
+    cuuint64_t dims[5] = {D, (cuuint64_t)p.grid_h, (cuuint64_t)p.grid_w, (cuuint64_t)H, (cuuint64_t)p.B};
+    cuuint64_t strides[4] = {(cuuint64_t)p.grid_w * H * D * es, (cuuint64_t)H * D * es, D * es,
+                             (cuuint64_t)p.T * H * D * es};
+    int lower[3] = {0, 0, 0}, upper[3] = {0, 0, 0};
+    cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    const CUtensorMapDataType dt = p.dtype == 1 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    return enc(m, dt, 5, const_cast<void *>(ptr), dims, strides, lower, upper, 64, kC, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Gate producer: W2 [H][r][Dk] as dims (Dk, r, H, 1, 1), box (64 channels, r rows): one head's
 // block lands as r rows of 128 bytes (SW128, MN-major B of Z = a W2); channels past Dk load as 0.
 bool encode_w2_map(CUtensorMap *m, const void *w2, int H, int Dk, int dtype) {
@@ -1318,7 +1364,7 @@ bool encode_w2_map(CUtensorMap *m, const void *w2, int H, int Dk, int dtype) {
 }
 
 // Encoded maps are cached per (pointers, shape, order, dtype): a repeated call
-// reuses them instead of encoding 32 maps again.
+// reuses them instead of encoding the maps again.
 struct MapKey {
     const void *ptr[kTensors];
     int B, H, grid_h, grid_w, order, dtype, Dk, Dv;
@@ -1327,12 +1373,13 @@ struct MapKey {
 struct MapEntry {
     MapKey key;
     CUtensorMap maps[kTensors][kHeights];
+    CUtensorMap cmaps[kTensors];  // column orders only
 };
 std::mutex g_map_mutex;
 std::list<MapEntry> g_map_cache;  // most recent first
 constexpr size_t kMapCacheSize = 32;
 
-bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
+bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights], CUtensorMap (&cout)[kTensors]) {
     MapKey key;
     std::memset(&key, 0, sizeof(key));
     key.ptr[T_Q] = p.q;
@@ -1351,6 +1398,7 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     for (auto it = g_map_cache.begin(); it != g_map_cache.end(); ++it) {
         if (it->key == key) {
             std::memcpy(out, it->maps, sizeof(out));
+            std::memcpy(cout, it->cmaps, sizeof(cout));
             g_map_cache.splice(g_map_cache.begin(), g_map_cache, it);
             return true;
         }
@@ -1360,7 +1408,12 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights]) {
     for (int t = 0; t < kTensors; ++t)
         for (int hi = 0; hi < kHeights; ++hi)
             if (!encode_map(&e.maps[t][hi], key.ptr[t], p, t == T_V ? p.Dv : p.Dk, box_height(hi))) return false;
+    std::memset(e.cmaps, 0, sizeof(e.cmaps));
+    if ((p.order >> 1) != 0)
+        for (int t = 0; t < kTensors; ++t)
+            if (!encode_col_map(&e.cmaps[t], key.ptr[t], p, p.H, t == T_V ? p.Dv : p.Dk)) return false;
     std::memcpy(out, e.maps, sizeof(out));
+    std::memcpy(cout, e.cmaps, sizeof(cout));
     g_map_cache.push_front(e);
     if (g_map_cache.size() > kMapCacheSize) g_map_cache.pop_back();
     return true;
@@ -1562,7 +1615,7 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
                       const Gate *gate, bool *gate_fused) {
     if (gate_fused) *gate_fused = false;
     TcParams tp;
-    if (!get_maps(p, tp.maps)) return cudaErrorInvalidValue;
+    if (!get_maps(p, tp.maps, tp.cmaps)) return cudaErrorInvalidValue;
     int n_sm = 0;
     cudaError_t e = sm_count(&n_sm);
     if (e != cudaSuccess) return e;
@@ -1679,11 +1732,12 @@ cudaError_t launch_tc_gate(const Problem &p, const GateSource &gs, cudaStream_t 
     // elements are zero-filled, so the a tile has 128-byte rows like the other tiles)
     Problem pq = p;
     pq.g = p.q;
-    if (!get_maps(pq, tp.maps)) return cudaErrorInvalidValue;
+    if (!get_maps(pq, tp.maps, tp.cmaps)) return cudaErrorInvalidValue;
     Problem pa = p;
     pa.H = 1;
     for (int hi = 0; hi < kHeights; ++hi)
         if (!encode_map(&tp.maps[T_G][hi], gs.a_low, pa, kRank, box_height(hi))) return cudaErrorInvalidValue;
+    if ((p.order >> 1) != 0 && !encode_col_map(&tp.cmaps[T_G], gs.a_low, p, 1, kRank)) return cudaErrorInvalidValue;
     if (!encode_w2_map(&tp.w2map, gs.w2, p.H, p.Dk, p.dtype)) return cudaErrorInvalidValue;
     tp.gbias = gs.bias;
     tp.tau_inv = 1.f / gs.tau;

@@ -129,6 +129,20 @@ __device__ __forceinline__ void tma_load_5d(void *dst, const CUtensorMap *m, uin
         "r"(smem_u32(bar))
         : "memory");
 }
+// 5-D im2col load global -> shared with zero filter offsets: the map's pixelsPerColumn
+// pixels from coordinate (c1, c2, c3, c4) on, its dimension 1 fastest and wrapping into
+// dimensions 2, 3 and 4 (channels c0 ... c0 + channelsPerPixel - 1 of each pixel, one row
+// each), completion counted on `bar` (tx bytes).
+__device__ __forceinline__ void tma_load_im2col_5d(void *dst, const CUtensorMap *m, uint64_t *bar, int c0,
+                                                   int c1, int c2, int c3, int c4) {
+    const uint16_t zero = 0;
+    asm volatile(
+        "cp.async.bulk.tensor.5d.shared::cluster.global.im2col.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5, %6}], [%7], {%8, %8, %8};" ::"r"(smem_u32(dst)),
+        "l"(reinterpret_cast<uint64_t>(m)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4),
+        "r"(smem_u32(bar)), "h"(zero)
+        : "memory");
+}
 // 5-D tiled prefetch global -> L2 (no shared memory, no completion to wait for).
 __device__ __forceinline__ void tma_prefetch_5d(const CUtensorMap *m, int c0, int c1, int c2, int c3, int c4) {
     asm volatile("cp.async.bulk.prefetch.tensor.5d.L2.global.tile [%0, {%1, %2, %3, %4, %5}];" ::"l"(
