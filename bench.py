@@ -9,6 +9,11 @@ H=12, Dk=Dv=64, bf16, scan order alternating per step across the four
 orders).  Prints ONE JSON line on rank 0.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload ID] [--impl reference]
+                  [--launch graph|eager]
+
+The K timed steps are captured once into one CUDA graph and replayed between two CUDA
+events (the default, --launch graph); the same steps as eager calls, each between its
+own events, are timed as well and reported as roofline.eager.
 
 Multi-GPU (torchrun, one rank per GPU): every rank runs its own batch of the
 same workload (weak scaling, no collective on the data path); value = tokens
@@ -50,8 +55,12 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
-    ap.add_argument("--graph", action="store_true",
-                    help="replay each step from a CUDA graph (one per scan order) instead of eager calls")
+    ap.add_argument("--launch", default="graph", choices=["graph", "eager"],
+                    help="graph (default): the K timed steps are captured once into one CUDA graph "
+                         "(through the caller-workspace entry points) and replayed, as the paper times its "
+                         "operator (Sec. 3.3); the eager per-step loop is timed as well and reported beside it. "
+                         "eager: one eager call per step, each bracketed by CUDA events")
+    ap.add_argument("--graph", action="store_true", help="same as --launch graph")
     ap.add_argument("--op", default="mixer", choices=["mixer", "sswiglu"],
                     help="mixer: the chunkwise GLA token mixer (default); sswiglu: the Spatial SwiGLU "
                          "gate-and-depthwise-conv step (Eq. spatial_swiglu) on --sw-workload")
@@ -63,7 +72,12 @@ def parse():
                     help="skip the 6400-token workload the default run also times")
     ap.add_argument("--batch", type=int, default=None,
                     help="override the workload's batch size (smaller cases for profiling)")
-    return ap.parse_args()
+    args = ap.parse_args()
+    if args.graph:
+        args.launch = "graph"
+    if args.schedule != "auto":  # the graph is captured through the automatic schedule's entry points
+        args.launch = "eager"
+    return args
 
 
 def dist_env():
@@ -137,7 +151,8 @@ def workload_config(w: wl.Workload, world: int, args=None, extra=None):
            "parallelism": f"replicas x{world} (independent batches, no collective)"}
     if args is not None:
         cfg["schedule"] = args.schedule
-        cfg["launch"] = "cuda-graph replay" if args.graph else "eager"
+        cfg["launch"] = ("one CUDA graph of the timed steps, replayed once" if args.launch == "graph"
+                         else "eager, CUDA events around each step")
         if args.gated:
             cfg["epilogue"] = "output gate u = SiLU(r) * RMSNorm(o), second kernel right after the mixer"
         if getattr(args, "gate_producer", False):
@@ -376,7 +391,9 @@ def run_sswiglu(args, rank: int, world: int, local: int):
     tpath = os.path.join(ROOT, "profiles", "traffic.json")
     if os.path.exists(tpath):
         with open(tpath) as f:
-            traffic = json.load(f).get(f"{sw.name}:sswiglu")
+            entry = json.load(f).get(f"{sw.name}:sswiglu")
+            if isinstance(entry, dict):
+                traffic = entry.get("dram_bytes")
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
                 "traffic": traffic, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs)" if src == "measured"
                 else "fallback", "kernel": "sswiglu_kernel (TMA value box with zero-padding halo, TMA gate box)",
@@ -544,34 +561,39 @@ def time_mixer(args, w: wl.Workload, rank: int, world: int, local: int, dev, pg)
     if gla.sync_status() != 0:
         raise RuntimeError("device status word set during warm-up")
 
-    run = step
-    if args.graph:
-        # one graph per (buffer set, scan order) pair of the rotation, captured through the
-        # caller-workspace entry points (no allocation, no synchronisation)
-        if schedule != "auto":
-            raise SystemExit("--graph times the automatic schedule only")
+    if args.launch == "graph":
+        # the K timed steps captured once into one CUDA graph through the caller-workspace entry
+        # points (no allocation, no synchronisation), rotating buffer sets and scan orders as
+        # the eager loop does; replayed once untimed (upload), then once timed
         ws = torch.empty(ws_n, dtype=torch.uint8, device=dev) if ws_n else None
-        n_graph = n_sets * len(orders) // math.gcd(n_sets, len(orders))
+        for i in range(max(3, args.warmup)):
+            s = sets[i % n_sets]
+            call(s, orders[i % len(orders)], ws=ws, graph=True)
+        torch.cuda.synchronize()
         cap = torch.cuda.Stream(dev)
         cap.wait_stream(stream)
-        graphs = []
+        graph = torch.cuda.CUDAGraph()
         with torch.cuda.stream(cap):
-            for j in range(n_graph):
-                g = torch.cuda.CUDAGraph()
-                with torch.cuda.graph(g, stream=cap):
-                    call(sets[j % n_sets], orders[j % len(orders)], strm=cap, ws=ws, graph=True)
-                graphs.append(g)
+            with torch.cuda.graph(graph, stream=cap):
+                for i in range(args.steps):
+                    call(sets[i % n_sets], orders[i % len(orders)], strm=cap, ws=ws, graph=True)
         stream.wait_stream(cap)
-        for j in range(max(3, args.warmup)):
-            graphs[j % n_graph].replay()
+        graph.replay()
         torch.cuda.synchronize()
         if gla.sync_status() != 0:
             raise RuntimeError("device status word set during graph warm-up")
-
-        def run(i):
-            graphs[i % n_graph].replay()
-
-    total_ms, per_launch_ms, clocks = timed_loop(run, args.steps, stream, not args.no_clocks, local, pg)
+        total_ms, _, clocks = timed_loop(lambda i: graph.replay(), 1, stream, not args.no_clocks, local, pg)
+        per_launch_ms = [total_ms / args.steps] * args.steps
+        timing = "CUDA events around one replay of the graph of all timed steps, divided by the steps"
+        # the same steps as eager calls, for comparison (not the headline)
+        e_total, e_per, _ = timed_loop(step, args.steps, stream, False, local, pg)
+        eager = {"ms_per_step": max_over_ranks(e_total, pg, dev) / args.steps,
+                 "kernel_ms": sum(e_per) / len(e_per),
+                 "timing": "CUDA events around each eager step"}
+    else:
+        total_ms, per_launch_ms, clocks = timed_loop(step, args.steps, stream, not args.no_clocks, local, pg)
+        timing = "CUDA events around each step on the launching stream"
+        eager = None
     if gla.sync_status() != 0:
         raise RuntimeError("device status word set during the timed region")
     total_ms = max_over_ranks(total_ms, pg, dev)
@@ -600,7 +622,9 @@ def time_mixer(args, w: wl.Workload, rank: int, world: int, local: int, dev, pg)
                 "frac": achieved / hbm_peak, "traffic": traffic,
                 "peak_source": f"{peak_src} (MEASURED_PEAKS.json hbm_gbs)" if peak_src == "measured" else "fallback",
                 "kernel": kernel_name, "kernel_ms": kernel_ms, "algorithmic_bytes_per_launch": alg_bytes,
-                "timing": "CUDA events around each step on the launching stream"}
+                "timing": timing}
+    if eager is not None:
+        roofline["eager"] = dict(eager, frac=alg_bytes / (eager["kernel_ms"] * 1e-3) / 1e9 / hbm_peak)
     if traffic_note:
         roofline["traffic_note"] = traffic_note
     return {"w": w, "inp": inp, "sets": sets, "value": value, "ms_per_step": ms_per_step,

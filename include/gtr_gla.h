@@ -158,9 +158,11 @@ gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, in
 int gtr_gla_balanced_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm);
 
 /* Introspection of the scan-order gather (Sec. 3.1, directional scanning): the
- * TMA boxes the tensor-core schedule loads for 64-token chunk c of a sequence
- * on a grid_h x grid_w patch grid, computed on the host by the same code the
- * kernel's producer runs.  Writes min(count, cap) boxes of 4 ints to `boxes`:
+ * TMA boxes of 64-token chunk c of a sequence on a grid_h x grid_w patch grid,
+ * computed on the host by the same code the kernel's producer runs.  The
+ * tensor-core schedule loads a chunk as these boxes unless gtr_gla_chunk_walk
+ * returns 1 for it (column-order chunks inside the sequence load as one walk).
+ * Writes min(count, cap) boxes of 4 ints to `boxes`:
  * rows (1-64), first row of the chunk's 64-row shared-memory tile, and the two
  * token coordinates of the box's first row (row orders: token index, 0; column
  * orders: column x, row y; x == grid_w marks a box that lies wholly outside the
@@ -168,6 +170,17 @@ int gtr_gla_balanced_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, 
  * all-zero padding chunks of a split's last segment.  Returns the chunk's box
  * count, or -1 for invalid arguments.  No device is used. */
 int gtr_gla_chunk_boxes(int grid_h, int grid_w, gtr_scan_t scan_order, int c, int *boxes, int cap);
+
+/* Whether the tensor-core schedule loads 64-token chunk c as one walk (Sec. 3.1,
+ * directional scanning): for a column order and a chunk wholly inside the
+ * sequence, each tensor's 64 tokens come in one TMA im2col load that starts at
+ * grid column *x, row *y (the chunk's first walk position; reverse orders load the
+ * forward range their chunk covers) and runs down that column and on into the
+ * next ones.  Returns 1 and sets *x, *y in that case; 0 when the chunk loads as
+ * the boxes of gtr_gla_chunk_boxes (row orders; chunks reaching past either end of
+ * the sequence); -1 for invalid arguments (x and y must not be NULL).  Computed on
+ * the host by the producer's own test; no device is used. */
+int gtr_gla_chunk_walk(int grid_h, int grid_w, gtr_scan_t scan_order, int c, int *x, int *y);
 
 /* gtr_gla_fwd with a caller-owned device workspace of workspace_bytes >=
  * gtr_gla_workspace_bytes() bytes, 256-byte aligned (may be NULL when that is

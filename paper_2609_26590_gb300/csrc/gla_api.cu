@@ -235,6 +235,14 @@ int gtr_gla_chunk_boxes(int grid_h, int grid_w, gtr_scan_t scan_order, int c, in
     return gtr::tc_chunk_boxes(scan_order, static_cast<int>(T), grid_h, grid_w, c, boxes, cap);
 }
 
+int gtr_gla_chunk_walk(int grid_h, int grid_w, gtr_scan_t scan_order, int c, int *x, int *y) {
+    if (grid_h < 1 || grid_w < 1 || (long long)grid_h * grid_w > 0x7fffffffLL) return -1;
+    if (scan_order < GTR_SCAN_ROW_FWD || scan_order > GTR_SCAN_COL_REV || c < 0 || !x || !y) return -1;
+    const long long T = (long long)grid_h * grid_w;
+    if ((long long)c * 64 > T + (1LL << 24)) return -1;  // far past the sequence: no schedule asks
+    return gtr::tc_chunk_walk(scan_order, static_cast<int>(T), grid_h, c, x, y);
+}
+
 gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm, int *nseg,
                                 int *seg_len) {
     if (!nseg || !seg_len || n_sm < 1) return GTR_ERR_INVALID_ARG;

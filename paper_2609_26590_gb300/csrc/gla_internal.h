@@ -38,6 +38,7 @@ bool tc_supported(const Problem &p);
 // enumeration, run on the host): up to cap boxes of 4 ints (rows, shared-memory row,
 // coordinate 2, coordinate 3); returns how many the chunk has.
 int tc_chunk_boxes(int order, int T, int grid_h, int grid_w, int c, int *boxes, int cap);
+int tc_chunk_walk(int order, int T, int grid_h, int c, int *x0, int *y0);
 // Segments per sequence and chunks per segment the tensor-core schedule uses for
 // this problem on a device with n_sm SMs (host arithmetic only; nseg 1: unsplit).
 void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len);

@@ -382,6 +382,17 @@ __host__ __device__ __forceinline__ void chunk_load_boxes(int order, int T, int 
     }
 }
 
+// Column orders, chunk c wholly inside the sequence: its 64 tokens (down column x0 from row y0
+// and on into the next columns) load as one im2col walk per tensor; returns false for row orders
+// and for chunks that reach past either end, which load boxes (chunk_load_boxes).
+__host__ __device__ __forceinline__ bool chunk_walk_start(int order, int T, int grid_h, int c, int *x0, int *y0) {
+    const int w0 = chunk_w0(order, T, c);
+    if ((order >> 1) == 0 || w0 < 0 || w0 + kC > T) return false;
+    *x0 = w0 / grid_h;
+    *y0 = w0 - *x0 * grid_h;
+    return true;
+}
+
 // fp16-pair mask of score columns 2e, 2e + 1 from a bit set of kept columns
 __device__ __forceinline__ uint32_t pmask(uint32_t vbits, int e) {
     return (((vbits >> (2 * e)) & 1u) ? 0x0000FFFFu : 0u) | (((vbits >> (2 * e + 1)) & 1u) ? 0xFFFF0000u : 0u);
@@ -635,12 +646,11 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     const bool w2 = GP && ps.cl == 0;
                     mbar_arrive_expect_tx(fb, (kSum ? kSlotBytes - kTile16 : kSlotBytes) + (w2 ? kW2Bytes : 0));
                     if (w2) tma_load_5d(smem + kOffW2 + ((g / L) & 1) * kW2Bytes, &p.w2map, fb, 0, 0, h, 0, 0);
-                    const int w0 = chunk_w0(p.order, p.T, c);
-                    if ((p.order >> 1) != 0 && w0 >= 0 && w0 + kC <= p.T) {
-                        // column orders, chunk inside the sequence: its 64 tokens (down a column and
-                        // on into the next ones) as one im2col load per tensor; boxes per column
-                        // segment cost the TMA unit one request each and ran up to 1.9x slower
-                        const int x0 = w0 / p.grid_h, y0 = w0 - x0 * p.grid_h;
+                    int x0, y0;
+                    if (chunk_walk_start(p.order, p.T, p.grid_h, c, &x0, &y0)) {
+                        // column orders, chunk inside the sequence: one im2col walk per tensor
+                        // (boxes per column segment cost the TMA unit one request each and ran
+                        // up to 1.9x slower)
                         if (!kSum) tma_load_im2col_5d(st + kQ, &p.cmaps[T_Q], fb, xk, y0, x0, h, b);
                         tma_load_im2col_5d(st + kK, &p.cmaps[T_K], fb, xk, y0, x0, h, b);
                         tma_load_im2col_5d(st + kV, &p.cmaps[T_V], fb, xv, y0, x0, h, b);
@@ -1585,6 +1595,10 @@ int tc_chunk_boxes(int order, int T, int grid_h, int grid_w, int c, int *boxes, 
         ++n;
     });
     return n;
+}
+
+int tc_chunk_walk(int order, int T, int grid_h, int c, int *x0, int *y0) {
+    return chunk_walk_start(order, T, grid_h, c, x0, y0) ? 1 : 0;
 }
 
 void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len) {

@@ -59,6 +59,8 @@ def load(path: Optional[str] = None):
         lib.gtr_sswiglu_dwconv.argtypes = [vp, vp, ctypes.c_longlong, vp, vp] + [ci] * 5 + [vp, vp]
         lib.gtr_gla_chunk_boxes.restype = ci
         lib.gtr_gla_chunk_boxes.argtypes = [ci] * 4 + [ctypes.POINTER(ci), ci]
+        lib.gtr_gla_chunk_walk.restype = ci
+        lib.gtr_gla_chunk_walk.argtypes = [ci] * 4 + [ctypes.POINTER(ci)] * 2
         lib.gtr_gla_split_plan.restype = ci
         lib.gtr_gla_split_plan.argtypes = [ci] * 7 + [ctypes.POINTER(ci)] * 2
         lib.gtr_gla_balanced_plan.restype = ci
@@ -220,6 +222,18 @@ def chunk_boxes(grid_h: int, grid_w: int, order: int, c: int):
     if n < 0 or n > cap:
         raise ValueError(f"gtr_gla_chunk_boxes returned {n}")
     return [tuple(buf[4 * i:4 * i + 4]) for i in range(n)]
+
+
+def chunk_walk(grid_h: int, grid_w: int, order: int, c: int):
+    """(x, y) grid position where the producer's single im2col walk load of chunk c
+    starts, or None when the chunk loads as boxes, through ``gtr_gla_chunk_walk``
+    (host only)."""
+    lib = load()
+    x, y = ctypes.c_int(-1), ctypes.c_int(-1)
+    r = lib.gtr_gla_chunk_walk(grid_h, grid_w, order, c, ctypes.byref(x), ctypes.byref(y))
+    if r < 0:
+        raise ValueError(f"gtr_gla_chunk_walk returned {r}")
+    return (x.value, y.value) if r == 1 else None
 
 
 def forward_ws(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,

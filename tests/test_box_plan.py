@@ -5,7 +5,9 @@ For every chunk of every grid, in every order, including the all-zero padding
 chunks of a split's last segment: the boxes cover the chunk's 64 tile rows
 exactly once, each box holds the tokens of the chunk's scan positions in scan
 order, and a box with rows outside the sequence loads only zeros (it lies wholly
-outside the tensor).  No GPU is used."""
+outside the tensor).  Column-order chunks inside the sequence load as one im2col
+walk instead (gtr_gla_chunk_walk): its start and traversal give the same rows.
+No GPU is used."""
 import math
 
 import pytest
@@ -90,6 +92,39 @@ def test_every_chunk_of_many_grids(gla, order):
             check_chunk(gla, gh, gw, order, c)
 
 
+@pytest.mark.parametrize("order", wl.ALL_ORDERS, ids=wl.ORDER_NAMES)
+def test_walk_loads(gla, order):
+    # a chunk loads as one im2col walk exactly when it is a column-order chunk wholly inside the
+    # sequence; the walk starts at the grid position of the chunk's first walk position and its
+    # 64 pixels (down the column, then on into the next ones) are the rows its boxes would load
+    grids = [(gh, gw) for gh in (1, 2, 3, 7, 8, 25, 40, 44, 63, 64, 65, 80) for gw in (1, 3, 13, 40, 44)]
+    for gh, gw in grids:
+        T = gh * gw
+        N = math.ceil(T / C)
+        rev = order in (wl.ROW_REV, wl.COL_REV)
+        for c in range(N + 2):
+            w0 = T - C * (c + 1) if rev else C * c
+            walk = gla.chunk_walk(gh, gw, order, c)
+            inside = 0 <= w0 and w0 + C <= T
+            if order in (wl.ROW_FWD, wl.ROW_REV) or not inside:
+                assert walk is None, (gh, gw, order, c)
+                continue
+            assert walk == (w0 // gh, w0 % gh), (gh, gw, order, c, walk)
+            x, y = walk
+            pixels = []
+            for _ in range(C):                  # the im2col traversal: rows fastest, then columns
+                pixels.append((x, y))
+                y += 1
+                if y == gh:
+                    x, y = x + 1, 0
+            boxes = gla.chunk_boxes(gh, gw, order, c)
+            rows = {}
+            for nrows, r0, c2, c3 in boxes:
+                for i in range(nrows):
+                    rows[r0 + i] = (c2, c3 + i)
+            assert [rows[r] for r in range(C)] == pixels, (gh, gw, order, c)
+
+
 def test_padding_chunks_load_only_zeros(gla):
     for gh, gw in [(44, 44), (40, 40), (5, 7), (64, 1)]:
         T = gh * gw
@@ -112,3 +147,10 @@ def test_rejects_invalid_arguments(gla):
     assert lib.gtr_gla_chunk_boxes(4, 4, 0, -1, buf, 2) == -1
     assert lib.gtr_gla_chunk_boxes(4, 4, 0, 0, None, 2) == -1
     assert lib.gtr_gla_chunk_boxes(4, 4, 2, 0, None, 0) >= 1     # count only
+    x, y = ctypes.c_int(), ctypes.c_int()
+    assert lib.gtr_gla_chunk_walk(0, 4, 2, 0, ctypes.byref(x), ctypes.byref(y)) == -1
+    assert lib.gtr_gla_chunk_walk(4, 4, 9, 0, ctypes.byref(x), ctypes.byref(y)) == -1
+    assert lib.gtr_gla_chunk_walk(4, 4, 2, -1, ctypes.byref(x), ctypes.byref(y)) == -1
+    assert lib.gtr_gla_chunk_walk(4, 4, 2, 0, None, ctypes.byref(y)) == -1
+    assert lib.gtr_gla_chunk_walk(16, 16, 2, 1, ctypes.byref(x), ctypes.byref(y)) == 1
+    assert (x.value, y.value) == (4, 0)
