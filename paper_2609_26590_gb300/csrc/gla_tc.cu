@@ -294,41 +294,34 @@ __device__ __forceinline__ StreamPos stream_pos(int v, int L, int nh, int lognv,
 // unit its range starts in, from the state the previous CTA handed over at the start of
 // its own run (long before).
 struct BalRange {
-    int u_lo, c_lo, u_hi, c_hi, u_first, n_full, G;
+    int base_head, base_full, base_tail;  // flattened chunk index = v + the base of v's piece
+    int c_hi, t0;                         // pieces: [0, c_hi) head, [c_hi, t0) whole units, [t0, G) tail
+    int G;
 };
 __device__ __forceinline__ BalRange bal_range(int N, int n_units) {
     const long long tot = static_cast<long long>(n_units) * N;
     const long long lo = tot * blockIdx.x / gridDim.x, hi = tot * (blockIdx.x + 1) / gridDim.x;
+    const int u_lo = static_cast<int>(lo / N), c_lo = static_cast<int>(lo - static_cast<long long>(u_lo) * N);
+    const int u_hi = static_cast<int>(hi / N), c_hi = static_cast<int>(hi - static_cast<long long>(u_hi) * N);
+    const int u_first = c_lo ? u_lo + 1 : u_lo;
     BalRange r;
-    r.u_lo = static_cast<int>(lo / N);
-    r.c_lo = static_cast<int>(lo - static_cast<long long>(r.u_lo) * N);
-    r.u_hi = static_cast<int>(hi / N);
-    r.c_hi = static_cast<int>(hi - static_cast<long long>(r.u_hi) * N);
-    r.u_first = r.c_lo ? r.u_lo + 1 : r.u_lo;
-    r.n_full = (r.u_hi - r.u_first) * N;
+    r.c_hi = c_hi;
+    r.t0 = c_hi + (u_hi - u_first) * N;
+    r.base_head = u_hi * N;                          // head: chunk v of unit u_hi
+    r.base_full = u_first * N - c_hi;                // whole units from u_first on
+    r.base_tail = static_cast<int>(lo) - r.t0;       // tail: chunk c_lo + (v - t0) of unit u_lo
     r.G = static_cast<int>(hi - lo);
     return r;
 }
-__device__ __forceinline__ StreamPos stream_pos_bal(int v, int N, int lognv, const BalRange &r) {
-    int unit, c;
-    bool start, hin = false, hout = false;
-    if (v < r.c_hi) {
-        unit = r.u_hi;
-        c = v;
-        start = v == 0;
-        hout = v == r.c_hi - 1;
-    } else if (v - r.c_hi < r.n_full) {
-        const int w = v - r.c_hi, k = w / N;
-        unit = r.u_first + k;
-        c = w - k * N;
-        start = c == 0;
-    } else {
-        const int w = v - r.c_hi - r.n_full;
-        unit = r.u_lo;
-        c = r.c_lo + w;
-        start = hin = w == 0;
-    }
-    return {unit >> lognv, unit & ((1 << lognv) - 1), c, 0, 0, c, start, hin, hout};
+// The piece is picked by two compares and the unit by one division, like the round-robin
+// decode; a three-way branch over the pieces made every role's per-chunk decode slower and
+// cost the whole kernel 10 %.
+__device__ __forceinline__ StreamPos stream_pos_bal(int v, int N, int lognv, int base_head, int base_full,
+                                                    int base_tail, int c_hi, int t0) {
+    const int g = v + (v < c_hi ? base_head : (v < t0 ? base_full : base_tail));
+    const int unit = g / N, c = g - unit * N;
+    const bool hin = v == t0;  // the tail's first chunk (t0 == G when there is no tail)
+    return {unit >> lognv, unit & ((1 << lognv) - 1), c, 0, 0, c, c == 0 || hin, hin, v == c_hi - 1};
 }
 
 // Visit the TMA load boxes of one chunk: calls f(map height index, smem row, c2, c3).
@@ -566,12 +559,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     // consecutive units flow through one pipeline
     BalRange br{};
     if constexpr (kBal) br = bal_range(N, p.n_units);
+    const int b_head = br.base_head, b_full = br.base_full, b_tail = br.base_tail, b_chi = br.c_hi, b_t0 = br.t0;
     const int G = kBal ? br.G
                        : L * nh *
                              ((p.n_units - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
                               static_cast<int>(gridDim.x));
     auto pos = [&](int v) -> StreamPos {
-        if constexpr (kBal) return stream_pos_bal(v, N, lognv, br);
+        if constexpr (kBal) return stream_pos_bal(v, N, lognv, b_head, b_full, b_tail, b_chi, b_t0);
         else return stream_pos(v, L, nh, lognv, kSplit ? p.nsu : 1);
     };
     const int rev = p.order & 1;
@@ -1567,6 +1561,7 @@ bool choose_balanced(const Problem &p, int n_sm) {
     if (pad64(p.Dk) != 64) return false;
     const long long units = (long long)p.B * p.H * (pad64(p.Dv) / 64);
     if (units <= n_sm) return false;
+    if (units * ((p.T + kC - 1) / kC) > 0x7fffffffLL) return false;  // the decode's flattened chunk index is an int
     const long long waves = (units + n_sm - 1) / n_sm;
     return waves * n_sm * 4 >= units * 5;  // ceil(U / SMs) >= 1.25 U / SMs
 }
