@@ -111,6 +111,7 @@ enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
 // by a range boundary handed from one CTA to the next; one key half).
 enum : int { kFull = 0, kSplitFull = 1, kSummary = 2, kBalanced = 3 };
 constexpr int kMinSegChunks = 2;          // a split segment keeps at least this many chunks
+constexpr uint32_t kBarSin = 4;           // named barrier: epi read the folded start state (ids 1-3: gen groups, epi)
 
 // Shared-memory map (byte offsets from a 1024-aligned base).
 constexpr int kSlotBytes = 4 * kTile16;                        // q @0, k @8K, v @16K, g @24K
@@ -613,6 +614,47 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         }
         fence_proxy_async_smem();
     }
+    // kSplitFull: the start state of the CTA's segment (a split launch gives every CTA one
+    // segment), folded from the summaries of the segments before it by all 512 threads, each
+    // taking 8 of a key half's 64 x 64 values and walking the summaries from the latest back
+    // (S_start = sum_s' (prod_{s' < s'' < seg} Diag(D_s'')) S_end(s'), Eq. chunk_boundary_main
+    // across segments) with several summaries' loads in flight.  A serial fold by the epi alone
+    // waited one L2 round trip per summary, about 8 us for the 13th segment.  The result lands in
+    // gen warpgroup 0's tf32 operand buffer, which the epi reads on entry; the group writes the
+    // buffer only after the epi's arrival on named barrier kBarSin.
+    if constexpr (MODE == kSplitFull) {
+        const StreamPos p0 = pos(0);
+        if (G > 0 && p0.seg > 0) {
+            float *sin = reinterpret_cast<float *>(smem + kOffOp);  // [NH][64 rows][64 columns] fp32
+            const size_t stride = (size_t)kDk * kDv + kDk;
+            const float *base = p.summary + (size_t)p0.bh * (p.nseg - 1) * stride;
+            const int r = threadIdx.x >> 3, col = (threadIdx.x & 7) * 8;
+#pragma unroll
+            for (int a = 0; a < NH; ++a) {
+                float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+                float coef = 1.f;
+#pragma unroll 4
+                for (int s2 = p0.seg - 1; s2 >= 0; --s2) {
+                    const float *bs = base + (size_t)s2 * stride;
+                    const float4 *x = reinterpret_cast<const float4 *>(bs + (size_t)(64 * a + r) * kDv + 64 * p0.vb + col);
+                    const float4 x0 = x[0], x1 = x[1];
+                    const float d = bs[(size_t)kDk * kDv + 64 * a + r];
+                    acc[0] = fmaf(coef, x0.x, acc[0]);
+                    acc[1] = fmaf(coef, x0.y, acc[1]);
+                    acc[2] = fmaf(coef, x0.z, acc[2]);
+                    acc[3] = fmaf(coef, x0.w, acc[3]);
+                    acc[4] = fmaf(coef, x1.x, acc[4]);
+                    acc[5] = fmaf(coef, x1.y, acc[5]);
+                    acc[6] = fmaf(coef, x1.z, acc[6]);
+                    acc[7] = fmaf(coef, x1.w, acc[7]);
+                    coef *= d;
+                }
+                float4 *dst = reinterpret_cast<float4 *>(sin + (64 * a + r) * 64 + col);
+                dst[0] = make_float4(acc[0], acc[1], acc[2], acc[3]);
+                dst[1] = make_float4(acc[4], acc[5], acc[6], acc[7]);
+            }
+        }
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -796,6 +838,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         // ======================================================= gen warpgroups (chunks c = gw mod 2)
         const int gw = (warp - 2) >> 2;          // 0: even chunks, 1: odd chunks
         const int bar_id = 1 + gw;
+        if constexpr (MODE == kSplitFull) {
+            if (gw == 0) named_barrier_sync(kBarSin, 256);  // the epi took the folded start state
+        }
         const int q4 = warp & 3, hc = lane >> 4;
         const int row = 16 * q4 + (lane & 15);   // smem row rho of this thread's accumulator row
         const int ch0 = 32 * hc;                 // its 32 key channels (A) / score columns (P)
@@ -1070,6 +1115,18 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 #pragma unroll
             for (int j = 0; j < 32; ++j) So[j] = 0.f;
         }
+        if constexpr (MODE == kSplitFull) {  // the start state the whole CTA folded (segments past the first)
+            if (G > 0 && pos(0).seg > 0) {
+                const float *sin = reinterpret_cast<const float *>(smem + kOffOp) + row * 64 + ch0;
+#pragma unroll
+                for (int j = 0; j < 32; ++j) S[j] = sin[j];
+                if constexpr (NH == 2) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) So[j] = sin[64 * 64 + j];
+                }
+            }
+            named_barrier_arrive(kBarSin, 256);  // gen warpgroup 0 may now use its operand buffer
+        }
         float dp = 1.f, dpo = 1.f;  // summaries: the segment's decay product per key half
         // Start state of a split sequence's segment seg > 0 (key half `half`): fold the
         // end states from zero of segments 0 .. seg-1 with their total decays,
@@ -1138,8 +1195,10 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                             for (int j = 0; j < 32; ++j) So[j] = 0.f;
                         }
                     } else if constexpr (kSplit) {
-                        start_state(S, 0, ps);
-                        if constexpr (NH == 2) start_state(So, 1, ps);
+                        if (MODE != kSplitFull || c != 0) {  // (c == 0: S holds the prologue's fold)
+                            start_state(S, 0, ps);
+                            if constexpr (NH == 2) start_state(So, 1, ps);
+                        }
                     }
                     dp = dpo = 1.f;
                 }

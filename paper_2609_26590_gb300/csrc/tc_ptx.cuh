@@ -90,6 +90,11 @@ __device__ __forceinline__ void fence_proxy_async_smem() {
 __device__ __forceinline__ void named_barrier_sync(uint32_t id, uint32_t nthreads) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
+// Arrive at a named barrier without waiting (the waiting side uses bar.sync with the
+// same thread count).
+__device__ __forceinline__ void named_barrier_arrive(uint32_t id, uint32_t nthreads) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
 // Named barrier that also ORs a predicate over the participating threads, so a
 // group takes a give-up decision uniformly (named barriers have no timeout: a
 // thread that left the loop alone would strand the others).
