@@ -111,6 +111,7 @@ enum : uint32_t { kModeF16 = 0, kModeTF32 = 1, kModeExact = 2 };
 // by a range boundary handed from one CTA to the next; one key half).
 enum : int { kFull = 0, kSplitFull = 1, kSummary = 2, kBalanced = 3 };
 constexpr int kMinSegChunks = 2;          // a split segment keeps at least this many chunks
+constexpr int kMaxUnsplitChunks = 5;      // shorter sequences are never split
 constexpr uint32_t kBarSin = 4;           // named barrier: epi read the folded start state (ids 1-3: gen groups, epi)
 
 // Shared-memory map (byte offsets from a 1024-aligned base).
@@ -1577,11 +1578,12 @@ int pad64(int d) { return (d + 63) / 64 * 64; }
 // SMs splits every sequence into segments of `len` chunks, so that the split
 // launch still fits one wave (units x ceil(N / len) <= SMs).  The split's critical
 // path is the last segment: `len` chunks in each of the two passes, plus the fold
-// of the nseg - 1 earlier summaries into its start state.  On a GB300 a chunk of
-// segment length costs about 2.5 us over both passes and a folded summary about
-// 0.55 us, so the length minimises 9 len + 2 ceil(N / len) + 10 (the second
-// launch), at least kMinSegChunks; the unsplit launch (about 6 per chunk) is
-// kept when it is cheaper.
+// of the nseg - 1 earlier summaries into its start state, which the output pass's
+// CTAs do together with many loads in flight.  A graph-replayed sweep of every
+// length on a GB300 (batch-1 and small-batch shapes, 64 <= N <= 256 chunks) fitted
+// about 1.95 us per chunk of length against 0.13 us per segment, so the length
+// minimises 15 len + ceil(N / len), at least kMinSegChunks.  Sequences of at most
+// kMaxUnsplitChunks chunks stay whole (5 chunks: 11.4 us whole, 13.4 us split).
 // The last segment may be shorter than the others: its chunks past the sequence
 // load as zeros (no key, decay 1), so they leave the state unchanged, and their
 // outputs are not stored.
@@ -1594,14 +1596,14 @@ Split choose_split(const Problem &p, int n_sm) {
     const long long N = (p.T + kC - 1) / kC;
     const long long units = (long long)p.B * p.H * (pad64(p.Dv) / 64);
     const Split none{1, static_cast<int>(N)};
-    if (units * 2 > n_sm) return none;
+    if (units * 2 > n_sm || N <= kMaxUnsplitChunks) return none;
     Split best = none;
-    long long best_cost = 6 * N;
+    long long best_cost = -1;
     for (long long L = kMinSegChunks; L < N; ++L) {
         const long long d = (N + L - 1) / L;
         if (units * d > n_sm) continue;
-        const long long cost = 9 * L + 2 * d + 10;
-        if (cost < best_cost) {
+        const long long cost = 15 * L + d;
+        if (best_cost < 0 || cost < best_cost) {
             best = Split{static_cast<int>(d), static_cast<int>(L)};
             best_cost = cost;
         }
@@ -1613,9 +1615,10 @@ Split choose_split(const Problem &p, int n_sm) {
 // round-robin deal would take at least 1.25 times the chunks per CTA of an even split,
 // every CTA takes an equal contiguous range of chunks instead.  Measured on a GB300
 // (graph-replayed, interleaved): B = 16, H = 12, 80 x 80, bf16 (192 units, ratio 1.58)
-// ran 1.23x faster balanced; B = 32, H = 12, 40 x 40 (384 units, ratio 1.19) 3 % slower
-// in bf16 and 4 % faster in fp16.  Units scattered over the CTAs cost about 8 % by
-// themselves (neighbouring CTAs no longer read the same token rows at the same time).
+// ran 1.23x faster balanced; B = 32, H = 12, 40 x 40 (384 units, ratio 1.19) 0.93x in
+// bf16 and 0.98x in fp16.  Contiguous ranges put every CTA at its own sequence and chunk,
+// so neighbouring CTAs no longer read the same token rows together: the loads then
+// stream at about 4.3 TB/s instead of 6.4 (copy-only probe of the same pattern).
 bool choose_balanced(const Problem &p, int n_sm) {
     if (pad64(p.Dk) != 64) return false;
     const long long units = (long long)p.B * p.H * (pad64(p.Dv) / 64);
