@@ -535,6 +535,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     volatile uint32_t *mode_s = reinterpret_cast<volatile uint32_t *>(smem + kOffMode);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // the output pass after a summary pass may start now: its CTAs set up (barriers, TMEM) on
+    // the free SMs and wait for this grid only before they read the summaries
+    if constexpr (MODE == kSummary) pdl_launch_dependents();
     // MODE kFull / kSplitFull: outputs (a split sequence's later segments start from
     // the state folded from the segment summaries).  MODE kSummary: per segment only
     // the end state from zero and the total decay (k, v and gates; no scores or outputs).
@@ -624,6 +627,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     // gen warpgroup 0's tf32 operand buffer, which the epi reads on entry; the group writes the
     // buffer only after the epi's arrival on named barrier kBarSin.
     if constexpr (MODE == kSplitFull) {
+        pdl_wait();  // the summaries are the previous grid's: this launch may start before it ends
         const StreamPos p0 = pos(0);
         if (G > 0 && p0.seg > 0) {
             float *sin = reinterpret_cast<float *>(smem + kOffOp);  // [NH][64 rows][64 columns] fp32
@@ -1484,7 +1488,7 @@ bool get_maps(const Problem &p, CUtensorMap (&out)[kTensors][kHeights], CUtensor
 }
 
 template <typename E, int NH, int NV, int MODE, bool GENOUT = false, bool GP = false, bool GATED = false>
-cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
+cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream, bool pdl = false) {
     // the shared-memory opt-in, once per process and device (setting it again is harmless)
     static std::atomic<unsigned long long> set_on_devices(0);
     int dev = 0;
@@ -1497,6 +1501,21 @@ cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
         if (e != cudaSuccess) return e;
         set_on_devices.fetch_or(bit);
     }
+    if (MODE == kSplitFull && pdl) {
+        // launched right after its summary pass: it may start while that grid runs (programmatic
+        // dependent launch) and waits for it before it reads the summaries
+        cudaLaunchAttribute attr;
+        attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr.val.programmaticStreamSerializationAllowed = 1;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = grid;
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = kSmemBytes;
+        cfg.stream = stream;
+        cfg.attrs = &attr;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, gla_tc_kernel<E, NH, NV, MODE, GENOUT, GP, GATED>, tp);
+    }
     gla_tc_kernel<E, NH, NV, MODE, GENOUT, GP, GATED><<<grid, kThreads, kSmemBytes, stream>>>(tp);
     return cudaSuccess;
 }
@@ -1504,15 +1523,17 @@ cudaError_t launch_kernel(dim3 grid, const TcParams &tp, cudaStream_t stream) {
 // One instantiation per (element type, key halves, value slices, pass).
 // gen_out: outputs stored by the gen warpgroups (fp16, one key half, outputs only)
 template <typename E, int MODE>
-cudaError_t launch_shape(dim3 grid, const TcParams &tp, cudaStream_t stream, bool gen_out = false) {
+cudaError_t launch_shape(dim3 grid, const TcParams &tp, cudaStream_t stream, bool gen_out = false, bool pdl = false) {
     if constexpr (std::is_same<E, __half>::value && MODE != kSummary) {
         if (gen_out && tp.nh == 1)
-            return tp.nv == 1 ? launch_kernel<E, 1, 1, MODE, true>(grid, tp, stream)
-                              : launch_kernel<E, 1, 2, MODE, true>(grid, tp, stream);
+            return tp.nv == 1 ? launch_kernel<E, 1, 1, MODE, true>(grid, tp, stream, pdl)
+                              : launch_kernel<E, 1, 2, MODE, true>(grid, tp, stream, pdl);
     }
     if (tp.nh == 1)
-        return tp.nv == 1 ? launch_kernel<E, 1, 1, MODE>(grid, tp, stream) : launch_kernel<E, 1, 2, MODE>(grid, tp, stream);
-    return tp.nv == 1 ? launch_kernel<E, 2, 1, MODE>(grid, tp, stream) : launch_kernel<E, 2, 2, MODE>(grid, tp, stream);
+        return tp.nv == 1 ? launch_kernel<E, 1, 1, MODE>(grid, tp, stream, pdl)
+                          : launch_kernel<E, 1, 2, MODE>(grid, tp, stream, pdl);
+    return tp.nv == 1 ? launch_kernel<E, 2, 1, MODE>(grid, tp, stream, pdl)
+                      : launch_kernel<E, 2, 2, MODE>(grid, tp, stream, pdl);
 }
 
 // kBalanced CTAs wait for their neighbour's hand-off: a cooperative launch guarantees
@@ -1721,10 +1742,12 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     const int seqs = static_cast<int>(p.B * p.H) * tp.nv;  // (sequence, value slice) pairs
     const bool half = p.dtype == 1;
     // persistent: one CTA per SM, each walking its share of the work units
+    unsigned sum_ctas = 0;
     if (nseg > 1) {  // pass 1: end state from zero and total decay of segments 0 .. nseg-2
         tp.nsu = nseg - 1;
         tp.n_units = seqs * tp.nsu;
         const dim3 grid(static_cast<unsigned>(tp.n_units < n_sm ? tp.n_units : n_sm));
+        sum_ctas = grid.x;
         e = half ? launch_shape<__half, kSummary>(grid, tp, stream) : launch_shape<__nv_bfloat16, kSummary>(grid, tp, stream);
         if (e != cudaSuccess) return e;
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -1768,10 +1791,14 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     // outputs from the gen warpgroups: fp16 launches of at most one wave (measured on a GB300:
     // +3 to +6 % there; with several units per CTA, or bf16, the epi storing them was faster)
     const bool gen_out = half && tp.n_units <= n_sm;
+    // the output pass of a split starts while its summary pass runs when both fit on the SMs at
+    // once (measured on a GB300: 1.04-1.06x at B = 1, H = 6, 40 x 40, 72 + 78 CTAs; with
+    // 96 + 128 CTAs at B = 2, H = 8, 128 x 128, Dk = Dv = 128, 0.95x)
+    const bool pdl = nseg > 1 && sum_ctas + grid.x <= static_cast<unsigned>(n_sm);
     if (fuse) {
         if (nseg > 1)
-            e = half ? launch_kernel<__half, 1, 1, kSplitFull, true, false, true>(grid, tp, stream)
-                     : launch_kernel<__nv_bfloat16, 1, 1, kSplitFull, true, false, true>(grid, tp, stream);
+            e = half ? launch_kernel<__half, 1, 1, kSplitFull, true, false, true>(grid, tp, stream, pdl)
+                     : launch_kernel<__nv_bfloat16, 1, 1, kSplitFull, true, false, true>(grid, tp, stream, pdl);
         else
             e = half ? launch_kernel<__half, 1, 1, kFull, true, false, true>(grid, tp, stream)
                      : launch_kernel<__nv_bfloat16, 1, 1, kFull, true, false, true>(grid, tp, stream);
@@ -1779,8 +1806,8 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
         return cudaGetLastError();
     }
     if (nseg > 1)
-        e = half ? launch_shape<__half, kSplitFull>(grid, tp, stream, gen_out)
-                 : launch_shape<__nv_bfloat16, kSplitFull>(grid, tp, stream);
+        e = half ? launch_shape<__half, kSplitFull>(grid, tp, stream, gen_out, pdl)
+                 : launch_shape<__nv_bfloat16, kSplitFull>(grid, tp, stream, false, pdl);
     else
         e = half ? launch_shape<__half, kFull>(grid, tp, stream, gen_out)
                  : launch_shape<__nv_bfloat16, kFull>(grid, tp, stream);

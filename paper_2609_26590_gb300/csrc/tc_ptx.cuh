@@ -111,6 +111,16 @@ __device__ __forceinline__ bool named_barrier_or(uint32_t id, uint32_t nthreads,
     return r != 0;
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// The grid launched after this one with programmatic stream serialisation may start now (its
+// CTAs take the SMs this grid leaves free); executed by every CTA of the primary grid.
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+// In such a dependent grid: wait until the grids before it completed and their memory
+// operations are visible (returns at once without a programmatic dependency).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ---------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap *m) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
