@@ -150,7 +150,7 @@ gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, in
 /* 1 when the tensor-core schedule balances these shapes on a device with n_sm SMs,
  * else 0 (also for invalid shapes or n_sm < 1).  Balanced: Dk <= 64, no sequence
  * split, more (sequence, 64-column value slice) units than SMs, and a round-robin
- * deal of whole units would give the busiest SM at least 1.25 times the chunks of an
+ * deal of whole units would give the busiest SM at least 1.1 times the chunks of an
  * even split; every
  * CTA then takes an equal contiguous range of the units' chunks, and a unit cut by
  * a range boundary continues from the state (Eq. chunk_boundary_main) the CTA

@@ -158,6 +158,33 @@ constexpr uint32_t kColA = 0, kColP = 128, kColU = 256, kColO = 384;
 
 enum { T_Q = 0, T_K = 1, T_V = 2, T_G = 3, kTensors = 4 };
 
+// Division by a launch constant 1 <= d < 2^31 of 0 <= n < 2^31 by a multiply-high and a
+// shift (Granlund and Montgomery, "Division by invariant integers using multiplication",
+// 1994, Thm. 4.2): with l = ceil(log2 d) and m = floor(2^32 (2^l - d) / d) + 1, the 33-bit
+// multiplier 2^32 + m satisfies 2^(32+l) < (2^32 + m) d <= 2^(32+l) + 2^l, so
+// n / d = (umulhi(n, m) + n) >> l, the sum exact in 32 bits for n < 2^31.  A few
+// instructions instead of an integer division's sequence: every role's per-chunk index
+// arithmetic uses it, which keeps the kernel's hot code small (the SM's instruction cache
+// is shared by all roles; the divisions of one decode cost a balanced launch 17 %).
+struct FastDiv {
+    int d;
+    uint32_t m, l;
+};
+inline FastDiv make_fastdiv(int d) {
+    if (d < 1) d = 1;
+    uint32_t l = 0;
+    while ((1ull << l) < static_cast<unsigned long long>(d)) ++l;
+    return FastDiv{d, static_cast<uint32_t>(((1ull << 32) * ((1ull << l) - d)) / d + 1), l};
+}
+__host__ __device__ __forceinline__ int fdiv(int n, const FastDiv &f) {
+#ifdef __CUDA_ARCH__
+    const uint32_t hi = __umulhi(static_cast<uint32_t>(n), f.m);
+#else
+    const uint32_t hi = static_cast<uint32_t>((static_cast<uint64_t>(static_cast<uint32_t>(n)) * f.m) >> 32);
+#endif
+    return static_cast<int>((hi + static_cast<uint32_t>(n)) >> f.l);
+}
+
 struct TcParams {
     CUtensorMap maps[kTensors][kHeights];  // box height box_height(i)
     CUtensorMap cmaps[kTensors];           // column orders: a chunk's 64-token walk as one im2col load
@@ -178,6 +205,8 @@ struct TcParams {
     unsigned long long *flags;             // kBalanced: per CTA, == epoch once its hand-off state (in
                                            // summary, [64][64] fp32 per CTA) is written; cleared when read
     unsigned long long epoch;              // kBalanced: nonzero, new for every launch
+    FastDiv fd_per, fd_nsu, fd_H, fd_gh, fd_L;  // division by L * nh, nsu, H, grid_h, L
+    FastDiv bal_n;                         // kBalanced: division by the chunks per sequence
     // gate producer (maps[T_G] then load the rank-16 projection a = x W1 instead of the gates)
     CUtensorMap w2map;                     // W2 [H][r][Dk], 16-bit, box (64 channels, r rows) SW128
     const float *gbias;                    // b [H][Dk] fp32
@@ -277,13 +306,13 @@ struct StreamPos {
 };
 // Units are (sequence, segment, value slice), the value slice fastest (the two
 // slices of a sequence read the same q, k and gates); a unit covers seg_len chunks.
-__device__ __forceinline__ StreamPos stream_pos(int v, int L, int nh, int lognv, int nsu) {
-    const int per = L * nh;
-    const int j = v / per, rem = v - j * per;
+__device__ __forceinline__ StreamPos stream_pos(int v, int L, int nh, int lognv, const FastDiv &per, bool split,
+                                                const FastDiv &nsu) {
+    const int j = fdiv(v, per), rem = v - j * per.d;
     const int unit = static_cast<int>(blockIdx.x) + j * static_cast<int>(gridDim.x);
     const int rest = unit >> lognv;
-    const int seg = nsu == 1 ? 0 : rest % nsu;
-    const int bh = nsu == 1 ? rest : rest / nsu;
+    const int bh = split ? fdiv(rest, nsu) : rest;
+    const int seg = split ? rest - bh * nsu.d : 0;
     const int cl = rem / nh;
     const int a = rem - cl * nh;
     return {bh, unit & ((1 << lognv) - 1), seg * L + cl, a, seg, cl, cl == 0 && a == 0, false, false};
@@ -315,15 +344,28 @@ __device__ __forceinline__ BalRange bal_range(int N, int n_units) {
     r.G = static_cast<int>(hi - lo);
     return r;
 }
-// The piece is picked by two compares and the unit by one division, like the round-robin
-// decode; a three-way branch over the pieces made every role's per-chunk decode slower and
-// cost the whole kernel 10 %.
+// The piece is picked by two compares and the unit by one multiply-high division; a
+// three-way branch over the pieces made every role's per-chunk decode slower and cost the
+// whole kernel 10 %, and an integer division here another 17 %.
 __device__ __forceinline__ StreamPos stream_pos_bal(int v, int N, int lognv, int base_head, int base_full,
-                                                    int base_tail, int c_hi, int t0) {
+                                                    int base_tail, int c_hi, int t0, const FastDiv &fn) {
     const int g = v + (v < c_hi ? base_head : (v < t0 ? base_full : base_tail));
-    const int unit = g / N, c = g - unit * N;
+    const int unit = fdiv(g, fn), c = g - unit * N;
     const bool hin = v == t0;  // the tail's first chunk (t0 == G when there is no tail)
     return {unit >> lognv, unit & ((1 << lognv) - 1), c, 0, 0, c, c == 0 || hin, hin, v == c_hi - 1};
+}
+
+// kBalanced: bounded wait for the previous CTA's hand-off flag.  Out of line: it runs once
+// per CTA, and inlined into the epi's loop it enlarged the kernel's hot code.
+__device__ __noinline__ bool handoff_wait(const volatile unsigned long long *f, unsigned long long epoch,
+                                          volatile uint32_t *abort_flag) {
+    bool got = *f == epoch;
+    const uint64_t t0 = global_timer_ns();
+    while (!got && !*abort_flag && global_timer_ns() - t0 < kWaitLimitNs) {
+        __nanosleep(64);
+        got = *f == epoch;
+    }
+    return got;
 }
 
 // Visit the TMA load boxes of one chunk: calls f(map height index, smem row, c2, c3).
@@ -336,7 +378,7 @@ __device__ __forceinline__ StreamPos stream_pos_bal(int v, int N, int lognv, int
 // segments), each loaded as at most two boxes: its multiple of 8 and the remainder.
 // One call site for f keeps the producer's issue code small.
 template <typename F>
-__host__ __device__ __forceinline__ void chunk_load_boxes(int order, int T, int grid_h, int grid_w, int c, F &&f) {
+__host__ __device__ __forceinline__ void chunk_load_boxes(int order, int T, const FastDiv &gh, int grid_w, int c, F &&f) {
     const int w0 = chunk_w0(order, T, c);
     if ((order >> 1) == 0) {
         f(kHeights - 1, 0, w0, 0);
@@ -361,8 +403,8 @@ __host__ __device__ __forceinline__ void chunk_load_boxes(int order, int T, int 
             len = w0 + kC - hi, row = hi - w0, c2 = grid_w, c3 = 0;
         } else {  // the next column segment
             if (w >= hi) break;
-            const int x = w / grid_h, y = w - x * grid_h;
-            len = grid_h - y;
+            const int x = fdiv(w, gh), y = w - x * gh.d;
+            len = gh.d - y;
             if (len > hi - w) len = hi - w;
             row = w - w0, c2 = x, c3 = y;
             w += len;
@@ -380,11 +422,11 @@ __host__ __device__ __forceinline__ void chunk_load_boxes(int order, int T, int 
 // Column orders, chunk c wholly inside the sequence: its 64 tokens (down column x0 from row y0
 // and on into the next columns) load as one im2col walk per tensor; returns false for row orders
 // and for chunks that reach past either end, which load boxes (chunk_load_boxes).
-__host__ __device__ __forceinline__ bool chunk_walk_start(int order, int T, int grid_h, int c, int *x0, int *y0) {
+__host__ __device__ __forceinline__ bool chunk_walk_start(int order, int T, const FastDiv &gh, int c, int *x0, int *y0) {
     const int w0 = chunk_w0(order, T, c);
     if ((order >> 1) == 0 || w0 < 0 || w0 + kC > T) return false;
-    *x0 = w0 / grid_h;
-    *y0 = w0 - *x0 * grid_h;
+    *x0 = fdiv(w0, gh);
+    *y0 = w0 - *x0 * gh.d;
     return true;
 }
 
@@ -394,11 +436,11 @@ __device__ __forceinline__ uint32_t pmask(uint32_t vbits, int e) {
 }
 
 // Spatial token of walk position w (-1 outside the sequence).
-__device__ __forceinline__ int walk_token(int order, int T, int grid_h, int grid_w, int w) {
+__device__ __forceinline__ int walk_token(int order, int T, const FastDiv &gh, int grid_w, int w) {
     if (w < 0 || w >= T) return -1;
     if ((order >> 1) == 0) return w;
-    const int x = w / grid_h;
-    return (w - x * grid_h) * grid_w + x;
+    const int x = fdiv(w, gh);
+    return (w - x * gh.d) * grid_w + x;
 }
 
 // Exact scores for one chunk (extreme or non-finite log-decays): serial prefix
@@ -570,8 +612,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                              ((p.n_units - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
                               static_cast<int>(gridDim.x));
     auto pos = [&](int v) -> StreamPos {
-        if constexpr (kBal) return stream_pos_bal(v, N, lognv, b_head, b_full, b_tail, b_chi, b_t0);
-        else return stream_pos(v, L, nh, lognv, kSplit ? p.nsu : 1);
+        if constexpr (kBal) return stream_pos_bal(v, N, lognv, b_head, b_full, b_tail, b_chi, b_t0, p.bal_n);
+        else return stream_pos(v, L, nh, lognv, p.fd_per, kSplit, p.fd_nsu);
     };
     const int rev = p.order & 1;
 
@@ -672,7 +714,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             for (int g = 0; g < G; ++g) {
                 const int sl = g % kSlots;
                 const StreamPos ps = pos(g);
-                const int b = ps.bh / p.H, h = ps.bh % p.H, c = ps.c;
+                const int b = fdiv(ps.bh, p.fd_H), h = ps.bh - b * p.H, c = ps.c;
                 const int xk = 64 * ps.a, xv = 64 * ps.vb;  // channel offsets of the key half, value slice
                 if (!mbar_wait(&bars[BAR_EMPTY + sl], ((g / kSlots) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
                     record_timeout(abort_flag);
@@ -686,9 +728,9 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     // ended at least four chunks earlier: its last Z completed before this slot freed)
                     const bool w2 = GP && ps.cl == 0;
                     mbar_arrive_expect_tx(fb, (kSum ? kSlotBytes - kTile16 : kSlotBytes) + (w2 ? kW2Bytes : 0));
-                    if (w2) tma_load_5d(smem + kOffW2 + ((g / L) & 1) * kW2Bytes, &p.w2map, fb, 0, 0, h, 0, 0);
+                    if (w2) tma_load_5d(smem + kOffW2 + (fdiv(g, p.fd_L) & 1) * kW2Bytes, &p.w2map, fb, 0, 0, h, 0, 0);
                     int x0, y0;
-                    if (chunk_walk_start(p.order, p.T, p.grid_h, c, &x0, &y0)) {
+                    if (chunk_walk_start(p.order, p.T, p.fd_gh, c, &x0, &y0)) {
                         // column orders, chunk inside the sequence: one im2col walk per tensor
                         // (boxes per column segment cost the TMA unit one request each and ran
                         // up to 1.9x slower)
@@ -696,7 +738,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         tma_load_im2col_5d(st + kK, &p.cmaps[T_K], fb, xk, y0, x0, h, b);
                         tma_load_im2col_5d(st + kV, &p.cmaps[T_V], fb, xv, y0, x0, h, b);
                         tma_load_im2col_5d(st + kG, &p.cmaps[T_G], fb, GP ? 0 : xk, y0, x0, GP ? 0 : h, b);
-                    } else chunk_load_boxes(p.order, p.T, p.grid_h, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
+                    } else chunk_load_boxes(p.order, p.T, p.fd_gh, p.grid_w, c, [&](int hi, int row, int c2, int c3) {
                         if (!kSum) tma_load_5d(st + kQ + row * 128, &p.maps[T_Q][hi], fb, xk, h, c2, c3, b);
                         tma_load_5d(st + kK + row * 128, &p.maps[T_K][hi], fb, xk, h, c2, c3, b);
                         tma_load_5d(st + kV + row * 128, &p.maps[T_V][hi], fb, xv, h, c2, c3, b);
@@ -753,7 +795,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                         // Z = a W2 (M = 64 tokens, N = 64 channels, K = r = 16: one MMA) into the
                         // chunk's A buffer; a tile K-major with 128-byte rows, W2 MN-major
                         const uint64_t da = kdesc(slot0 + (c % kSlots) * kSlotBytes + kG);
-                        const uint64_t dw = mndesc(smem_u32(smem + kOffW2) + ((c / L) & 1) * kW2Bytes);
+                        const uint64_t dw = mndesc(smem_u32(smem + kOffW2) + (fdiv(c, p.fd_L) & 1) * kW2Bytes);
                         mma_f16_ss_warp(tmem + kColA + (c & 1) * 64, da, dw, idesc_z, 0);
                         mma_commit_warp(&bars[BAR_ZFULL + (c & 1)]);
                     }
@@ -867,8 +909,8 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             tmem_ld_wait();
             uint32_t ow[16];
             const StreamPos po = pos(co);
-            const int b = po.bh / p.H, h = po.bh % p.H;
-            const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
+            const int b = fdiv(po.bh, p.fd_H), h = po.bh - b * p.H;
+            const int t = walk_token(p.order, p.T, p.fd_gh, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
             if constexpr (GATED) {
                 // u = SiLU(r) * o / sqrt(mean_j o_j^2 + eps) * w over the head's Dv outputs: this
                 // thread holds 32 of the row's columns, the lane 16 apart the other 32 (padded
@@ -931,7 +973,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 const StreamPos pz = pos(c);
                 const int wz = chunk_w0(p.order, p.T, pz.c) + row;
                 const bool live = wz >= 0 && wz < p.T;
-                const float *bz = p.gbias + (size_t)(pz.bh % p.H) * p.Dk;
+                const float *bz = p.gbias + (size_t)(pz.bh - fdiv(pz.bh, p.fd_H) * p.H) * p.Dk;
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     // 8 channels of the bias (Dk is a multiple of 8: all inside it or all past it)
@@ -1159,173 +1201,182 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
             mbar_arrive(&bars[BAR_PURDY + 0]);
             mbar_arrive(&bars[BAR_PURDY + 1]);
         }
-        for (int c = 0; ok && c <= G; ++c) {
-            if (c < G) {
-                const int sl = c % kSlots, bb = c & 1;
-                const uint32_t ph = (c >> 1) & 1;
-                const StreamPos ps = pos(c);
-                if (ps.start) {  // a run of a unit starts: its state (every key half)
-                    if (kBal && ps.hin) {
-                        // the previous CTA's hand-off (a bounded wait on its flag), then the flag
-                        // is cleared for the next launch
-                        const volatile unsigned long long *f = p.flags + blockIdx.x - 1;
-                        bool got = *f == p.epoch;
-                        const uint64_t t0 = global_timer_ns();
-                        while (!got && !*abort_flag && global_timer_ns() - t0 < kWaitLimitNs) {
-                            __nanosleep(64);
-                            got = *f == p.epoch;
-                        }
-                        if (named_barrier_or(3, 128, !got)) {  // the epi gives up together
-                            ok = false;
-                            break;
-                        }
-                        __threadfence();
-                        const float4 *x = reinterpret_cast<const float4 *>(p.summary + (size_t)(blockIdx.x - 1) * kD * kD +
-                                                                           (size_t)row * kD + ch0);
+        // kBalanced: the loop runs in three pieces (head run, whole units, tail run) with the
+        // hand-offs between them, so that the per-chunk loop itself carries no hand-off code
+        // (in the loop it slowed every chunk: the SM's instruction cache is shared by all roles)
+        const int cut0 = kBal ? b_chi : G + 1, cut1 = kBal ? b_t0 : G + 1;
+        int c = 0;
+#pragma unroll 1
+        for (int piece = 0; ok && piece < (kBal ? 3 : 1); ++piece) {
+            if (kBal && piece == 2 && b_t0 < G) {
+                // the tail run starts from the previous CTA's hand-off (a bounded wait on its
+                // flag, which is then cleared for the next launch)
+                const volatile unsigned long long *f = p.flags + blockIdx.x - 1;
+                const bool got = handoff_wait(f, p.epoch, abort_flag);
+                if (named_barrier_or(3, 128, !got)) {  // the epi gives up together
+                    ok = false;
+                    break;
+                }
+                __threadfence();
+                const float4 *x = reinterpret_cast<const float4 *>(p.summary + (size_t)(blockIdx.x - 1) * kD * kD +
+                                                                   (size_t)row * kD + ch0);
 #pragma unroll
-                        for (int j = 0; j < 8; ++j) {
-                            const float4 w = x[j];
-                            S[4 * j] = w.x;
-                            S[4 * j + 1] = w.y;
-                            S[4 * j + 2] = w.z;
-                            S[4 * j + 3] = w.w;
-                        }
-                        named_barrier_sync(3, 128);  // the epi's four warps read their rows
-                        if (threadIdx.x == 10 * 32) *const_cast<volatile unsigned long long *>(f) = 0ull;
-                    } else if (!kSplit || kSum || ps.seg == 0) {
+                for (int j = 0; j < 8; ++j) {
+                    const float4 w = __ldcg(x + j);  // from L2: another SM wrote it
+                    S[4 * j] = w.x;
+                    S[4 * j + 1] = w.y;
+                    S[4 * j + 2] = w.z;
+                    S[4 * j + 3] = w.w;
+                }
+                named_barrier_sync(3, 128);  // the epi's four warps read their rows
+                if (threadIdx.x == 10 * 32) *const_cast<volatile unsigned long long *>(f) = 0ull;
+            }
+            const int c_end = piece == 0 ? cut0 : (piece == 1 ? cut1 : G + 1);
+            for (; ok && c < c_end; ++c) {
+                if (c < G) {
+                    const int sl = c % kSlots, bb = c & 1;
+                    const uint32_t ph = (c >> 1) & 1;
+                    const StreamPos ps = pos(c);
+                    if (ps.start) {  // a run of a unit starts: its state (every key half)
+                        if (kBal && ps.hin) {
+                            // S holds the previous CTA's hand-off (taken before this piece)
+                        } else if (!kSplit || kSum || ps.seg == 0) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) S[j] = 0.f;
-                        if constexpr (NH == 2) {
+                            for (int j = 0; j < 32; ++j) S[j] = 0.f;
+                            if constexpr (NH == 2) {
 #pragma unroll
-                            for (int j = 0; j < 32; ++j) So[j] = 0.f;
+                                for (int j = 0; j < 32; ++j) So[j] = 0.f;
+                            }
+                        } else if constexpr (kSplit) {
+                            if (MODE != kSplitFull || c != 0) {  // (c == 0: S holds the prologue's fold)
+                                start_state(S, 0, ps);
+                                if constexpr (NH == 2) start_state(So, 1, ps);
+                            }
                         }
-                    } else if constexpr (kSplit) {
-                        if (MODE != kSplitFull || c != 0) {  // (c == 0: S holds the prologue's fold)
-                            start_state(S, 0, ps);
-                            if constexpr (NH == 2) start_state(So, 1, ps);
-                        }
+                        dp = dpo = 1.f;
                     }
-                    dp = dpo = 1.f;
-                }
-                bool fail = !mbar_wait(&bars[BAR_REFS + sl], (c / kSlots) & 1, abort_flag, kWaitLimitNs);
-                // buffer bb was last read by O(c-2) (epi outputs with one key half: observed by
-                // the readout of the previous iteration already)
-                if (!kSum && (NH == 2 || kGenOut) && c >= 2)
-                    fail = fail || !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs);
-                if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
-                    ok = false;
-                    break;
-                }
-                const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + sl * kRefFloats;
-                const bool fold = (mode_s[sl] == kModeF16);
-                const float c1 = fold ? ref[2 * kD + row] : 1.f;
-                const float c2 = fold ? ref[3 * kD + row] : 1.f;
-                const float dc = decay_s[sl * kD + row];
-                if (!kSum) {
-                    // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout)
-                    uint8_t *sb = smem + kOffS + bb * kTile16;
+                    bool fail = !mbar_wait(&bars[BAR_REFS + sl], (c / kSlots) & 1, abort_flag, kWaitLimitNs);
+                    // buffer bb was last read by O(c-2) (epi outputs with one key half: observed by
+                    // the readout of the previous iteration already)
+                    if (!kSum && (NH == 2 || kGenOut) && c >= 2)
+                        fail = fail || !mbar_wait(&bars[BAR_OFULL + bb], ph ^ 1, abort_flag, kWaitLimitNs);
+                    if (__any_sync(0xffffffffu, fail || *abort_flag != 0u)) {  // the warp leaves together
+                        ok = false;
+                        break;
+                    }
+                    const float *ref = reinterpret_cast<const float *>(smem + kOffRef) + sl * kRefFloats;
+                    const bool fold = (mode_s[sl] == kModeF16);
+                    const float c1 = fold ? ref[2 * kD + row] : 1.f;
+                    const float c2 = fold ? ref[3 * kD + row] : 1.f;
+                    const float dc = decay_s[sl * kD + row];
+                    if (!kSum) {
+                        // S'_[c] = Diag(c1) S_[c] (fp16, MN-major B of the readout)
+                        uint8_t *sb = smem + kOffS + bb * kTile16;
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        *reinterpret_cast<uint4 *>(sb + sw128(row, (ch0 + 8 * q) * 2)) = make_uint4(
-                            h2bits(S[8 * q + 0] * c1, S[8 * q + 1] * c1), h2bits(S[8 * q + 2] * c1, S[8 * q + 3] * c1),
-                            h2bits(S[8 * q + 4] * c1, S[8 * q + 5] * c1), h2bits(S[8 * q + 6] * c1, S[8 * q + 7] * c1));
-                    fence_proxy_async_smem();
+                        for (int q = 0; q < 4; ++q)
+                            *reinterpret_cast<uint4 *>(sb + sw128(row, (ch0 + 8 * q) * 2)) = make_uint4(
+                                h2bits(S[8 * q + 0] * c1, S[8 * q + 1] * c1), h2bits(S[8 * q + 2] * c1, S[8 * q + 3] * c1),
+                                h2bits(S[8 * q + 4] * c1, S[8 * q + 5] * c1), h2bits(S[8 * q + 6] * c1, S[8 * q + 7] * c1));
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // with the outputs of c-2 read out
+                    }
+                    // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
+                    fail = !mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs);
+                    if (__any_sync(0xffffffffu, fail)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    if constexpr (NH == 2) {  // two states live: read U in halves to save registers
+#pragma unroll
+                        for (int hf = 0; hf < 2; ++hf) {
+                            uint32_t r[16];
+                            tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16 * hf, r);
+                            tmem_ld_wait();
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) S[16 * hf + j] = fmaf(dc, S[16 * hf + j], c2 * __uint_as_float(r[j]));
+                        }
+                    } else {
+                        uint32_t r[32];
+                        tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
+                        tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
+                    }
+                    tc_fence_before();
+                    if (kSum) {
+                        dp *= dc;
+                        if (ps.cl == L - 1) {  // the segment's summary
+                            float *base = p.summary + ((size_t)ps.bh * (p.nseg - 1) + ps.seg) * sum_stride;
+                            float4 *dst = reinterpret_cast<float4 *>(base + (size_t)(64 * ps.a + row) * kDv + 64 * ps.vb + ch0);
+#pragma unroll
+                            for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
+                            if (ps.vb == 0 && hc == 0) base[(size_t)kDk * kDv + 64 * ps.a + row] = dp;
+                        }
+                    } else if (ps.c == N - 1 && p.final_state != nullptr && 64 * ps.a + row < p.Dk) {
+                        // the sequence's final state [Dk][Dv] (padded channels and columns stay behind)
+                        const int col0 = 64 * ps.vb + ch0;
+                        float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)ps.bh * p.Dk + 64 * ps.a + row) * p.Dv + col0);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            if (col0 + 4 * j < p.Dv) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
+                    }
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(&bars[BAR_ORDY + bb]);  // with the outputs of c-2 read out
+                    if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // U(c) drained: counts for chunk c + 2
+                    if constexpr (NH == 2) {  // the other key half comes next
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) {
+                            const float t = S[j];
+                            S[j] = So[j];
+                            So[j] = t;
+                        }
+                        const float t = dp;
+                        dp = dpo;
+                        dpo = t;
+                    }
                 }
-                // state carry: S_[c+1] = Diag(d_c) S_[c] + Diag(c2) U_c
-                fail = !mbar_wait(&bars[BAR_UFULL + bb], ph, abort_flag, kWaitLimitNs);
-                if (__any_sync(0xffffffffu, fail)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                if constexpr (NH == 2) {  // two states live: read U in halves to save registers
+                if (!kSum && !kGenOut && c >= nh && c % nh == 0) {
+                    // outputs of the real chunk whose last key half is c-1
+                    const int co = c - 1, ob = (co / nh) & 1;
+                    const bool fail = !mbar_wait(&bars[BAR_OFULL + (co & 1)], (co >> 1) & 1, abort_flag, kWaitLimitNs);
+                    if (__any_sync(0xffffffffu, fail)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    uint32_t ow[16];  // the row's 32 outputs packed in pairs
 #pragma unroll
                     for (int hf = 0; hf < 2; ++hf) {
                         uint32_t r[16];
-                        tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16 * hf, r);
+                        tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 16 * hf, r);
                         tmem_ld_wait();
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) S[16 * hf + j] = fmaf(dc, S[16 * hf + j], c2 * __uint_as_float(r[j]));
+                        for (int j = 0; j < 8; ++j) ow[8 * hf + j] = Elem<E>::pack(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
                     }
-                } else {
-                    uint32_t r[32];
-                    tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 0, *reinterpret_cast<uint32_t(*)[16]>(&r[0]));
-                    tmem_ld_16x32bx2_x16(tmem + lane_base + kColU + bb * 64 + 16, *reinterpret_cast<uint32_t(*)[16]>(&r[16]));
-                    tmem_ld_wait();
+                    tc_fence_before();
+                    const StreamPos po = pos(co);
+                    const int b = fdiv(po.bh, p.fd_H), h = po.bh - b * p.H;
+                    const int t = walk_token(p.order, p.T, p.fd_gh, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
+                    if (t >= 0) {  // the row's columns inside Dv (padded columns stay behind)
+                        const int col0 = 64 * po.vb + ch0;
+                        uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * p.Dv + col0);
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) S[j] = fmaf(dc, S[j], c2 * __uint_as_float(r[j]));
-                }
-                tc_fence_before();
-                if (kSum) {
-                    dp *= dc;
-                    if (ps.cl == L - 1) {  // the segment's summary
-                        float *base = p.summary + ((size_t)ps.bh * (p.nseg - 1) + ps.seg) * sum_stride;
-                        float4 *dst = reinterpret_cast<float4 *>(base + (size_t)(64 * ps.a + row) * kDv + 64 * ps.vb + ch0);
-#pragma unroll
-                        for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
-                        if (ps.vb == 0 && hc == 0) base[(size_t)kDk * kDv + 64 * ps.a + row] = dp;
+                        for (int q = 0; q < 4; ++q)
+                            if (col0 + 8 * q < p.Dv) dst[q] = make_uint4(ow[4 * q], ow[4 * q + 1], ow[4 * q + 2], ow[4 * q + 3]);
                     }
-                } else if (kBal && ps.hout) {  // the state at the end of the head run -> the next CTA
-                    float4 *dst = reinterpret_cast<float4 *>(p.summary + (size_t)blockIdx.x * kD * kD + (size_t)row * kD + ch0);
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
-                    __threadfence();
-                    named_barrier_sync(3, 128);  // the epi's four warps wrote their rows
-                    if (threadIdx.x == 10 * 32)
-                        *reinterpret_cast<volatile unsigned long long *>(p.flags + blockIdx.x) = p.epoch;
-                } else if (ps.c == N - 1 && p.final_state != nullptr && 64 * ps.a + row < p.Dk) {
-                    // the sequence's final state [Dk][Dv] (padded channels and columns stay behind)
-                    const int col0 = 64 * ps.vb + ch0;
-                    float4 *dst = reinterpret_cast<float4 *>(p.final_state + ((size_t)ps.bh * p.Dk + 64 * ps.a + row) * p.Dv + col0);
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        if (col0 + 4 * j < p.Dv) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&bars[BAR_PURDY + bb]);  // U(c) drained: counts for chunk c + 2
-                if constexpr (NH == 2) {  // the other key half comes next
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const float t = S[j];
-                        S[j] = So[j];
-                        So[j] = t;
-                    }
-                    const float t = dp;
-                    dp = dpo;
-                    dpo = t;
                 }
             }
-            if (!kSum && !kGenOut && c >= nh && c % nh == 0) {
-                // outputs of the real chunk whose last key half is c-1
-                const int co = c - 1, ob = (co / nh) & 1;
-                const bool fail = !mbar_wait(&bars[BAR_OFULL + (co & 1)], (co >> 1) & 1, abort_flag, kWaitLimitNs);
-                if (__any_sync(0xffffffffu, fail)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                uint32_t ow[16];  // the row's 32 outputs packed in pairs
+            if (kBal && piece == 0 && b_chi > 0 && ok) {
+                // the state at the end of the head run -> the next CTA
+                float4 *dst = reinterpret_cast<float4 *>(p.summary + (size_t)blockIdx.x * kD * kD + (size_t)row * kD + ch0);
 #pragma unroll
-                for (int hf = 0; hf < 2; ++hf) {
-                    uint32_t r[16];
-                    tmem_ld_16x32bx2_x16(tmem + lane_base + kColO + ob * 64 + 16 * hf, r);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) ow[8 * hf + j] = Elem<E>::pack(__uint_as_float(r[2 * j]), __uint_as_float(r[2 * j + 1]));
-                }
-                tc_fence_before();
-                const StreamPos po = pos(co);
-                const int b = po.bh / p.H, h = po.bh % p.H;
-                const int t = walk_token(p.order, p.T, p.grid_h, p.grid_w, chunk_w0(p.order, p.T, po.c) + row);
-                if (t >= 0) {  // the row's columns inside Dv (padded columns stay behind)
-                    const int col0 = 64 * po.vb + ch0;
-                    uint4 *dst = reinterpret_cast<uint4 *>(out + (((size_t)b * p.T + t) * p.H + h) * p.Dv + col0);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        if (col0 + 8 * q < p.Dv) dst[q] = make_uint4(ow[4 * q], ow[4 * q + 1], ow[4 * q + 2], ow[4 * q + 3]);
-                }
+                for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
+                __threadfence();
+                named_barrier_sync(3, 128);  // the epi's four warps wrote their rows
+                if (threadIdx.x == 10 * 32)
+                    *reinterpret_cast<volatile unsigned long long *>(p.flags + blockIdx.x) = p.epoch;
             }
         }
         if (!ok) record_timeout(abort_flag);
@@ -1633,20 +1684,20 @@ Split choose_split(const Problem &p, int n_sm) {
 }
 
 // Balanced ranges (one key half, unsplit): when the units are more than the SMs and a
-// round-robin deal would take at least 1.25 times the chunks per CTA of an even split,
+// round-robin deal would take at least 1.1 times the chunks per CTA of an even split,
 // every CTA takes an equal contiguous range of chunks instead.  Measured on a GB300
-// (graph-replayed, interleaved): B = 16, H = 12, 80 x 80, bf16 (192 units, ratio 1.58)
-// ran 1.23x faster balanced; B = 32, H = 12, 40 x 40 (384 units, ratio 1.19) 0.93x in
-// bf16 and 0.98x in fp16.  Contiguous ranges put every CTA at its own sequence and chunk,
-// so neighbouring CTAs no longer read the same token rows together: the loads then
-// stream at about 4.3 TB/s instead of 6.4 (copy-only probe of the same pattern).
+// (graph-replayed, interleaved, against whole units): B = 32, H = 12, 40 x 40 (384 units,
+// ratio 1.19) 1.10x in bf16 and 1.05x in fp16; B = 16, H = 12, 80 x 80 (192 units, ratio
+// 1.58) 1.52x; B = 24 (288 units, ratio 1.06) 0.98x and B = 38 (456 units, ratio 1.00)
+// 0.96x, hence the threshold.  The balanced kernel costs about 6 % a chunk more than the
+// round-robin one (the hand-offs and the longer decode).
 bool choose_balanced(const Problem &p, int n_sm) {
-    if (pad64(p.Dk) != 64) return false;
+    if (pad64(p.Dk) != 64 || n_sm < 1) return false;
     const long long units = (long long)p.B * p.H * (pad64(p.Dv) / 64);
     if (units <= n_sm) return false;
     if (units * ((p.T + kC - 1) / kC) > 0x7fffffffLL) return false;  // the decode's flattened chunk index is an int
     const long long waves = (units + n_sm - 1) / n_sm;
-    return waves * n_sm * 4 >= units * 5;  // ceil(U / SMs) >= 1.25 U / SMs
+    return waves * n_sm * 10 >= units * 11;  // ceil(U / SMs) >= 1.1 U / SMs
 }
 
 // hand-off states ([64][64] fp32 per CTA) and flags (one 64-bit word per CTA)
@@ -1663,7 +1714,7 @@ size_t summary_bytes(const Problem &p, int nseg) {
 
 int tc_chunk_boxes(int order, int T, int grid_h, int grid_w, int c, int *boxes, int cap) {
     int n = 0;
-    chunk_load_boxes(order, T, grid_h, grid_w, c, [&](int hi, int row, int c2, int c3) {
+    chunk_load_boxes(order, T, make_fastdiv(grid_h), grid_w, c, [&](int hi, int row, int c2, int c3) {
         if (n < cap) {
             boxes[4 * n + 0] = box_height(hi);
             boxes[4 * n + 1] = row;
@@ -1676,7 +1727,7 @@ int tc_chunk_boxes(int order, int T, int grid_h, int grid_w, int c, int *boxes, 
 }
 
 int tc_chunk_walk(int order, int T, int grid_h, int c, int *x0, int *y0) {
-    return chunk_walk_start(order, T, grid_h, c, x0, y0) ? 1 : 0;
+    return chunk_walk_start(order, T, make_fastdiv(grid_h), c, x0, y0) ? 1 : 0;
 }
 
 void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len) {
@@ -1715,6 +1766,8 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     tp.final_state = p.final_state;
     tp.H = p.H;
     tp.grid_h = p.grid_h;
+    tp.fd_H = make_fastdiv(p.H);
+    tp.fd_gh = make_fastdiv(p.grid_h);
     tp.grid_w = p.grid_w;
     tp.order = p.order;
     tp.T = static_cast<int>(p.T);
@@ -1725,7 +1778,8 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     tp.nv = pad64(p.Dv) / 64;
     Split sp = choose_split(p, n_sm);
     Ran r;
-    r.planned = sp.nseg > 1 ? kRanTcSplit : (choose_balanced(p, n_sm) ? kRanTcBalanced : kRanTc);
+    const bool bal = choose_balanced(p, n_sm);
+    r.planned = sp.nseg > 1 ? kRanTcSplit : (bal ? kRanTcBalanced : kRanTc);
     r.ran = kRanTc;
     if (sp.nseg > 1 && (workspace == nullptr || workspace_bytes < summary_bytes(p, sp.nseg)))
         sp = Split{1, tp.n_chunks};
@@ -1733,6 +1787,8 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     const int nseg = sp.nseg;
     tp.nseg = nseg;
     tp.seg_len = sp.len;
+    tp.fd_L = make_fastdiv(sp.len);
+    tp.fd_per = make_fastdiv(sp.len * tp.nh);
     tp.summary = static_cast<float *>(workspace);
     tp.flags = nullptr;
     tp.epoch = 0;
@@ -1745,6 +1801,7 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
     unsigned sum_ctas = 0;
     if (nseg > 1) {  // pass 1: end state from zero and total decay of segments 0 .. nseg-2
         tp.nsu = nseg - 1;
+        tp.fd_nsu = make_fastdiv(tp.nsu);
         tp.n_units = seqs * tp.nsu;
         const dim3 grid(static_cast<unsigned>(tp.n_units < n_sm ? tp.n_units : n_sm));
         sum_ctas = grid.x;
@@ -1753,13 +1810,15 @@ cudaError_t launch_tc(const Problem &p, cudaStream_t stream, void *workspace, si
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     tp.nsu = nseg;
+    tp.fd_nsu = make_fastdiv(nseg);
     tp.n_units = seqs * nseg;
-    if (nseg == 1 && choose_balanced(p, n_sm) && workspace != nullptr && workspace_bytes >= handoff_bytes(n_sm)) {
+    if (nseg == 1 && bal && workspace != nullptr && workspace_bytes >= handoff_bytes(n_sm)) {
         // equal contiguous chunk ranges, one CTA per SM
         r.ran = kRanTcBalanced;
         if (ran) *ran = r;
         tp.flags = reinterpret_cast<unsigned long long *>(static_cast<char *>(workspace) + (size_t)n_sm * 64 * 64 * sizeof(float));
         tp.epoch = next_epoch();
+        tp.bal_n = make_fastdiv(tp.n_chunks);
         const dim3 bgrid(static_cast<unsigned>(n_sm));
         if (half)
             e = tp.nv == 1 ? launch_balanced<__half, 1>(bgrid, tp, stream) : launch_balanced<__half, 2>(bgrid, tp, stream);
@@ -1846,6 +1905,8 @@ cudaError_t launch_tc_gate(const Problem &p, const GateSource &gs, cudaStream_t 
     tp.final_state = p.final_state;
     tp.H = p.H;
     tp.grid_h = p.grid_h;
+    tp.fd_H = make_fastdiv(p.H);
+    tp.fd_gh = make_fastdiv(p.grid_h);
     tp.grid_w = p.grid_w;
     tp.order = p.order;
     tp.T = static_cast<int>(p.T);
@@ -1857,6 +1918,9 @@ cudaError_t launch_tc_gate(const Problem &p, const GateSource &gs, cudaStream_t 
     tp.nseg = 1;
     tp.nsu = 1;
     tp.seg_len = tp.n_chunks;
+    tp.fd_nsu = make_fastdiv(1);
+    tp.fd_L = make_fastdiv(tp.n_chunks);
+    tp.fd_per = make_fastdiv(tp.n_chunks);
     const char *drop = std::getenv("GTR_GLA_TEST_DROP_LOAD");
     tp.drop_load = (drop != nullptr && drop[0] == '1') ? 1 : 0;
     tp.n_units = static_cast<int>(p.B * p.H) * tp.nv;

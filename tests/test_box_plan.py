@@ -10,6 +10,8 @@ walk instead (gtr_gla_chunk_walk): its start and traversal give the same rows.
 No GPU is used."""
 import math
 
+import numpy as np
+
 import pytest
 
 from paper_2609_26590_gb300 import build as gbuild
@@ -123,6 +125,28 @@ def test_walk_loads(gla, order):
                 for i in range(nrows):
                     rows[r0 + i] = (c2, c3 + i)
             assert [rows[r] for r in range(C)] == pixels, (gh, gw, order, c)
+
+
+def test_walk_start_division_large_grids(gla):
+    # the walk start is the grid position (w0 // grid_h, w0 % grid_h), computed with a
+    # multiply-high division by grid_h (Granlund-Montgomery): checked here for many divisors,
+    # powers of two and their neighbours, and walk positions up to the largest sequences
+    rng = np.random.default_rng(31)
+    divisors = [1, 2, 3, 5, 7, 63, 64, 65, 127, 128, 129, 255, 256, 257, 1000, 4095, 4096, 4097,
+                32767, 32768, 32769, 65535, 65536, 65537, 1 << 20, (1 << 20) + 1, (1 << 24) - 1]
+    divisors += [int(d) for d in rng.integers(1, 1 << 20, size=60)]
+    for gh in divisors:
+        gw = max(1, (1 << 30) // gh)
+        T = gh * gw
+        N = T // C
+        cs = {0, 1, N - 1, N // 2} | {int(c) for c in rng.integers(0, N, size=40)}
+        for c in sorted(cs):
+            w0 = C * c
+            if w0 + C > T:
+                continue
+            assert gla.chunk_walk(gh, gw, wl.COL_FWD, c) == (w0 // gh, w0 % gh), (gh, gw, c)
+            wr = T - C * (c + 1)
+            assert gla.chunk_walk(gh, gw, wl.COL_REV, c) == (wr // gh, wr % gh), (gh, gw, c)
 
 
 def test_padding_chunks_load_only_zeros(gla):
