@@ -47,7 +47,7 @@ void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len);
 // flags when it balances chunk ranges (tc_balanced_plan), else 0.
 size_t tc_workspace_bytes(const Problem &p);
 // 1 when the tensor-core schedule gives every CTA an equal contiguous range of chunks
-// (more units than SMs, a round-robin deal at least 1.25 times an even split's share) on a device
+// (more units than SMs, a round-robin deal at least 1.1 times an even split's share) on a device
 // with n_sm SMs; its workspace then holds one hand-off state and flag per SM.
 int tc_balanced_plan(const Problem &p, int n_sm);
 // Which schedule a launch ran, and which one it would have run with enough workspace
