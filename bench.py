@@ -747,10 +747,13 @@ def main():
 
     res = time_mixer(args, w, rank, world, local, dev, pg)
     head = {k: res[k] for k in ("value", "ms_per_step", "roofline", "clocks", "launches")}
-    e2e = time_e2e(args, res, world, dev, pg) if args.e2e_steps > 0 and not args.gated else None
+    # the host-buffer entry point runs the plain mixer: no end-to-end leg for the gated and
+    # gate-producer variants, and the oracle baseline times the plain mixer's inputs
+    e2e = (time_e2e(args, res, world, dev, pg)
+           if args.e2e_steps > 0 and not args.gated and not args.gate_producer else None)
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.gate_producer:
         inp64 = {n: wl.storage_to_f64(res["inp"][n], w.dtype) for n in ("q", "k", "v", "g")}
         val, el, n_pairs, cores = time_oracle(w, inp64, w.orders[0], budget_s=10.0)
         cpu = {"value": val, "unit": "tokens/s", "cores": cores, "kind": "oracle",
