@@ -355,15 +355,16 @@ __device__ __forceinline__ StreamPos stream_pos_bal(int v, int N, int lognv, int
     return {unit >> lognv, unit & ((1 << lognv) - 1), c, 0, 0, c, c == 0 || hin, hin, v == c_hi - 1};
 }
 
-// kBalanced: bounded wait for the previous CTA's hand-off flag.  Out of line: it runs once
-// per CTA, and inlined into the epi's loop it enlarged the kernel's hot code.
-__device__ __noinline__ bool handoff_wait(const volatile unsigned long long *f, unsigned long long epoch,
+// kBalanced: bounded wait for the previous CTA's hand-off flag, read with acquire semantics at
+// GPU scope (the writer fenced before setting it), so the waiting thread needs no fence of its
+// own, which would also wait for its output stores in flight.  Out of line: it runs once per CTA.
+__device__ __noinline__ bool handoff_wait(const unsigned long long *f, unsigned long long epoch,
                                           volatile uint32_t *abort_flag) {
-    bool got = *f == epoch;
+    bool got = ld_acquire_u64(f) == epoch;
     const uint64_t t0 = global_timer_ns();
     while (!got && !*abort_flag && global_timer_ns() - t0 < kWaitLimitNs) {
         __nanosleep(64);
-        got = *f == epoch;
+        got = ld_acquire_u64(f) == epoch;
     }
     return got;
 }
@@ -1209,15 +1210,19 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
 #pragma unroll 1
         for (int piece = 0; ok && piece < (kBal ? 3 : 1); ++piece) {
             if (kBal && piece == 2 && b_t0 < G) {
-                // the tail run starts from the previous CTA's hand-off (a bounded wait on its
-                // flag, which is then cleared for the next launch)
-                const volatile unsigned long long *f = p.flags + blockIdx.x - 1;
-                const bool got = handoff_wait(f, p.epoch, abort_flag);
+                // the tail run starts from the previous CTA's hand-off: one thread waits for its
+                // flag (bounded) and clears it for the next launch; the barrier orders the other
+                // threads' reads after its acquire
+                unsigned long long *f = p.flags + blockIdx.x - 1;
+                bool got = true;
+                if (threadIdx.x == 10 * 32) {
+                    got = handoff_wait(f, p.epoch, abort_flag);
+                    if (got) *reinterpret_cast<volatile unsigned long long *>(f) = 0ull;
+                }
                 if (named_barrier_or(3, 128, !got)) {  // the epi gives up together
                     ok = false;
                     break;
                 }
-                __threadfence();
                 const float4 *x = reinterpret_cast<const float4 *>(p.summary + (size_t)(blockIdx.x - 1) * kD * kD +
                                                                    (size_t)row * kD + ch0);
 #pragma unroll
@@ -1228,8 +1233,6 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     S[4 * j + 2] = w.z;
                     S[4 * j + 3] = w.w;
                 }
-                named_barrier_sync(3, 128);  // the epi's four warps read their rows
-                if (threadIdx.x == 10 * 32) *const_cast<volatile unsigned long long *>(f) = 0ull;
             }
             const int c_end = piece == 0 ? cut0 : (piece == 1 ? cut1 : G + 1);
             for (; ok && c < c_end; ++c) {
@@ -1373,10 +1376,13 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                 float4 *dst = reinterpret_cast<float4 *>(p.summary + (size_t)blockIdx.x * kD * kD + (size_t)row * kD + ch0);
 #pragma unroll
                 for (int j = 0; j < 8; ++j) dst[j] = make_float4(S[4 * j], S[4 * j + 1], S[4 * j + 2], S[4 * j + 3]);
-                __threadfence();
-                named_barrier_sync(3, 128);  // the epi's four warps wrote their rows
-                if (threadIdx.x == 10 * 32)
+                // the epi's four warps wrote their rows; one thread fences (for them all, after the
+                // barrier) and sets the flag, so only its warp waits for its stores in flight
+                named_barrier_sync(3, 128);
+                if (threadIdx.x == 10 * 32) {
+                    __threadfence();
                     *reinterpret_cast<volatile unsigned long long *>(p.flags + blockIdx.x) = p.epoch;
+                }
             }
         }
         if (!ok) record_timeout(abort_flag);
