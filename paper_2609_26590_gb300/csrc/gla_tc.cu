@@ -302,7 +302,6 @@ struct StreamPos {
     int cl;      // chunk within the segment
     bool start;  // a run of the unit starts here: its state is set
     bool hin;    // kBalanced: the run starts from the previous CTA's hand-off state
-    bool hout;   // kBalanced: after this chunk the state goes to the next CTA
 };
 // Units are (sequence, segment, value slice), the value slice fastest (the two
 // slices of a sequence read the same q, k and gates); a unit covers seg_len chunks.
@@ -315,7 +314,7 @@ __device__ __forceinline__ StreamPos stream_pos(int v, int L, int nh, int lognv,
     const int seg = split ? rest - bh * nsu.d : 0;
     const int cl = rem / nh;
     const int a = rem - cl * nh;
-    return {bh, unit & ((1 << lognv) - 1), seg * L + cl, a, seg, cl, cl == 0 && a == 0, false, false};
+    return {bh, unit & ((1 << lognv) - 1), seg * L + cl, a, seg, cl, cl == 0 && a == 0, false};
 }
 
 // kBalanced: the units' chunks in order, unit by unit, cut into gridDim.x equal contiguous
@@ -352,7 +351,7 @@ __device__ __forceinline__ StreamPos stream_pos_bal(int v, int N, int lognv, int
     const int g = v + (v < c_hi ? base_head : (v < t0 ? base_full : base_tail));
     const int unit = fdiv(g, fn), c = g - unit * N;
     const bool hin = v == t0;  // the tail's first chunk (t0 == G when there is no tail)
-    return {unit >> lognv, unit & ((1 << lognv) - 1), c, 0, 0, c, c == 0 || hin, hin, v == c_hi - 1};
+    return {unit >> lognv, unit & ((1 << lognv) - 1), c, 0, 0, c, c == 0 || hin, hin};
 }
 
 // kBalanced: bounded wait for the previous CTA's hand-off flag, read with acquire semantics at
