@@ -157,6 +157,21 @@ gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, in
  * before it handed over through the workspace.  Host arithmetic only. */
 int gtr_gla_balanced_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm);
 
+/* The chunks one CTA of the balanced schedule processes, in its order, computed on
+ * the host by the kernel's own decode (no device is used).  n_units (sequence,
+ * value slice) units of n_chunks 64-token chunks each, in unit order, are cut into
+ * `grid` equal contiguous ranges (1 <= grid <= n_units, so a range is at least one
+ * unit long).  CTA `cta` (0 <= cta < grid) first runs the head of the unit its
+ * range ends in (chunks 0 .. *head - 1, from a zero state; the state after them is
+ * handed to CTA cta + 1), then its whole units, then the tail of the unit its range
+ * starts in, from the state CTA cta - 1 handed over (Eq. chunk_boundary_main across
+ * CTAs).  Writes min(count, cap) entries of 4 ints: unit, chunk, start (1 where a
+ * unit's state is set: chunk 0, or the tail's first chunk) and hand-in (1 at the
+ * tail's first chunk); *head receives the head run's length.  Returns the CTA's
+ * chunk count, or -1 for invalid arguments (entries may be NULL when cap is 0;
+ * head must not be NULL). */
+int gtr_gla_balanced_walk(int n_units, int n_chunks, int grid, int cta, int *entries, int cap, int *head);
+
 /* Introspection of the scan-order gather (Sec. 3.1, directional scanning): the
  * TMA boxes of 64-token chunk c of a sequence on a grid_h x grid_w patch grid,
  * computed on the host by the same code the kernel's producer runs.  The

@@ -243,6 +243,12 @@ int gtr_gla_chunk_walk(int grid_h, int grid_w, gtr_scan_t scan_order, int c, int
     return gtr::tc_chunk_walk(scan_order, static_cast<int>(T), grid_h, c, x, y);
 }
 
+int gtr_gla_balanced_walk(int n_units, int n_chunks, int grid, int cta, int *entries, int cap, int *head) {
+    if (n_units < 1 || n_chunks < 1 || grid < 1 || grid > n_units || cta < 0 || cta >= grid) return -1;
+    if ((long long)n_units * n_chunks > 0x7fffffffLL || cap < 0 || (cap > 0 && entries == nullptr) || !head) return -1;
+    return gtr::tc_balanced_walk(n_units, n_chunks, grid, cta, entries, cap, head);
+}
+
 gtr_status_t gtr_gla_split_plan(int B, int H, int grid_h, int grid_w, int Dk, int Dv, int n_sm, int *nseg,
                                 int *seg_len) {
     if (!nseg || !seg_len || n_sm < 1) return GTR_ERR_INVALID_ARG;

@@ -39,6 +39,9 @@ bool tc_supported(const Problem &p);
 // coordinate 2, coordinate 3); returns how many the chunk has.
 int tc_chunk_boxes(int order, int T, int grid_h, int grid_w, int c, int *boxes, int cap);
 int tc_chunk_walk(int order, int T, int grid_h, int c, int *x0, int *y0);
+// The balanced schedule's walk of CTA cta of grid over n_units units of N chunks: entries of
+// (unit, chunk, start, hand-in), *head = the head run's length; returns the chunk count.
+int tc_balanced_walk(int n_units, int N, int grid, int cta, int *entries, int cap, int *head);
 // Segments per sequence and chunks per segment the tensor-core schedule uses for
 // this problem on a device with n_sm SMs (host arithmetic only; nseg 1: unsplit).
 void tc_split_plan(const Problem &p, int n_sm, int *nseg, int *seg_len);

@@ -317,9 +317,9 @@ __device__ __forceinline__ StreamPos stream_pos(int v, int L, int nh, int lognv,
     return {bh, unit & ((1 << lognv) - 1), seg * L + cl, a, seg, cl, cl == 0 && a == 0, false};
 }
 
-// kBalanced: the units' chunks in order, unit by unit, cut into gridDim.x equal contiguous
+// kBalanced: the units' chunks in order, unit by unit, cut into `grid` equal contiguous
 // ranges (each at least one unit long, so no range lies inside one unit), decoded once per
-// CTA.  A CTA first runs the head [0, c_hi) of the unit its range ends in (from zero; its
+// CTA (`cta`; the host runs the same code for gtr_gla_balanced_walk).  A CTA first runs the head [0, c_hi) of the unit its range ends in (from zero; its
 // end state goes to the next CTA), then its whole units, then the tail [c_lo, N) of the
 // unit its range starts in, from the state the previous CTA handed over at the start of
 // its own run (long before).
@@ -328,9 +328,9 @@ struct BalRange {
     int c_hi, t0;                         // pieces: [0, c_hi) head, [c_hi, t0) whole units, [t0, G) tail
     int G;
 };
-__device__ __forceinline__ BalRange bal_range(int N, int n_units) {
+__host__ __device__ __forceinline__ BalRange bal_range(int N, int n_units, int cta, int grid) {
     const long long tot = static_cast<long long>(n_units) * N;
-    const long long lo = tot * blockIdx.x / gridDim.x, hi = tot * (blockIdx.x + 1) / gridDim.x;
+    const long long lo = tot * cta / grid, hi = tot * (cta + 1) / grid;
     const int u_lo = static_cast<int>(lo / N), c_lo = static_cast<int>(lo - static_cast<long long>(u_lo) * N);
     const int u_hi = static_cast<int>(hi / N), c_hi = static_cast<int>(hi - static_cast<long long>(u_hi) * N);
     const int u_first = c_lo ? u_lo + 1 : u_lo;
@@ -346,8 +346,8 @@ __device__ __forceinline__ BalRange bal_range(int N, int n_units) {
 // The piece is picked by two compares and the unit by one multiply-high division; a
 // three-way branch over the pieces made every role's per-chunk decode slower and cost the
 // whole kernel 10 %, and an integer division here another 17 %.
-__device__ __forceinline__ StreamPos stream_pos_bal(int v, int N, int lognv, int base_head, int base_full,
-                                                    int base_tail, int c_hi, int t0, const FastDiv &fn) {
+__host__ __device__ __forceinline__ StreamPos stream_pos_bal(int v, int N, int lognv, int base_head, int base_full,
+                                                             int base_tail, int c_hi, int t0, const FastDiv &fn) {
     const int g = v + (v < c_hi ? base_head : (v < t0 ? base_full : base_tail));
     const int unit = fdiv(g, fn), c = g - unit * N;
     const bool hin = v == t0;  // the tail's first chunk (t0 == G when there is no tail)
@@ -605,7 +605,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
     // buffer below follows the stream index (O: the real chunk's index), so
     // consecutive units flow through one pipeline
     BalRange br{};
-    if constexpr (kBal) br = bal_range(N, p.n_units);
+    if constexpr (kBal) br = bal_range(N, p.n_units, static_cast<int>(blockIdx.x), static_cast<int>(gridDim.x));
     const int b_head = br.base_head, b_full = br.base_full, b_tail = br.base_tail, b_chi = br.c_hi, b_t0 = br.t0;
     const int G = kBal ? br.G
                        : L * nh *
@@ -1733,6 +1733,20 @@ int tc_chunk_boxes(int order, int T, int grid_h, int grid_w, int c, int *boxes, 
         ++n;
     });
     return n;
+}
+
+int tc_balanced_walk(int n_units, int N, int grid, int cta, int *entries, int cap, int *head) {
+    const BalRange r = bal_range(N, n_units, cta, grid);
+    const FastDiv fn = make_fastdiv(N);
+    for (int v = 0; v < r.G && v < cap; ++v) {
+        const StreamPos ps = stream_pos_bal(v, N, 0, r.base_head, r.base_full, r.base_tail, r.c_hi, r.t0, fn);
+        entries[4 * v + 0] = ps.bh;  // with one value slice per unit, the unit itself
+        entries[4 * v + 1] = ps.c;
+        entries[4 * v + 2] = ps.start ? 1 : 0;
+        entries[4 * v + 3] = ps.hin ? 1 : 0;
+    }
+    *head = r.c_hi;
+    return r.G;
 }
 
 int tc_chunk_walk(int order, int T, int grid_h, int c, int *x0, int *y0) {

@@ -61,6 +61,8 @@ def load(path: Optional[str] = None):
         lib.gtr_gla_chunk_boxes.argtypes = [ci] * 4 + [ctypes.POINTER(ci), ci]
         lib.gtr_gla_chunk_walk.restype = ci
         lib.gtr_gla_chunk_walk.argtypes = [ci] * 4 + [ctypes.POINTER(ci)] * 2
+        lib.gtr_gla_balanced_walk.restype = ci
+        lib.gtr_gla_balanced_walk.argtypes = [ci] * 4 + [ctypes.POINTER(ci), ci, ctypes.POINTER(ci)]
         lib.gtr_gla_split_plan.restype = ci
         lib.gtr_gla_split_plan.argtypes = [ci] * 7 + [ctypes.POINTER(ci)] * 2
         lib.gtr_gla_balanced_plan.restype = ci
@@ -234,6 +236,20 @@ def chunk_walk(grid_h: int, grid_w: int, order: int, c: int):
     if r < 0:
         raise ValueError(f"gtr_gla_chunk_walk returned {r}")
     return (x.value, y.value) if r == 1 else None
+
+
+def balanced_walk(n_units: int, n_chunks: int, grid: int, cta: int):
+    """(entries, head) of CTA ``cta`` of the balanced schedule, through
+    ``gtr_gla_balanced_walk`` (host only): entries are (unit, chunk, start, hand_in)
+    tuples in the CTA's order, head the length of its head run."""
+    lib = load()
+    head = ctypes.c_int(-1)
+    n = lib.gtr_gla_balanced_walk(n_units, n_chunks, grid, cta, None, 0, ctypes.byref(head))
+    if n < 0:
+        raise ValueError(f"gtr_gla_balanced_walk returned {n}")
+    buf = (ctypes.c_int * (4 * max(n, 1)))()
+    lib.gtr_gla_balanced_walk(n_units, n_chunks, grid, cta, buf, n, ctypes.byref(head))
+    return [tuple(buf[4 * i:4 * i + 4]) for i in range(n)], head.value
 
 
 def forward_ws(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, log_gate: torch.Tensor,
