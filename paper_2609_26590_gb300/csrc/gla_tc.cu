@@ -1206,22 +1206,23 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
         // (in the loop it slowed every chunk: the SM's instruction cache is shared by all roles)
         const int cut0 = kBal ? b_chi : G + 1, cut1 = kBal ? b_t0 : G + 1;
         int c = 0;
+        // Every epi warp passes the pieces' boundaries, also one that gave up (its warps decide on
+        // their own inside the loop): the hand-offs' named barriers then always see all four.
 #pragma unroll 1
-        for (int piece = 0; ok && piece < (kBal ? 3 : 1); ++piece) {
+        for (int piece = 0; piece < (kBal ? 3 : 1); ++piece) {
             if (kBal && piece == 2 && b_t0 < G) {
                 // the tail run starts from the previous CTA's hand-off: one thread waits for its
                 // flag (bounded) and clears it for the next launch; the barrier orders the other
                 // threads' reads after its acquire
                 unsigned long long *f = p.flags + blockIdx.x - 1;
                 bool got = true;
-                if (threadIdx.x == 10 * 32) {
+                if (ok && threadIdx.x == 10 * 32) {
                     got = handoff_wait(f, p.epoch, abort_flag);
                     if (got) *reinterpret_cast<volatile unsigned long long *>(f) = 0ull;
                 }
-                if (named_barrier_or(3, 128, !got)) {  // the epi gives up together
-                    ok = false;
-                    break;
-                }
+                if (named_barrier_or(3, 128, !ok || !got)) ok = false;  // the epi gives up together
+            }
+            if (kBal && piece == 2 && b_t0 < G && ok) {
                 const float4 *x = reinterpret_cast<const float4 *>(p.summary + (size_t)(blockIdx.x - 1) * kD * kD +
                                                                    (size_t)row * kD + ch0);
 #pragma unroll
@@ -1370,6 +1371,7 @@ __global__ void __launch_bounds__(kThreads, 1) gla_tc_kernel(const __grid_consta
                     }
                 }
             }
+            if (kBal && piece == 0 && b_chi > 0 && named_barrier_or(3, 128, !ok)) ok = false;
             if (kBal && piece == 0 && b_chi > 0 && ok) {
                 // the state at the end of the head run -> the next CTA
                 float4 *dst = reinterpret_cast<float4 *>(p.summary + (size_t)blockIdx.x * kD * kD + (size_t)row * kD + ch0);
