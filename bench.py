@@ -533,9 +533,17 @@ def time_mixer(args, w: wl.Workload, rank: int, world: int, local: int, dev, pg)
     split = not args.gate_producer and ws_n > 0 and gla.split_plan(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv,
                                          torch.cuda.get_device_properties(dev).multi_processor_count)[0] > 1
     launches_per_step = 2 if split else 1
+    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
     if split:
         kernel_name += ", segment-summary pass + output pass"
-    if args.gated:  # the output gate runs as one more kernel right after the mixer
+    elif ws_n > 0 and not args.gate_producer and gla.balanced_plan(w.B, w.H, w.grid_h, w.grid_w, w.Dk, w.Dv, n_sm):
+        kernel_name += ", balanced ranges (one CTA per SM, state hand-offs between them)"
+    # the library fuses the output gate into the tensor-core kernel's stores for one key half and one
+    # value slice when the sequences fill at most half of the SMs; otherwise it is one more kernel
+    gate_fused = tc and schedule != "simt" and w.Dk <= 64 and w.Dv <= 64 and 2 * w.B * w.H <= n_sm
+    if args.gated and gate_fused:
+        kernel_name += ", output gate fused into the output stores"
+    elif args.gated:
         launches_per_step += 1
         kernel_name += " + output-gate kernel"
     if args.gate_producer:
